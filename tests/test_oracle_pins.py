@@ -1,0 +1,433 @@
+"""Pins of the oracle against facts that do not come from the oracle itself.
+
+Each function of ``oracle`` is checked against at least one of: values printed
+in the paper (Boxes 4-6, arXiv 2608.22646), values worked out by hand from the
+printed formulas (``tests/golden``), closed forms, high-precision brute force
+(mpmath) on tiny inputs, invariants, and hand-worked controller trajectories
+that exercise every branch of Algorithm 1.
+
+Coverage map (function -> pins):
+  cai_o_bf16_to_double     -> exact bit patterns (test_bf16_decode)
+  cai_o_head_rows          -> mpmath brute force, V=2 closed form, uniform,
+                              one-hot gap closed form, ties, sum-to-one,
+                              c = exp(m - LSE), transposed-operand catch
+  cai_o_theta_e            -> Box 4 printed values, floor, quarter mode
+  cai_o_theta_block        -> hand-worked golden table, endpoints, monotone
+  cai_o_pos_factor         -> Box 6 printed tiers, quarter mode
+  cai_o_theta_token        -> clip bounds
+  cai_o_budget             -> Box 5 hand table, boundaries
+  cai_o_low_yield          -> count and fraction readings
+  cai_o_controller_step    -> hand trajectories G1, G2, budget force,
+                              DONE, T-exhausted, flush, gating OFF, and
+                              invariants over synthetic trajectories
+"""
+import math
+import os
+
+import mpmath
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+
+GOLDEN = os.path.join(os.path.dirname(__file__), "golden")
+
+
+def _rows(name):
+    out = []
+    with open(os.path.join(GOLDEN, name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                out.append(line.split())
+    return out
+
+
+def bf16_from_float(x):
+    """Round-to-nearest-even float32 -> bf16 bits (test-side helper)."""
+    a = np.asarray(x, np.float32).reshape(-1)
+    u = a.view(np.uint32).astype(np.uint64)
+    r = ((u + 0x7FFF + ((u >> 16) & 1)) >> 16).astype(np.uint16)
+    return r.reshape(np.shape(x))
+
+
+# ------------------------------------------------------------------ bf16 --
+
+def test_bf16_decode():
+    lib = oracle.lib()
+    assert lib.cai_o_bf16_to_double(0x3F80) == 1.0
+    assert lib.cai_o_bf16_to_double(0xC000) == -2.0
+    assert lib.cai_o_bf16_to_double(0x3F81) == 1.0 + 2.0 ** -7
+    assert lib.cai_o_bf16_to_double(0x0001) == 2.0 ** -133          # smallest subnormal
+    assert lib.cai_o_bf16_to_double(0x8000) == 0.0
+    assert math.isinf(lib.cai_o_bf16_to_double(0x7F80))
+    assert lib.cai_o_bf16_to_double(0x4049) == 3.140625
+
+
+# ------------------------------------------------------------------ head --
+
+def _brute(Wf, hf):
+    """mpmath (60 digits) logits, softmax, confidence, lowest-index argmax."""
+    mpmath.mp.dps = 60
+    V, H = Wf.shape
+    z = [mpmath.fsum(mpmath.mpf(float(Wf[v, k])) * mpmath.mpf(float(hf[k])) for k in range(H))
+         for v in range(V)]
+    m = max(z)
+    idx = min(v for v in range(V) if z[v] == m)
+    S = mpmath.fsum(mpmath.e ** (zv - m) for zv in z)
+    return [float(zv) for zv in z], float(1 / S), idx, float(m + mpmath.log(S))
+
+
+@pytest.mark.parametrize("seed", range(12))
+def test_head_bruteforce_tiny(seed):
+    rng = np.random.default_rng(seed)
+    V = int(rng.integers(2, 9))
+    H = int(rng.integers(1, 5))
+    Wf = rng.normal(0, 1.5, (V, H)).astype(np.float32)
+    hf = rng.normal(0, 1.5, (H,)).astype(np.float32)
+    Wb, hb = bf16_from_float(Wf), bf16_from_float(hf)
+    Wd = Wb.astype(np.uint32) << 16
+    hd = hb.astype(np.uint32) << 16
+    Wq = Wd.view(np.float32).reshape(V, H)
+    hq = hd.view(np.float32)
+    z_ref, c_ref, idx_ref, lse_ref = _brute(Wq, hq)
+    out = oracle.head_rows(Wb, hb.reshape(1, H))
+    assert out["idx"][0] == idx_ref
+    assert abs(out["conf"][0] - c_ref) < 1e-13
+    assert abs(out["lse"][0] - lse_ref) < 1e-12
+    z, p, idx = oracle.softmax_row(Wb, hb)
+    np.testing.assert_allclose(z, z_ref, rtol=0, atol=1e-12)
+    assert abs(p.sum() - 1.0) < 1e-12
+    assert idx == idx_ref
+
+
+def test_head_transposed_operand_is_caught():
+    # W is deliberately non-square and asymmetric: z = W h differs from any
+    # use of W's columns.  h picks column 1 only, so z_v = W[v, 1].
+    W = np.array([[1, 2, 0], [3, -4, 0], [0, 8, 1], [5, 6, 7]], np.float32)
+    h = np.array([0, 1, 0], np.float32)
+    out = oracle.head_rows(bf16_from_float(W), bf16_from_float(h).reshape(1, 3))
+    assert out["idx"][0] == 2          # max of column 1 = 8 at row 2
+    assert abs(out["zmax"][0] - 8.0) < 1e-15
+    assert abs(out["gap"][0] - 2.0) < 1e-15   # 8 - 6
+
+
+@pytest.mark.parametrize("delta", [0.0, 0.3, 1.0, 4.0, 9.5])
+def test_head_two_way_closed_form(delta):
+    # V = 2: c = sigma(|z1 - z2|).
+    W = np.array([[1.0], [0.0]], np.float32)
+    h = np.array([delta], np.float32)
+    Wb, hb = bf16_from_float(W), bf16_from_float(h)
+    d = float((hb.astype(np.uint32) << 16).view(np.float32)[0])
+    out = oracle.head_rows(Wb, hb.reshape(1, 1))
+    assert abs(out["conf"][0] - 1.0 / (1.0 + math.exp(-abs(d)))) < 1e-15
+    assert out["idx"][0] == 0
+
+
+@pytest.mark.parametrize("V", [3, 17, 1000])
+def test_head_uniform_and_ties(V):
+    # All logits equal: c = 1/V and the argmax is the lowest index.
+    W = np.ones((V, 4), np.float32)
+    h = np.full((4,), 0.5, np.float32)
+    out = oracle.head_rows(bf16_from_float(W), bf16_from_float(h).reshape(1, 4))
+    assert abs(out["conf"][0] - 1.0 / V) < 1e-15
+    assert out["idx"][0] == 0
+    assert out["gap"][0] == 0.0
+
+
+@pytest.mark.parametrize("V,win,delta", [(10, 7, 2.0), (4096, 4095, 5.0), (64, 0, 0.75)])
+def test_head_one_hot_gap(V, win, delta):
+    # One logit raised by delta above V-1 equal ones: c = 1 / (1 + (V-1) e^-delta).
+    W = np.zeros((V, 1), np.float32)
+    W[win, 0] = 1.0
+    h = np.array([delta], np.float32)
+    out = oracle.head_rows(bf16_from_float(W), bf16_from_float(h).reshape(1, 1))
+    assert out["idx"][0] == win
+    assert abs(out["conf"][0] - 1.0 / (1.0 + (V - 1) * math.exp(-delta))) < 1e-14
+
+
+def test_head_invariants_random():
+    rng = np.random.default_rng(5)
+    V, H, M = 300, 64, 6
+    W = bf16_from_float(rng.normal(0, 0.3, (V, H)))
+    R = bf16_from_float(rng.normal(0, 1.0, (M, H)))
+    out = oracle.head_rows(W, R, n_threads=3)
+    for i in range(M):
+        z, p, idx = oracle.softmax_row(W, R[i])
+        assert abs(p.sum() - 1.0) < 1e-12
+        assert idx == out["idx"][i]
+        assert abs(out["conf"][i] - p.max()) < 1e-15
+        assert abs(out["conf"][i] - math.exp(out["zmax"][i] - out["lse"][i])) < 1e-13
+        s = np.sort(z)
+        assert abs(out["gap"][i] - (s[-1] - s[-2])) < 1e-12
+    # thread count does not change any bit
+    out1 = oracle.head_rows(W, R, n_threads=1)
+    for k in out:
+        np.testing.assert_array_equal(out[k], out1[k])
+
+
+# ------------------------------------------------------------ thresholds --
+
+def test_theta_e_printed_values():
+    cfg = oracle.Config()
+    for b, te in _rows("block_end_thresholds.txt"):
+        assert abs(oracle.theta_e(cfg, int(b)) - float(te)) < 1e-12
+    # floor for b > 4 (non-increasing, never below the b = 4 value)
+    vals = [oracle.theta_e(cfg, b) for b in range(1, 17)]
+    assert all(vals[i + 1] <= vals[i] for i in range(15))
+    assert min(vals) == pytest.approx(0.40, abs=1e-12)
+    # quarter mode over 16 blocks: blocks 1-4 -> 0.70, 5-8 -> 0.60, 9-12 -> 0.50, 13-16 -> 0.40
+    q = oracle.Config(n_blocks=16, flags=oracle.GATING | oracle.POS_FACTOR | oracle.QUARTER_BLOCKS)
+    assert [round(oracle.theta_e(q, b), 12) for b in (1, 4, 5, 8, 9, 12, 13, 16)] == \
+        [0.7, 0.7, 0.6, 0.6, 0.5, 0.5, 0.4, 0.4]
+
+
+def test_theta_block_golden():
+    for T, b, t, th in _rows("theta_schedule.txt"):
+        cfg = oracle.Config(T=int(T))
+        assert abs(oracle.theta_block(cfg, int(b), int(t)) - float(th)) < 6e-7, (T, b, t)
+
+
+@pytest.mark.parametrize("T", [8, 20, 32, 64])
+@pytest.mark.parametrize("b", [1, 2, 4, 7])
+def test_theta_block_shape(T, b):
+    cfg = oracle.Config(T=T, n_blocks=8)
+    te = oracle.theta_e(cfg, b)
+    th = [oracle.theta_block(cfg, b, t) for t in range(T)]
+    assert all(th[i + 1] <= th[i] + 1e-15 for i in range(T - 1))
+    assert all(te < x <= 0.9 + 1e-15 for x in th)
+    # warm-up: exactly the steps with t < 0.15 T hold theta_s
+    for t in range(T):
+        assert (th[t] == 0.9) == (t < 0.15 * T) or (t >= 0.15 * T and abs(th[t] - 0.9) < 1e-3)
+    # continuity at wT and the end point theta_e at t = T (cosine of pi)
+    wT = 0.15 * T
+    alpha = (0.9 - te) / 2
+    # the first post-warm-up step sits within alpha*(pi*u)^2/2 of theta_s
+    t1 = math.ceil(wT)
+    u1 = (t1 - wT) / (T - wT)
+    assert 0.9 - th[t1] <= alpha * (math.pi * u1) ** 2 / 2 + 1e-12
+    # extrapolating one step past T - 1 lands on theta_e to first order
+    uL = (T - 1 - wT) / (T - wT)
+    assert th[T - 1] - te <= alpha * (math.pi * (1 - uL)) ** 2 / 2 + 1e-12
+
+
+def test_position_factor_printed():
+    cfg = oracle.Config(P=64)
+    for p, r in _rows("position_factors.txt"):
+        assert oracle.pos_factor(cfg, int(p)) == float(r)
+    off = oracle.Config(P=64, flags=oracle.GATING)
+    assert oracle.pos_factor(off, 0) == 1.0 and oracle.pos_factor(off, 63) == 1.0
+    q = oracle.Config(P=32, flags=oracle.POS_FACTOR | oracle.QUARTER_POS)
+    assert [oracle.pos_factor(q, p) for p in (0, 7, 8, 15, 16, 23, 24, 31)] == \
+        [0.8, 0.8, 0.9, 0.9, 1.05, 1.05, 1.1, 1.1]
+
+
+def test_theta_token_clip():
+    cfg = oracle.Config(T=32, P=64)
+    # 0.90 * 1.10 = 0.99 is clipped to 0.98
+    assert oracle.theta_token(cfg, 1, 0, 60) == pytest.approx(0.98, abs=1e-15)
+    # 0.90 * 0.80 = 0.72 unclipped
+    assert oracle.theta_token(cfg, 1, 0, 3) == pytest.approx(0.72, abs=1e-12)
+    # block 4, last step: theta ~ 0.4017, times 0.80 -> 0.3213, unclipped
+    assert oracle.theta_token(cfg, 4, 31, 0) == pytest.approx(0.401666 * 0.8, abs=1e-6)
+    # a lower floor makes the 0.20 clip bite
+    low = oracle.Config(T=32, P=64, theta_e1=0.2, theta_e_min=0.1)
+    assert oracle.theta_token(low, 2, 31, 0) == pytest.approx(0.20, abs=1e-15)
+
+
+def test_budget_table():
+    cfg = oracle.Config(P=64)
+    for p, s, bud in _rows("budget_table.txt"):
+        assert oracle.budget(cfg, float(s), int(p)) == int(bud), (p, s)
+    q = oracle.Config(P=32, flags=oracle.GATING | oracle.QUARTER_POS)
+    assert oracle.budget(q, 0.9, 15) == 8 and oracle.budget(q, 0.9, 16) == 32
+    assert oracle.budget(q, 0.9, 24) == 64
+
+
+def test_low_yield_readings():
+    cnt = oracle.Config()
+    assert oracle.low_yield(cnt, 0) and oracle.low_yield(cnt, 1) and not oracle.low_yield(cnt, 2)
+    frac = oracle.Config(eta_mode=1, eta_bar=0.015, n_blocks=8, P=32)   # L = 256, 1.5% = 3.84
+    assert oracle.low_yield(frac, 3) and not oracle.low_yield(frac, 4)
+
+
+# ------------------------------------------------------------- controller --
+
+def _feed(cfg, seq):
+    """Run controller steps on block 0 with per-step (conf[B,P], idx[B,P])."""
+    st = oracle.State(cfg)
+    for t, (c, i) in enumerate(seq):
+        oracle.controller_step(st, 0, t, np.asarray(c, np.float64), np.asarray(i, np.int32))
+        if np.all(st.exit_reason[:, 0] != oracle.RUNNING):
+            break
+    return st
+
+
+def test_trajectory_G1_grinding_exit():
+    # eta = 0, 0, 1, 0 -> ell = 1, 2, 3, 4 -> grinding at t = 3 (Box 7, K = 4).
+    cfg = oracle.Config(B=1, P=4, T=10, n_blocks=1)
+    idx = [[10, 11, 12, 13]]
+    seq = [([[0.1, 0.1, 0.1, 0.1]], idx),
+           ([[0.1, 0.1, 0.1, 0.1]], idx),
+           ([[0.95, 0.1, 0.1, 0.1]], idx),
+           ([[0.0, 0.41, 0.40, 0.2]], idx)]
+    st = _feed(cfg, seq)
+    assert st.exit_reason[0, 0] == oracle.EXIT_GRIND
+    assert st.exit_step[0, 0] == 3
+    assert st.ell[0] == 4
+    # token 0 by threshold at t=2; token 1 forced (0.41 > 0.40); token 2 not (strict >)
+    assert list(st.tok[0]) == [10, 11, -1, -1]
+    assert list(st.cstep[0]) == [2, 3, -1, -1]
+    assert st.unresolved[0, 0] == 2
+    # all budgets 64 (s = 0.1 < 0.25)
+    assert list(st.budget[0]) == [64] * 4
+
+
+def test_trajectory_G2_counter_reset():
+    # eta = 0, 2, 0, 0, 0, 0 -> ell = 1, 0, 1, 2, 3, 4 -> exit at t = 5.
+    cfg = oracle.Config(B=1, P=6, T=10, n_blocks=1)
+    idx = [list(range(6))]
+    lo = [0.1] * 6
+    seq = [([lo], idx), ([[0.99, 0.99] + [0.1] * 4], idx)] + [([lo], idx)] * 4
+    ells = []
+    st = oracle.State(cfg)
+    for t, (c, i) in enumerate(seq):
+        oracle.controller_step(st, 0, t, np.asarray(c), np.asarray(i, np.int32))
+        ells.append(int(st.ell[0]))
+    assert ells == [1, 0, 1, 2, 3, 4]
+    assert st.exit_reason[0, 0] == oracle.EXIT_GRIND and st.exit_step[0, 0] == 5
+
+
+def _budget_force_seq(P, T):
+    # token 0: s = 0.6 at p = 0 -> B = 8; c stays 0.5 < theta.  Tokens 1..P-1
+    # commit two per step (c = 0.99) so the low-yield counter stays at 0.
+    seq = []
+    for t in range(T):
+        c = [0.5] + [0.0] * (P - 1)
+        for j in (1 + 2 * t, 2 + 2 * t):
+            if j < P:
+                c[j] = 0.99
+        c[0] = 0.6 if t == 0 else 0.5
+        seq.append(([c], [list(range(100, 100 + P))]))
+    return seq
+
+
+def test_budget_force_commit_at_exactly_B():
+    P, T = 22, 12
+    cfg = oracle.Config(B=1, P=P, T=T, n_blocks=1)
+    st = _feed(cfg, _budget_force_seq(P, T))
+    assert st.budget[0, 0] == 8
+    assert st.tok[0, 0] == 100 and st.cstep[0, 0] == 8
+    # gating OFF: no budgets, token 0 is never committed by budget
+    off = oracle.Config(B=1, P=P, T=T, n_blocks=1, flags=oracle.POS_FACTOR)
+    st2 = _feed(off, _budget_force_seq(P, T))
+    assert st2.tok[0, 0] == -1
+    assert st2.exit_reason[0, 0] == oracle.EXIT_TMAX and st2.exit_step[0, 0] == T - 1
+
+
+def test_done_exit_and_batch_independence():
+    cfg = oracle.Config(B=2, P=3, T=8, n_blocks=2)
+    idx = [[1, 2, 3], [4, 5, 6]]
+    seq = [([[0.99, 0.99, 0.5], [0.99, 0.99, 0.99]], idx),
+           ([[0.0, 0.0, 0.99], [0.0, 0.0, 0.0]], idx)]
+    st = oracle.State(cfg)
+    for t, (c, i) in enumerate(seq):
+        oracle.controller_step(st, 0, t, np.asarray(c), np.asarray(i, np.int32))
+    # sequence 1 finished at t = 0 (all three committed), sequence 0 at t = 1
+    assert st.exit_reason[1, 0] == oracle.EXIT_DONE and st.exit_step[1, 0] == 0
+    assert st.exit_reason[0, 0] == oracle.EXIT_DONE and st.exit_step[0, 0] == 1
+    assert list(st.tok[0, :3]) == [1, 2, 3] and list(st.tok[1, :3]) == [4, 5, 6]
+    # block 1 untouched
+    assert np.all(st.tok[:, 3:] == -1)
+    # an exited sequence ignores later steps
+    oracle.controller_step(st, 0, 2, np.full((2, 3), 0.999), np.full((2, 3), 77, np.int32))
+    assert list(st.tok[1, :3]) == [4, 5, 6]
+
+
+def test_t_exhausted_and_flush():
+    cfg = oracle.Config(B=1, P=2, T=3, n_blocks=1, flags=oracle.POS_FACTOR)
+    idx = [[7, 8]]
+    seq = [([[0.1, 0.2]], idx), ([[0.1, 0.2]], idx), ([[0.3, 0.95]], idx)]
+    st = _feed(cfg, seq)
+    assert st.exit_reason[0, 0] == oracle.EXIT_TMAX and st.exit_step[0, 0] == 2
+    assert list(st.tok[0]) == [-1, 8] and st.unresolved[0, 0] == 1
+    fl = oracle.Config(B=1, P=2, T=3, n_blocks=1, flags=oracle.POS_FACTOR | oracle.FLUSH_ON_EXIT)
+    st2 = _feed(fl, seq)
+    assert list(st2.tok[0]) == [7, 8] and st2.unresolved[0, 0] == 0
+    assert list(st2.cstep[0]) == [2, 2]
+
+
+def test_threshold_inclusive_and_position_factor_in_commit():
+    # t = 0, theta_s = 0.9: p < 16 needs c >= 0.72 (inclusive), p in [16, 32) needs 0.81
+    cfg = oracle.Config(B=1, P=32, T=32, n_blocks=1)
+    c = np.full((1, 32), 0.1)
+    th0 = oracle.theta_token(cfg, 1, 0, 0)     # 0.9 * 0.8 in double
+    th17 = oracle.theta_token(cfg, 1, 0, 17)   # 0.9 * 0.9 in double
+    assert th0 == pytest.approx(0.72, abs=1e-15) and th17 == pytest.approx(0.81, abs=1e-15)
+    c[0, 0] = th0                        # exactly the threshold -> commits
+    c[0, 1] = np.nextafter(th0, 0.0)     # one ulp below -> does not
+    c[0, 16] = 0.80                      # below 0.81 -> does not
+    c[0, 17] = th17                      # commits
+    st = oracle.State(cfg)
+    oracle.controller_step(st, 0, 0, c, np.arange(32, dtype=np.int32).reshape(1, 32))
+    assert [st.tok[0, p] for p in (0, 1, 16, 17)] == [0, -1, -1, 17]
+    assert st.eta[0] == 2
+
+
+def _check_invariants(st: oracle.State, cfg: oracle.Config, history):
+    """Invariants of Algorithm 1 over a finished trajectory."""
+    gating = bool(cfg.flags & oracle.GATING)
+    # committed tokens never change (history holds tok snapshots per step)
+    for a, b in zip(history, history[1:]):
+        done = a != -1
+        assert np.all(b[done] == a[done])
+    committed = st.tok != -1
+    if gating:
+        assert np.all(st.cstep[committed] <= st.budget[committed])
+    for b in range(cfg.B):
+        for blk in range(cfg.n_blocks):
+            sl = slice(blk * cfg.P, (blk + 1) * cfg.P)
+            cs = st.cstep[b, sl]
+            if st.exit_step[b, blk] >= 0:
+                assert np.all(cs[cs >= 0] <= st.exit_step[b, blk])
+            assert st.unresolved[b, blk] == np.sum(st.tok[b, sl] == -1)
+
+
+@pytest.mark.parametrize("mode", ["calibrated", "literal"])
+def test_toy_trajectory_invariants(mode):
+    wl = synth.WORKLOADS["toy"]
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w)
+    hs = synth.HiddenStates(wl, W, mode)
+    cfg = oracle.Config(B=wl.B, P=wl.P, T=wl.T, n_blocks=wl.n_blocks)
+    history = []
+    Ms = []
+    etas = []
+
+    def on_step(st, blk, t, out):
+        history.append(st.tok.copy())
+        Ms.append((blk, t, out["M"]))
+        etas.append(int(st.eta.sum()))
+
+    st = oracle.run_trajectory(cfg, W, hs, on_step=on_step)
+    _check_invariants(st, cfg, history)
+    # M_{t+1} = M_t - (tokens committed at t), within a block
+    for k in range(len(Ms) - 1):
+        (b0, t0, m0), (b1, t1, m1) = Ms[k], Ms[k + 1]
+        if b0 == b1:
+            before = np.sum(history[k - 1] != -1) if k > 0 else 0
+            n_new = int(np.sum(history[k] != -1) - before)    # commits made at step k
+            assert m1 == m0 - n_new
+    if mode == "literal":
+        # c ~ 1/V: every budget is 64 and every block exits by grinding at t = 3
+        assert np.all(st.budget == 64)
+        assert np.all(st.exit_reason == oracle.EXIT_GRIND) and np.all(st.exit_step == 3)
+        assert np.all(st.tok == -1)
+
+
+def test_theta_e_non_increasing_in_trajectory_configs():
+    for nb in (4, 8, 16):
+        cfg = oracle.Config(n_blocks=nb)
+        vals = [oracle.theta_e(cfg, b) for b in range(1, nb + 1)]
+        assert all(x >= y for x, y in zip(vals, vals[1:]))

@@ -298,6 +298,7 @@ void cai_o_controller_step(const cai_o_cfg* c, cai_o_state* st, int32_t blk, int
   for (int32_t b = 0; b < B; ++b) {
     const int32_t eb = b * c->n_blocks + blk;
     if (st->exit_reason[eb] != CAI_O_RUNNING) continue;
+    if (t == 0) st->ell[b] = 0; /* Algorithm 1: ell <- 0 before the block's first step */
     int32_t eta = 0;
     /* commit loop: foreach masked token i */
     for (int32_t p = 0; p < P; ++p) {

@@ -1,0 +1,413 @@
+"""Benchmark of the CAI-dLLM fused decoding head + commit rule on GB300.
+
+One bench "step" is one whole generation of the workload: every block, each
+block run step by step (step zero, then denoising steps until every sequence
+exits, with the host polling the device's done flag one step behind), every
+step being gather -> LM head with online softmax -> merge + commit.  The metric
+is masked positions decoded per second, summed over all steps (sum of M_t)
+and over all ranks, divided by the device time of the timed region.
+
+Default workload (N = 1): LLaDA-8B-shaped, B = 1, H = 4096, V = 126464,
+generation length 256 in 8 blocks of 32, up to 32 steps per block, seeded
+synthetic bf16 weight and hidden states (``synth``).  The weight (1.04 GB) is
+larger than L2, so every step reads it from HBM.
+
+Arms:
+  (default)          the sm_103a path through the C ABI (``paper_2608_22646_gb300``);
+  --impl reference   the fp64 CPU oracle as it stands, on the host cores, on a
+                     bounded sample of the same workload (there is no published
+                     implementation of the method to run).
+
+Multi-GPU: under torchrun each rank decodes its own batch (sequences are
+independent, no collective on the data path); value = all ranks' positions /
+the slowest rank's time ("weak" scaling).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+if ROOT not in sys.path:
+    sys.path.insert(0, ROOT)
+
+METRIC = "masked positions decoded/s (fused head+commit) at 1 GB300; % of HBM/tensor roofline"
+UNIT = "positions/s"
+PROFILES = os.path.join(ROOT, "profiles")
+
+
+def _peaks():
+    p = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(p):
+        with open(p) as f:
+            d = json.load(f)
+        return d["hbm_gbs"], d["bf16_tflops"], d.get("bf16_tflops_sustained"), "measured"
+    return 6800.0, 1900.0, 1700.0, "fallback"
+
+
+def _workload_desc(wl, gen):
+    return {"workload": f"{wl.name}: B={wl.B} H={wl.H} V={wl.V} gen_len={wl.gen_len} "
+                        f"block={wl.P} T={wl.T}",
+            "B": wl.B, "H": wl.H, "V": wl.V, "gen_len": wl.gen_len, "block": wl.P,
+            "max_steps_per_block": wl.T, "hidden_generator": gen,
+            "l2": "inputs larger than L2 (LM-head weight %.2f GB read every step)"
+                  % (wl.V * wl.H * 2 / 1e9)}
+
+
+class Clocks:
+    """nvidia-smi sampling of SM clocks and throttle reasons during a region."""
+    FIELDS = ("index,clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, index: int):
+        self.index = index
+        self.proc = None
+        self.path = os.path.join("/tmp", f"cai_clocks_{os.getpid()}.csv")
+
+    def __enter__(self):
+        try:
+            self.f = open(self.path, "w")
+            self.proc = subprocess.Popen(
+                ["nvidia-smi", "-i", str(self.index), f"--query-gpu={self.FIELDS}",
+                 "--format=csv,noheader,nounits", "-lms", "100"],
+                stdout=self.f, stderr=subprocess.DEVNULL)
+            time.sleep(0.3)
+        except (OSError, ValueError):
+            self.proc = None
+        return self
+
+    def __exit__(self, *a):
+        if self.proc is not None:
+            time.sleep(0.15)
+            self.proc.terminate()
+            try:
+                self.proc.wait(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+            self.f.close()
+
+    def summary(self):
+        if self.proc is None or not os.path.exists(self.path):
+            return None
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        with open(self.path) as f:
+            for line in f:
+                parts = [x.strip() for x in line.split(",")]
+                if len(parts) < 9:
+                    continue
+                try:
+                    sm.append(float(parts[1]))
+                    mx = float(parts[2])
+                except ValueError:
+                    continue
+                for n, v in zip(names, parts[5:9]):
+                    if v.lower() == "active":
+                        reasons.add(n)
+        os.remove(self.path)
+        if not sm:
+            return None
+        return {"sm_mhz": statistics.median(sm), "sm_max_mhz": mx, "reasons": sorted(reasons),
+                "samples": len(sm)}
+
+
+def _traffic_record(kernel_src: str):
+    """DRAM bytes per launch of the LM-head kernel from the committed ncu
+    summary, if it was taken on the current kernel source."""
+    p = os.path.join(PROFILES, "lm_head_traffic.json")
+    if not os.path.exists(p):
+        return None
+    with open(p) as f:
+        rec = json.load(f)
+    with open(kernel_src, "rb") as f:
+        h = hashlib.sha256(f.read()).hexdigest()[:16]
+    return rec if rec.get("kernel_sha") == h else None
+
+
+def run_trajectory(cai, ctx, hidden, wl, lag_poll=True, stream=None):
+    """All blocks of one generation.  ``hidden[blk][t]`` is the step's input."""
+    for blk in range(wl.n_blocks):
+        if blk:
+            cai.cai_block_advance(ctx, stream)
+        cai.cai_first_step(ctx, hidden[blk][0], stream)
+        for t in range(1, wl.T):
+            if lag_poll and t >= 2 and cai.cai_poll(ctx, 1, 60000):
+                break
+            cai.cai_denoise_step(ctx, hidden[blk][t], stream)
+
+
+def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0):
+    """The oracle as it stands on the host cores: full steps of the same
+    trajectory (all masked rows of each step), for about budget_s seconds."""
+    import oracle
+    cfg = oracle.Config(B=wl.B, P=wl.P, T=wl.T, n_blocks=wl.n_blocks)
+    st = oracle.State(cfg)
+    Wb = oracle.bf16_bits(W)
+    threads = os.cpu_count() or 1
+    rows = 0
+    steps = 0
+    t0 = time.perf_counter()
+    for blk in range(wl.n_blocks):
+        for t in range(wl.T):
+            h = oracle.bf16_bits(hs_fn(blk, t))
+            out = oracle.step(st, Wb, h, blk, t, threads)
+            rows += out["M"]
+            steps += 1
+            if np.all(st.exit_reason[:, blk] != 0) or time.perf_counter() - t0 > budget_s:
+                break
+        if time.perf_counter() - t0 > budget_s:
+            break
+    dt = time.perf_counter() - t0
+    return {"value": rows / dt, "unit": UNIT, "cores": threads, "kind": "oracle",
+            "sample": f"first {steps} denoising steps of the trajectory ({rows} masked rows, "
+                      f"fp64, one thread per row), {dt:.1f} s"}
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=30)
+    ap.add_argument("--warmup", type=int, default=3)
+    ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
+    ap.add_argument("--workload", default="llada")
+    ap.add_argument("--generator", default="calibrated", choices=["calibrated", "literal"])
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    ap.add_argument("--no-e2e", action="store_true")
+    args = ap.parse_args()
+
+    import torch
+    import synth
+
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    rank = int(os.environ.get("RANK", "0"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    dist = None
+    if world > 1:
+        import torch.distributed as dist
+        torch.cuda.set_device(local)
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    wl = synth.WORKLOADS[args.workload]
+
+    if args.impl == "reference":
+        if rank != 0:
+            if dist:
+                dist.barrier()
+                dist.destroy_process_group()
+            return
+        run_reference(args, wl)
+        if dist:
+            dist.barrier()
+            dist.destroy_process_group()
+        return
+
+    import paper_2608_22646_gb300 as cai
+    from paper_2608_22646_gb300 import build as cai_build
+    cai_build.build()
+    dev = torch.device("cuda", local)
+    torch.cuda.set_device(dev)
+    stream = torch.cuda.current_stream(dev)
+
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device=dev)
+    hs = synth.HiddenStates(wl, W, args.generator, seed=wl.seed_h + 1000 * rank)
+    hidden = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    torch.cuda.synchronize()
+
+    cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    ctx = cai.cai_init(cfg, W)
+
+    for _ in range(args.warmup):
+        cai.cai_reset(ctx)
+        run_trajectory(cai, ctx, hidden, wl)
+    torch.cuda.synchronize()
+    st0 = cai.cai_state_download(ctx)
+    positions = int(st0["m_hist"].sum())
+    nonzero_launch = int((st0["m_hist"] > 0).sum())
+    launches_per_traj = int((st0["m_hist"] > 0).sum())
+    stats0 = cai.cai_get_stats(ctx)
+
+    cai.cai_profile(ctx, True)
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with Clocks(local) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            cai.cai_reset(ctx)
+            run_trajectory(cai, ctx, hidden, wl)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    cai.cai_profile(ctx, False)
+    ms = ev0.elapsed_time(ev1)
+    stats1 = cai.cai_get_stats(ctx)
+    st1 = cai.cai_state_download(ctx)
+    assert np.array_equal(st1["m_hist"], st0["m_hist"]), "trajectory changed between runs"
+    head_launches = stats1["head_launches"] - stats0["head_launches"]
+    head_ms = stats1["head_ms"] - stats0["head_ms"]
+    gpu_launches = stats1["launches"] - stats0["launches"]
+
+    if dist:
+        t = torch.tensor([ms], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        ms = float(t.item())
+    total_positions = positions * args.steps * world
+    value = total_positions / (ms / 1e3)
+
+    # Roofline of the dominant kernel (LM head): algorithmic bytes of every
+    # launch = W once (2 V H, only when it decodes rows) + the masked rows (2 M H).
+    hbm, tf_burst, tf_sus, peak_kind = _peaks()
+    alg_bytes = args.steps * (nonzero_launch * 2.0 * wl.V * wl.H + positions * 2.0 * wl.H)
+    alg_flops = args.steps * positions * 2.0 * wl.V * wl.H
+    head_s = head_ms / 1e3
+    mean_m = positions / max(1, nonzero_launch)
+    bound = "hbm" if mean_m < hbm * 1e9 / (tf_burst * 1e12) * 2 else "tensor"
+    tr = _traffic_record(os.path.join(ROOT, "paper_2608_22646_gb300", "csrc", "head_kernel.cuh"))
+    if bound == "hbm":
+        achieved = alg_bytes / head_s / 1e9
+        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
+                "frac": round(achieved / hbm, 4),
+                "traffic": (tr["dram_bytes_per_launch"] if tr and tr.get("workload") == wl.name
+                            else None),
+                "algorithmic_bytes_per_launch": round(alg_bytes / max(1, head_launches)),
+                "kernel": "lm_head_softmax_kernel", "peak_source": f"{peak_kind} hbm_gbs",
+                "head_launches": head_launches, "head_ms_total": round(head_ms, 3)}
+    else:
+        achieved = alg_flops / head_s / 1e12
+        pk = tf_sus or tf_burst
+        roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": pk, "unit": "TFLOP/s",
+                "frac": round(achieved / pk, 4), "traffic": None,
+                "kernel": "lm_head_softmax_kernel", "peak_source": f"{peak_kind} bf16 sustained",
+                "head_launches": head_launches, "head_ms_total": round(head_ms, 3)}
+
+    line = {
+        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4),
+        "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
+        "data": "synthetic (seeded LLaDA/Dream-shaped weight and hidden states; no model weights)",
+        "config": {**_workload_desc(wl, args.generator), "parallelism": f"replicas x{world}",
+                   "positions_per_step": positions, "head_launches_per_step": launches_per_traj,
+                   "steps_per_generation": int((st0["m_hist"] > 0).sum())},
+        "roofline": roof,
+        "gpu_launches": int(gpu_launches),
+        "clocks": clk.summary(),
+    }
+
+    if not args.no_e2e:
+        line["e2e"] = e2e_run(cai, ctx, hs, wl, args, dist, dev)
+    if rank == 0 and world == 1 and not args.no_cpu_baseline:
+        line["cpu_baseline"] = cpu_baseline(wl, W, lambda b, t: hidden[b][t])
+    cai.cai_free(ctx)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
+    if dist:
+        dist.destroy_process_group()
+
+
+def e2e_run(cai, ctx, hs, wl, args, dist, dev):
+    """Same metric through the public C ABI with host buffers: every step's
+    hidden states come from pinned host memory (copied inside the step call),
+    every step's done flag is read from host-mapped memory, and each
+    generation's tokens are copied back to pinned host memory."""
+    import torch
+    host = [[hs(blk, t).cpu().pin_memory() for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    out = torch.empty((wl.B, wl.n_blocks * wl.P), dtype=torch.int32).pin_memory()
+    steps = max(3, args.steps // 3)
+    stream = torch.cuda.current_stream(dev)
+    cai.cai_reset(ctx)
+    run_trajectory(cai, ctx, host, wl)
+    cai.cai_read_tokens(ctx, out)
+    torch.cuda.synchronize()
+    s0 = cai.cai_get_stats(ctx)["steps"]
+    if dist:
+        dist.barrier()
+    t0 = time.perf_counter()
+    for _ in range(steps):
+        cai.cai_reset(ctx)
+        run_trajectory(cai, ctx, host, wl)
+        cai.cai_read_tokens(ctx, out)
+        stream.synchronize()
+    dt = time.perf_counter() - t0
+    st = cai.cai_state_download(ctx)
+    n_step_calls = (cai.cai_get_stats(ctx)["steps"] - s0) / steps
+    world = 1
+    if dist:
+        t = torch.tensor([dt], device=dev)
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+        dt = float(t.item())
+        world = dist.get_world_size()
+    positions = int(st["m_hist"].sum())
+    return {"value": round(positions * steps * world / dt, 1), "unit": UNIT,
+            "h2d_bytes_per_step": int(n_step_calls * wl.B * wl.P * wl.H * 2),
+            "d2h_bytes_per_step": int(wl.B * wl.n_blocks * wl.P * 4 + n_step_calls * 32),
+            "timing": "host wall clock around whole generations, pinned host inputs"}
+
+
+def run_reference(args, wl):
+    """The oracle on the host cores: each bench step is one denoising step of
+    the trajectory (every masked row of that step), in trajectory order."""
+    import torch
+    import oracle
+    import synth
+    oracle.build()
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device="cpu")
+    hs = synth.HiddenStates(wl, W, args.generator)
+    cfg = oracle.Config(B=wl.B, P=wl.P, T=wl.T, n_blocks=wl.n_blocks)
+    st = oracle.State(cfg)
+    Wb = oracle.bf16_bits(W)
+    threads = os.cpu_count() or 1
+    order = [(b, t) for b in range(wl.n_blocks) for t in range(wl.T)]
+    pos = 0
+    rows = 0
+    dt = 0.0
+    k = 0
+
+    def one():
+        nonlocal pos
+        while True:
+            b, t = order[pos % len(order)]
+            pos += 1
+            if t == 0:
+                if b == 0:
+                    st.__init__(cfg)
+                st.ell[:] = 0
+            if np.all(st.exit_reason[:, b] != 0):
+                continue
+            h = oracle.bf16_bits(hs(b, t))
+            t0 = time.perf_counter()
+            out = oracle.step(st, Wb, h, b, t, threads)
+            return out["M"], time.perf_counter() - t0
+
+    for _ in range(args.warmup):
+        one()
+    for _ in range(args.steps):
+        m, s = one()
+        rows += m
+        dt += s
+        k += 1
+    v = rows / dt
+    line = {"impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": UNIT,
+            "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": round(dt / k * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+            "config": _workload_desc(wl, args.generator),
+            "cpu_baseline": {"value": round(v, 3), "unit": UNIT, "cores": threads,
+                             "kind": "oracle",
+                             "sample": f"{k} denoising steps of the trajectory, {rows} masked rows"},
+            "e2e": {"value": round(v, 3), "unit": UNIT, "h2d_bytes_per_step": 0,
+                    "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+if __name__ == "__main__":
+    main()

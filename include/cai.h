@@ -1,0 +1,259 @@
+/*
+ * cai.h: C ABI of the GB300 (sm_103a) decoding head and commit controller
+ * of CAI-dLLM, "Convergence Aware Inference for diffusion LLMs"
+ * (arXiv 2608.22646).
+ *
+ * One denoising step, for the masked positions of the current output block of
+ * every sequence in the batch:
+ *   1. logits z = W h for each masked row (Box 1: p_theta(x_i | x^(t)) over the
+ *      vocabulary), on tcgen05 tensor cores, never written to memory;
+ *   2. the full-vocabulary softmax reduced to the confidence
+ *      c_i = max_v p(v) and the greedy token argmax_v p(v) (Box 1, temperature 0
+ *      per Section 5 "Setup");
+ *   3. the commit rule of Algorithm 1: first-step confidence s_i (Box 2),
+ *      token budgets B_i (Box 5, Eq. token_budget), the cosine threshold
+ *      schedule with block end thresholds theta_e^(b) (Boxes 3-4), position
+ *      thresholds (Box 6, Eqs. position_threshold and position_commit), the
+ *      grinding detector and its force commit (Box 7, Eq. grinding-detector),
+ *      all behind the model-adaptive gate (Section 4.6).
+ *
+ * Execution model.  Every call that takes a stream is asynchronous on that
+ * stream (a CUDA stream handle, or NULL for the legacy default stream); the
+ * library never synchronises the device on the step path.  The batch runs
+ * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
+ * per sequence) and contribute no rows afterwards.  A context is not thread
+ * safe; use one context per host thread.
+ *
+ * Status.  Every int-returning call returns CAI_OK (0) or a negative CAI_ERR_*
+ * code; no C++ exception crosses the ABI.  After CAI_ERR_CUDA or
+ * CAI_ERR_DEVICE the context is poisoned ("sticky"): every later call except
+ * cai_free and cai_strerror returns the same code.
+ */
+#ifndef CAI_H
+#define CAI_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+/* ------------------------------------------------------------------ status */
+#define CAI_OK 0
+#define CAI_ERR_ARG (-1)         /* NULL pointer, bad enum, bad value            */
+#define CAI_ERR_SHAPE (-2)       /* unsupported sizes (see cai_config)           */
+#define CAI_ERR_ORDER (-3)       /* call out of order (see each step call)       */
+#define CAI_ERR_CUDA (-4)        /* a CUDA runtime call failed (sticky)          */
+#define CAI_ERR_TIMEOUT (-5)     /* cai_poll gave up waiting (not sticky)        */
+#define CAI_ERR_DEVICE (-6)      /* a kernel's bounded wait gave up (sticky)     */
+#define CAI_ERR_UNSUPPORTED (-7) /* the current device is not compute 10.3       */
+#define CAI_ERR_NOMEM (-8)       /* an allocation failed                         */
+
+/* ------------------------------------------------------------------- flags */
+#define CAI_GATING 1u           /* Section 4.6 gate ON: budgets, grinding exit, force commit */
+#define CAI_POS_FACTOR 2u       /* Box 6 position factors r_pos (else r = 1)                */
+#define CAI_FLUSH_ON_EXIT 4u    /* commit still-masked tokens to their argmax when a block exits */
+#define CAI_QUARTER_POS 8u      /* position/budget tiers at P/4, P/2, 3P/4 instead of 16/32/48 */
+#define CAI_QUARTER_BLOCKS 16u  /* theta_e^(b) indexed by the quarter of the output block b is in */
+
+#define CAI_PRESET_LLADA 0      /* gating ON  (Section 5: LLaDA-8B-Instruct) */
+#define CAI_PRESET_DREAM 1      /* gating OFF (Section 5: Dream-7B-Instruct) */
+
+#define CAI_MASK_TOKEN (-1)     /* token id of a still-masked position */
+
+/* exit reasons of a block, per sequence (Algorithm 1) */
+#define CAI_RUNNING 0
+#define CAI_EXIT_DONE 1         /* no masked token remained                 */
+#define CAI_EXIT_GRIND 2        /* grinding phase detected (Box 7)          */
+#define CAI_EXIT_TMAX 3         /* reached local step T - 1                 */
+
+/*
+ * Workload and controller hyperparameters.  Algorithm 1 inputs: T, theta_s,
+ * theta_e^(b) (via theta_e1 - theta_e_step (b - 1), floored at theta_e_min),
+ * theta_fb, w (warmup_pct / 100), K, eta_bar.
+ *
+ * Shape limits (else CAI_ERR_SHAPE): B >= 1; 1 <= P <= 256; H % 64 == 0 and
+ * 64 <= H <= 16384; V >= 64; 1 <= T <= 32767; n_blocks >= 1; B * P <= 65536.
+ */
+typedef struct cai_config {
+  int32_t B;           /* sequences in the batch                                  */
+  int32_t P;           /* block length (positions per block)                      */
+  int32_t H;           /* hidden size                                             */
+  int32_t V;           /* vocabulary size                                         */
+  int32_t T;           /* maximum denoising steps per block                       */
+  int32_t n_blocks;    /* blocks per generation (generation length / P)           */
+  double theta_s;      /* Box 3 start threshold, 0.90                             */
+  double theta_e1;     /* Box 4 end threshold of block 1, 0.70                    */
+  double theta_e_step; /* Box 4 decrease per block, 0.10                          */
+  double theta_e_min;  /* floor of theta_e^(b) for b > 4, 0.40                     */
+  int32_t warmup_pct;  /* Box 3 warm-up fraction w in percent, 15                 */
+  int32_t K;           /* Box 7 patience window, 4                                */
+  double theta_fb;     /* Box 7 force-commit threshold, 0.40                      */
+  double clip_lo;      /* Box 6 clip range, 0.20                                  */
+  double clip_hi;      /*                   0.98                                  */
+  double eta_bar;      /* Box 7 low-yield threshold: 1.5 (count) or 0.015 (fraction) */
+  int32_t eta_mode;    /* 0: eta counts new commits; 1: eta / (n_blocks P)        */
+  uint32_t flags;      /* CAI_* flags above                                       */
+} cai_config;
+
+typedef struct cai_ctx cai_ctx;
+
+/*
+ * Device views of the controller state (all device pointers, owned by the
+ * context, valid until cai_free).  L = n_blocks * P.  Row-major.
+ */
+typedef struct cai_state_view {
+  int32_t* tok;         /* [B, L] committed token id, CAI_MASK_TOKEN while masked   */
+  float* conf;          /* [B, L] c_i at the last step that saw the token masked    */
+  float* s0;            /* [B, L] first-step confidence s_i (Box 2)                 */
+  uint8_t* budget;      /* [B, L] B_i in {8, 32, 64} (Box 5), 0 before the block    */
+  int16_t* cstep;       /* [B, L] local step at which the token committed, -1       */
+  int32_t* cand;        /* [B, L] argmax at the last step that saw the token masked */
+  int32_t* ell;         /* [B] low-yield counter of the current block (Algorithm 1) */
+  int32_t* eta;         /* [B] tokens committed by the commit rule at the last step */
+  int32_t* exit_reason; /* [B, n_blocks] CAI_RUNNING / CAI_EXIT_*                   */
+  int32_t* exit_step;   /* [B, n_blocks] local step of the exit, -1                 */
+  int32_t* unresolved;  /* [B, n_blocks] tokens left masked at the exit             */
+  int32_t* m_hist;      /* [n_blocks, T] masked rows decoded by each step (M_t)     */
+} cai_state_view;
+
+/*
+ * Host copy of the controller state, for cai_state_download / cai_state_upload.
+ * Each pointer is caller-owned host memory of the size given in
+ * cai_state_view, or NULL to skip that field.  blk and t_next are the host
+ * counters: the 0-based current block and the next local step to run.
+ */
+typedef struct cai_host_state {
+  int32_t* tok;
+  float* conf;
+  float* s0;
+  uint8_t* budget;
+  int16_t* cstep;
+  int32_t* cand;
+  int32_t* ell;
+  int32_t* eta;
+  int32_t* exit_reason;
+  int32_t* exit_step;
+  int32_t* unresolved;
+  int32_t* m_hist;
+  int32_t blk;
+  int32_t t_next;
+} cai_host_state;
+
+/* Counters kept by the context (host side) since cai_init. */
+typedef struct cai_stats {
+  int64_t steps;            /* step calls issued                                   */
+  int64_t launches;         /* kernels launched by this context                    */
+  int64_t head_launches;    /* launches of the LM-head kernel                      */
+  double head_ms;           /* summed device time of profiled LM-head launches     */
+  int64_t head_profiled;    /* LM-head launches timed (cai_profile enabled)        */
+  int32_t grid;             /* CTAs of the LM-head kernel                          */
+  int32_t stages;           /* pipeline stages of the LM-head kernel               */
+  int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
+  int32_t reserved;
+} cai_stats;
+
+/* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")
+ * for the given preset and shapes.  Returns CAI_ERR_ARG for a bad preset. */
+int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, int32_t H,
+                       int32_t V, int32_t T, int32_t n_blocks);
+
+/*
+ * Create a context.  W is the LM-head weight [V, H] bf16, row-major.  If W is
+ * a device pointer it must stay valid and unchanged until cai_free (the
+ * library reads it in place and never frees it); if it is host memory the
+ * library copies it into an owned device buffer before returning.  All state
+ * starts at block 0, t = 0, every token masked.  Allocates device memory and
+ * one page of mapped pinned host memory.  Synchronous.
+ * Errors: CAI_ERR_ARG (NULL cfg/W/out), CAI_ERR_SHAPE, CAI_ERR_UNSUPPORTED,
+ * CAI_ERR_NOMEM, CAI_ERR_CUDA.
+ */
+int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out);
+
+/*
+ * Local step t = 0 of the current block (Algorithm 1, step-zero init): every
+ * position of every sequence is masked, so M = B P rows are decoded.  Stores
+ * s_i and B_i, then applies the commit rule with theta^(b)(0).
+ * hidden: the block's final hidden states [B, P, H] bf16, row-major; row
+ * (b, p) is the one that predicts position p of the block.  Device pointer:
+ * read on the stream, must stay valid until the stream passes this call.
+ * Host pointer (pinned or pageable): copied to the device inside the call.
+ * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call
+ * cai_block_advance or cai_reset first).
+ */
+int cai_first_step(cai_ctx* ctx, const void* hidden, void* stream);
+
+/*
+ * Local steps t = 1 .. T - 1 of the current block: decodes only the rows that
+ * are still masked in sequences that have not exited; a step issued after all
+ * sequences exited decodes nothing.  hidden as for cai_first_step.
+ * Errors: CAI_ERR_ORDER before cai_first_step of the block, after T steps, or
+ * after cai_poll has reported that every sequence exited the block.
+ */
+int cai_denoise_step(cai_ctx* ctx, const void* hidden, void* stream);
+
+/*
+ * Move to the next block (b += 1).  Host bookkeeping only; the low-yield
+ * counters are reset by the next cai_first_step.  Sequences still running in
+ * the old block keep CAI_RUNNING there.  Errors: CAI_ERR_ORDER if the current
+ * block never ran a step or it is the last block.
+ */
+int cai_block_advance(cai_ctx* ctx, void* stream);
+
+/* Start a new generation with the same weight: every token masked, block 0,
+ * counters cleared.  Asynchronous on the stream (device memsets only). */
+int cai_reset(cai_ctx* ctx, void* stream);
+
+/*
+ * Bounded host wait for the device's commit of the step issued `lag` step
+ * calls ago (lag = 0: the last one), read from mapped pinned memory without a
+ * device synchronisation.  On CAI_OK, *all_done is 1 if every sequence has
+ * exited the current block as of that step (or a later one), else 0.
+ * Errors: CAI_ERR_TIMEOUT after timeout_ms (not sticky); CAI_ERR_DEVICE if a
+ * kernel reported a failed bounded wait; CAI_ERR_ARG for lag < 0.
+ */
+int cai_poll(cai_ctx* ctx, int32_t lag, int32_t timeout_ms, int32_t* all_done);
+
+/* Device pointers of the state arrays (no copy, no synchronisation). */
+int cai_get_state(cai_ctx* ctx, cai_state_view* out);
+
+/* Synchronous copy of the whole state to caller host buffers (device
+ * synchronise first), and back (checkpoint / resume, teacher forcing). */
+int cai_state_download(cai_ctx* ctx, cai_host_state* dst);
+int cai_state_upload(cai_ctx* ctx, const cai_host_state* src);
+
+/* Asynchronous copy of the committed tokens [B, L] int32 into host memory on
+ * the stream (pinned memory for a truly asynchronous copy). */
+int cai_read_tokens(cai_ctx* ctx, int32_t* host_tokens, void* stream);
+
+/* Time every LM-head launch with CUDA events on its stream (enable = 1) or
+ * stop (0).  cai_get_stats synchronises the events and reports the sum. */
+int cai_profile(cai_ctx* ctx, int32_t enable);
+int cai_get_stats(cai_ctx* ctx, cai_stats* out);
+
+/* Release everything the context owns.  Synchronises the device first.
+ * NULL is a no-op. */
+void cai_free(cai_ctx* ctx);
+
+/* Static string for a status code. */
+const char* cai_strerror(int status);
+
+/*
+ * Testing hook: make the n-th device allocation from now fail (n >= 1), as if
+ * cudaMalloc had returned an error; n = 0 disables.  Process-wide.
+ */
+int cai_test_fail_alloc_after(int32_t n);
+
+/*
+ * Testing hook: cap the number of CTAs of the LM-head kernel for contexts
+ * created from now on (n >= 1), so that small vocabularies still give each
+ * CTA several 128-row tiles; n = 0 restores one CTA per SM.  Process-wide.
+ */
+int cai_test_head_grid_limit(int32_t n);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* CAI_H */

@@ -1,0 +1,282 @@
+"""Python binding of the CAI-dLLM decoding-head library (``libcai.so``).
+
+Argument marshalling only: every step of the decoding head and commit rule
+runs in the library's sm_103a kernels (``csrc/``).  Function names follow the
+C ABI in ``include/cai.h``.  Tensors are passed as PyTorch tensors (their
+``data_ptr``) or raw integer pointers; streams as ``torch.cuda.Stream``, a raw
+handle, or ``None`` for PyTorch's current stream.  A failing status raises
+``CaiError`` carrying the status code.
+
+There is no CPU fallback: the first call into the binding raises
+``ImportError`` when the library is not built (``paper_2608_22646_gb300.build``).
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import numpy as np
+
+_PKG = os.path.dirname(os.path.abspath(__file__))
+LIB_PATH = os.path.join(_PKG, "libcai.so")
+
+CAI_OK = 0
+CAI_ERR_ARG = -1
+CAI_ERR_SHAPE = -2
+CAI_ERR_ORDER = -3
+CAI_ERR_CUDA = -4
+CAI_ERR_TIMEOUT = -5
+CAI_ERR_DEVICE = -6
+CAI_ERR_UNSUPPORTED = -7
+CAI_ERR_NOMEM = -8
+
+CAI_GATING = 1
+CAI_POS_FACTOR = 2
+CAI_FLUSH_ON_EXIT = 4
+CAI_QUARTER_POS = 8
+CAI_QUARTER_BLOCKS = 16
+
+CAI_PRESET_LLADA = 0
+CAI_PRESET_DREAM = 1
+
+CAI_MASK_TOKEN = -1
+CAI_RUNNING, CAI_EXIT_DONE, CAI_EXIT_GRIND, CAI_EXIT_TMAX = 0, 1, 2, 3
+
+# Every symbol include/cai.h declares.
+EXPORTS = ("cai_config_default", "cai_init", "cai_first_step", "cai_denoise_step",
+           "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
+           "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
+           "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit")
+
+
+class CaiError(RuntimeError):
+    def __init__(self, status: int, what: str = ""):
+        self.status = status
+        super().__init__(f"{what}: {status} ({cai_strerror(status)})")
+
+
+class cai_config(ctypes.Structure):
+    _fields_ = [
+        ("B", ctypes.c_int32), ("P", ctypes.c_int32), ("H", ctypes.c_int32),
+        ("V", ctypes.c_int32), ("T", ctypes.c_int32), ("n_blocks", ctypes.c_int32),
+        ("theta_s", ctypes.c_double), ("theta_e1", ctypes.c_double),
+        ("theta_e_step", ctypes.c_double), ("theta_e_min", ctypes.c_double),
+        ("warmup_pct", ctypes.c_int32), ("K", ctypes.c_int32),
+        ("theta_fb", ctypes.c_double), ("clip_lo", ctypes.c_double), ("clip_hi", ctypes.c_double),
+        ("eta_bar", ctypes.c_double), ("eta_mode", ctypes.c_int32), ("flags", ctypes.c_uint32),
+    ]
+
+
+_STATE_FIELDS = ("tok", "conf", "s0", "budget", "cstep", "cand", "ell", "eta", "exit_reason",
+                 "exit_step", "unresolved", "m_hist")
+
+
+class cai_state_view(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in _STATE_FIELDS]
+
+
+class cai_host_state(ctypes.Structure):
+    _fields_ = [(n, ctypes.c_void_p) for n in _STATE_FIELDS] + [
+        ("blk", ctypes.c_int32), ("t_next", ctypes.c_int32)]
+
+
+class cai_stats(ctypes.Structure):
+    _fields_ = [("steps", ctypes.c_int64), ("launches", ctypes.c_int64),
+                ("head_launches", ctypes.c_int64), ("head_ms", ctypes.c_double),
+                ("head_profiled", ctypes.c_int64), ("grid", ctypes.c_int32),
+                ("stages", ctypes.c_int32), ("n_max", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+
+
+def _load():
+    if not os.path.exists(LIB_PATH):
+        raise ImportError(f"libcai.so is not built ({LIB_PATH}); run paper_2608_22646_gb300.build")
+    lib = ctypes.CDLL(LIB_PATH)
+    vp, i32 = ctypes.c_void_p, ctypes.c_int32
+    sig = {
+        "cai_config_default": (ctypes.c_int, [ctypes.POINTER(cai_config), i32, i32, i32, i32, i32, i32, i32]),
+        "cai_init": (ctypes.c_int, [ctypes.POINTER(cai_config), vp, vp, ctypes.POINTER(vp)]),
+        "cai_first_step": (ctypes.c_int, [vp, vp, vp]),
+        "cai_denoise_step": (ctypes.c_int, [vp, vp, vp]),
+        "cai_block_advance": (ctypes.c_int, [vp, vp]),
+        "cai_reset": (ctypes.c_int, [vp, vp]),
+        "cai_poll": (ctypes.c_int, [vp, i32, i32, ctypes.POINTER(i32)]),
+        "cai_get_state": (ctypes.c_int, [vp, ctypes.POINTER(cai_state_view)]),
+        "cai_state_download": (ctypes.c_int, [vp, ctypes.POINTER(cai_host_state)]),
+        "cai_state_upload": (ctypes.c_int, [vp, ctypes.POINTER(cai_host_state)]),
+        "cai_read_tokens": (ctypes.c_int, [vp, vp, vp]),
+        "cai_profile": (ctypes.c_int, [vp, i32]),
+        "cai_get_stats": (ctypes.c_int, [vp, ctypes.POINTER(cai_stats)]),
+        "cai_free": (None, [vp]),
+        "cai_strerror": (ctypes.c_char_p, [ctypes.c_int]),
+        "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
+        "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
+    }
+    for name, (res, args) in sig.items():
+        f = getattr(lib, name)
+        f.restype = res
+        f.argtypes = args
+    return lib
+
+
+_lib = None
+
+
+def lib():
+    global _lib
+    if _lib is None:
+        _lib = _load()
+    return _lib
+
+
+def _check(status: int, what: str):
+    if status != CAI_OK:
+        raise CaiError(status, what)
+
+
+def _ptr(x) -> int | None:
+    if x is None:
+        return None
+    if isinstance(x, int):
+        return x
+    if isinstance(x, np.ndarray):
+        return x.ctypes.data
+    return x.data_ptr()
+
+
+def _stream(s) -> int | None:
+    if s is None:
+        import torch
+        if torch.cuda.is_available():
+            return torch.cuda.current_stream().cuda_stream
+        return None
+    if isinstance(s, int):
+        return s
+    return s.cuda_stream
+
+
+def cai_strerror(status: int) -> str:
+    return lib().cai_strerror(status).decode()
+
+
+def cai_config_default(preset: int, B: int, P: int, H: int, V: int, T: int, n_blocks: int) -> cai_config:
+    c = cai_config()
+    _check(lib().cai_config_default(ctypes.byref(c), preset, B, P, H, V, T, n_blocks),
+           "cai_config_default")
+    return c
+
+
+class Ctx:
+    """Owning handle of a ``cai_ctx*``; also keeps the sizes for the copies."""
+
+    def __init__(self, handle: int, cfg: cai_config, W):
+        self.handle = handle
+        self.cfg = cfg
+        self._W = W  # the weight must outlive the context
+
+    @property
+    def L(self) -> int:
+        return self.cfg.n_blocks * self.cfg.P
+
+
+def cai_init(cfg: cai_config, W, stream=None) -> Ctx:
+    h = ctypes.c_void_p()
+    _check(lib().cai_init(ctypes.byref(cfg), _ptr(W), _stream(stream), ctypes.byref(h)), "cai_init")
+    return Ctx(h.value, cfg, W)
+
+
+def cai_first_step(ctx: Ctx, hidden, stream=None) -> None:
+    _check(lib().cai_first_step(ctx.handle, _ptr(hidden), _stream(stream)), "cai_first_step")
+
+
+def cai_denoise_step(ctx: Ctx, hidden, stream=None) -> None:
+    _check(lib().cai_denoise_step(ctx.handle, _ptr(hidden), _stream(stream)), "cai_denoise_step")
+
+
+def cai_block_advance(ctx: Ctx, stream=None) -> None:
+    _check(lib().cai_block_advance(ctx.handle, _stream(stream)), "cai_block_advance")
+
+
+def cai_reset(ctx: Ctx, stream=None) -> None:
+    _check(lib().cai_reset(ctx.handle, _stream(stream)), "cai_reset")
+
+
+def cai_poll(ctx: Ctx, lag: int = 0, timeout_ms: int = 10000) -> bool:
+    done = ctypes.c_int32(0)
+    _check(lib().cai_poll(ctx.handle, lag, timeout_ms, ctypes.byref(done)), "cai_poll")
+    return bool(done.value)
+
+
+def cai_get_state(ctx: Ctx) -> dict:
+    v = cai_state_view()
+    _check(lib().cai_get_state(ctx.handle, ctypes.byref(v)), "cai_get_state")
+    return {n: getattr(v, n) for n in _STATE_FIELDS}
+
+
+def _host_arrays(ctx: Ctx) -> dict:
+    c = ctx.cfg
+    B, L, nb = c.B, ctx.L, c.n_blocks
+    return {
+        "tok": np.zeros((B, L), np.int32), "conf": np.zeros((B, L), np.float32),
+        "s0": np.zeros((B, L), np.float32), "budget": np.zeros((B, L), np.uint8),
+        "cstep": np.zeros((B, L), np.int16), "cand": np.zeros((B, L), np.int32),
+        "ell": np.zeros(B, np.int32), "eta": np.zeros(B, np.int32),
+        "exit_reason": np.zeros((B, nb), np.int32), "exit_step": np.zeros((B, nb), np.int32),
+        "unresolved": np.zeros((B, nb), np.int32), "m_hist": np.zeros((nb, c.T), np.int32),
+    }
+
+
+def cai_state_download(ctx: Ctx) -> dict:
+    arrs = _host_arrays(ctx)
+    hs = cai_host_state(**{n: arrs[n].ctypes.data for n in _STATE_FIELDS})
+    _check(lib().cai_state_download(ctx.handle, ctypes.byref(hs)), "cai_state_download")
+    arrs["blk"] = hs.blk
+    arrs["t_next"] = hs.t_next
+    return arrs
+
+
+def cai_state_upload(ctx: Ctx, state: dict) -> None:
+    ref = _host_arrays(ctx)
+    keep = {}
+    kw = {}
+    for n in _STATE_FIELDS:
+        if n in state and state[n] is not None:
+            a = np.ascontiguousarray(state[n], dtype=ref[n].dtype).reshape(ref[n].shape)
+            keep[n] = a
+            kw[n] = a.ctypes.data
+    hs = cai_host_state(**kw, blk=int(state["blk"]), t_next=int(state["t_next"]))
+    _check(lib().cai_state_upload(ctx.handle, ctypes.byref(hs)), "cai_state_upload")
+
+
+def cai_read_tokens(ctx: Ctx, host_tokens, stream=None) -> None:
+    _check(lib().cai_read_tokens(ctx.handle, _ptr(host_tokens), _stream(stream)), "cai_read_tokens")
+
+
+def cai_profile(ctx: Ctx, enable: bool) -> None:
+    _check(lib().cai_profile(ctx.handle, 1 if enable else 0), "cai_profile")
+
+
+def cai_get_stats(ctx: Ctx) -> dict:
+    s = cai_stats()
+    _check(lib().cai_get_stats(ctx.handle, ctypes.byref(s)), "cai_get_stats")
+    return {n: getattr(s, n) for n, _ in cai_stats._fields_}
+
+
+def cai_free(ctx: Ctx) -> None:
+    if ctx.handle:
+        lib().cai_free(ctx.handle)
+        ctx.handle = 0
+
+
+def cai_test_fail_alloc_after(n: int) -> None:
+    _check(lib().cai_test_fail_alloc_after(n), "cai_test_fail_alloc_after")
+
+
+def cai_test_head_grid_limit(n: int) -> None:
+    _check(lib().cai_test_head_grid_limit(n), "cai_test_head_grid_limit")
+
+
+def config_from_dict(d: dict) -> cai_config:
+    c = cai_config()
+    for k, v in d.items():
+        setattr(c, k, v)
+    return c

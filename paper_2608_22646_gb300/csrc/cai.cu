@@ -1,0 +1,694 @@
+// Host side of the C ABI declared in include/cai.h: context ownership, argument
+// validation, TMA descriptor set-up, launch sequencing of one denoising step
+// (gather -> LM head + softmax -> merge + commit), the host-side threshold
+// schedule (Boxes 3, 4 and 6 of arXiv 2608.22646, in double), polling and
+// state transfer.
+#include <cuda.h>
+#include <cuda_runtime.h>
+
+#include <atomic>
+#include <chrono>
+#include <cmath>
+#include <cstdio>
+#include <cstring>
+#include <new>
+#include <thread>
+#include <vector>
+
+#include "cai.h"
+#include "step_kernels.cuh"
+
+using namespace cai;
+
+namespace {
+
+std::atomic<int> g_fail_alloc_after{0};
+std::atomic<int> g_head_grid_limit{0};
+
+int dev_alloc(void** p, size_t bytes) {
+  *p = nullptr;
+  int n = g_fail_alloc_after.load();
+  if (n > 0) {
+    if (n == 1) {
+      g_fail_alloc_after.store(0);
+      return CAI_ERR_NOMEM;
+    }
+    g_fail_alloc_after.store(n - 1);
+  }
+  if (bytes == 0) bytes = 16;
+  cudaError_t e = cudaMalloc(p, bytes);
+  if (e == cudaErrorMemoryAllocation) {
+    cudaGetLastError();
+    return CAI_ERR_NOMEM;
+  }
+  if (e != cudaSuccess) return CAI_ERR_CUDA;
+  return CAI_OK;
+}
+
+typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t, void*,
+                                  const cuuint64_t*, const cuuint64_t*, const cuuint32_t*,
+                                  const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
+                                  CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
+
+EncodeTiledFn get_encoder() {
+  static EncodeTiledFn fn = nullptr;
+  if (fn) return fn;
+  void* ptr = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
+                                       &q) != cudaSuccess ||
+      q != cudaDriverEntryPointSuccess)
+    return nullptr;
+  fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  return fn;
+}
+
+// Row-major bf16 matrix [rows, cols] with a box of box_rows x 64 columns and
+// the 128-byte swizzle that the MMA descriptors expect.
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+  EncodeTiledFn enc = get_encoder();
+  if (!enc) return false;
+  cuuint64_t dims[2] = {cols, rows};
+  cuuint64_t strides[1] = {cols * 2};
+  cuuint32_t box[2] = {static_cast<cuuint32_t>(kBlockK), box_rows};
+  cuuint32_t estr[2] = {1, 1};
+  return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
+}
+
+int round_up(int x, int m) { return (x + m - 1) / m * m; }
+int next_pow2(int x) {
+  int p = 1;
+  while (p < x) p <<= 1;
+  return p;
+}
+
+bool is_device_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
+}
+
+}  // namespace
+
+struct cai_ctx {
+  cai_config cfg{};
+  int L = 0, BP = 0, rows_cap = 0;
+  const void* W = nullptr;
+  void* W_owned = nullptr;
+  StateArrays st{};
+  int* list = nullptr;
+  int* row_of = nullptr;
+  int* d_M = nullptr;
+  unsigned* ticket = nullptr;
+  uint32_t* err = nullptr;
+  __nv_bfloat16* hc = nullptr;
+  float4* part = nullptr;
+  void* hidden_stage = nullptr;
+  HostFlag* hf_host = nullptr;
+  HostFlag* hf_dev = nullptr;
+  CUtensorMap tm_w128{}, tm_w64{}, tm_h{};
+  int G = 0, n_stages = 0, n_max = 0, acc_stride = 0, tmem_cols = 0, b_stage_bytes = 0;
+  size_t head_smem = 0;
+  int blk = 0, t_next = 0;
+  int64_t last_step_id = -1;
+  bool block_done_seen = false;
+  int sticky = CAI_OK;
+  cai_stats stats{};
+  bool profiling = false;
+  std::vector<cudaEvent_t> ev_pool;  // pairs (start, stop)
+  size_t ev_used = 0;                // events recorded since the last stats call
+  std::vector<void*> allocs;
+};
+
+namespace {
+
+int fail(cai_ctx* c, int code) {
+  if (c && (code == CAI_ERR_CUDA || code == CAI_ERR_DEVICE) && c->sticky == CAI_OK) c->sticky = code;
+  return code;
+}
+
+int check_launch(cai_ctx* c) {
+  cudaError_t e = cudaGetLastError();
+  if (e != cudaSuccess) {
+    fprintf(stderr, "cai: CUDA error %s\n", cudaGetErrorString(e));
+    return fail(c, CAI_ERR_CUDA);
+  }
+  return CAI_OK;
+}
+
+int validate(const cai_config* c) {
+  if (c->B < 1 || c->P < 1 || c->P > kMaxP || c->H < 64 || c->H > 16384 || (c->H % 64) != 0 ||
+      c->V < 64 || c->T < 1 || c->T > 32767 || c->n_blocks < 1 ||
+      static_cast<int64_t>(c->B) * c->P > 65536 ||
+      static_cast<int64_t>(c->n_blocks) * c->P > (1 << 24))
+    return CAI_ERR_SHAPE;
+  if (c->warmup_pct < 0 || c->warmup_pct > 100 || c->K < 1 || (c->eta_mode != 0 && c->eta_mode != 1) ||
+      !(c->clip_lo <= c->clip_hi) || (c->flags & ~31u) != 0)
+    return CAI_ERR_ARG;
+  return CAI_OK;
+}
+
+int alloc_into(cai_ctx* c, void** dst, size_t bytes) {
+  int r = dev_alloc(dst, bytes);
+  if (r == CAI_OK) c->allocs.push_back(*dst);
+  return r;
+}
+
+void release(cai_ctx* c) {
+  for (void* p : c->allocs) cudaFree(p);
+  c->allocs.clear();
+  if (c->hf_host) cudaFreeHost(c->hf_host);
+  c->hf_host = nullptr;
+  for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
+  c->ev_pool.clear();
+}
+
+// ---- threshold schedule (Boxes 3, 4, 6), double precision on the host ----
+
+double theta_e_of(const cai_config& c, int b1) {
+  int be = b1;
+  if (c.flags & CAI_QUARTER_BLOCKS) be = 1 + (4 * (b1 - 1)) / c.n_blocks;
+  double th = c.theta_e1 - c.theta_e_step * static_cast<double>(be - 1);
+  return th < c.theta_e_min ? c.theta_e_min : th;
+}
+
+double theta_block_of(const cai_config& c, int b1, int t) {
+  if (100 * t < c.warmup_pct * c.T) return c.theta_s;
+  const double wT = static_cast<double>(c.warmup_pct) * c.T / 100.0;
+  const double u = (t - wT) / (c.T - wT);
+  const double te = theta_e_of(c, b1);
+  return te + 0.5 * (c.theta_s - te) * (1.0 + std::cos(M_PI * u));
+}
+
+double pos_factor_of(const cai_config& c, int p) {
+  if (!(c.flags & CAI_POS_FACTOR)) return 1.0;
+  int q1 = 16, q2 = 32, q3 = 48;
+  if (c.flags & CAI_QUARTER_POS) {
+    q1 = c.P / 4;
+    q2 = c.P / 2;
+    q3 = 3 * c.P / 4;
+  }
+  return p < q1 ? 0.80 : p < q2 ? 0.90 : p < q3 ? 1.05 : 1.10;
+}
+
+int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  const cai_config& cfg = c->cfg;
+  const void* hid = hidden;
+  if (!is_device_ptr(hidden)) {
+    if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
+                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
+      return fail(c, CAI_ERR_CUDA);
+    hid = c->hidden_stage;
+  }
+  const int t = c->t_next;
+  const int64_t step_id = c->last_step_id + 1;
+
+  GatherParams gp{};
+  gp.hidden = static_cast<const __nv_bfloat16*>(hid);
+  gp.hc = c->hc;
+  gp.list = c->list;
+  gp.row_of = c->row_of;
+  gp.d_M = c->d_M;
+  gp.m_hist = c->st.m_hist;
+  gp.ell = c->st.ell;
+  gp.hist_idx = c->blk * cfg.T + t;
+  gp.B = cfg.B;
+  gp.BP = c->BP;
+  gp.H = cfg.H;
+  gp.first = first ? 1 : 0;
+  const int g_grid = c->rows_cap / kGatherRowsPerCta;
+  gather_rows_kernel<<<g_grid, kGatherThreads, 0, stream>>>(gp);
+  c->stats.launches++;
+
+  HeadParams hp{};
+  hp.d_M = c->d_M;
+  hp.part = c->part;
+  hp.err = c->err;
+  hp.V = cfg.V;
+  hp.H = cfg.H;
+  hp.units = (cfg.V + kUnitRows - 1) / kUnitRows;
+  hp.n_stages = c->n_stages;
+  hp.b_stage_bytes = c->b_stage_bytes;
+  hp.acc_stride = c->acc_stride;
+  hp.tmem_cols = c->tmem_cols;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (c->profiling) {
+    if (c->ev_used + 2 > c->ev_pool.size()) {
+      for (int k = 0; k < 2; ++k) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+        c->ev_pool.push_back(e);
+      }
+    }
+    e0 = c->ev_pool[c->ev_used];
+    e1 = c->ev_pool[c->ev_used + 1];
+    c->ev_used += 2;
+    cudaEventRecord(e0, stream);
+  }
+  lm_head_softmax_kernel<<<c->G, kHeadThreads, c->head_smem, stream>>>(c->tm_w128, c->tm_w64,
+                                                                       c->tm_h, hp);
+  if (c->profiling) cudaEventRecord(e1, stream);
+  c->stats.launches++;
+  c->stats.head_launches++;
+
+  CommitParams cp{};
+  cp.part = c->part;
+  cp.n_part = 4 * c->G;
+  cp.st = c->st;
+  cp.list = c->list;
+  cp.row_of = c->row_of;
+  cp.d_M = c->d_M;
+  cp.ticket = c->ticket;
+  cp.hf = c->hf_dev;
+  cp.err = c->err;
+  cp.B = cfg.B;
+  cp.P = cfg.P;
+  cp.L = c->L;
+  cp.n_blocks = cfg.n_blocks;
+  cp.T = cfg.T;
+  cp.blk = c->blk;
+  cp.t = t;
+  cp.step_id = static_cast<int>(step_id);
+  cp.K = cfg.K;
+  cp.eta_mode = cfg.eta_mode;
+  cp.eta_bar = static_cast<float>(cfg.eta_bar);
+  cp.theta_fb = static_cast<float>(cfg.theta_fb);
+  cp.budget_half = (cfg.flags & CAI_QUARTER_POS) ? cfg.P / 2 : 32;
+  cp.budget_late = (cfg.flags & CAI_QUARTER_POS) ? 3 * cfg.P / 4 : 48;
+  cp.flags = cfg.flags;
+  const double tb = theta_block_of(cfg, c->blk + 1, t);
+  for (int p = 0; p < cfg.P; ++p) {
+    double th = tb * pos_factor_of(cfg, p);
+    th = th < cfg.clip_lo ? cfg.clip_lo : th;
+    th = th > cfg.clip_hi ? cfg.clip_hi : th;
+    cp.theta_tab[p] = static_cast<float>(th);
+  }
+  merge_commit_kernel<<<cfg.B, kCommitThreads, 0, stream>>>(cp);
+  c->stats.launches++;
+  c->stats.steps++;
+  int r = check_launch(c);
+  if (r != CAI_OK) return r;
+  c->last_step_id = step_id;
+  c->t_next = t + 1;
+  return CAI_OK;
+}
+
+}  // namespace
+
+extern "C" {
+
+int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, int32_t H, int32_t V,
+                       int32_t T, int32_t n_blocks) {
+  if (!cfg || (preset != CAI_PRESET_LLADA && preset != CAI_PRESET_DREAM)) return CAI_ERR_ARG;
+  cai_config c{};
+  c.B = B;
+  c.P = P;
+  c.H = H;
+  c.V = V;
+  c.T = T;
+  c.n_blocks = n_blocks;
+  c.theta_s = 0.90;
+  c.theta_e1 = 0.70;
+  c.theta_e_step = 0.10;
+  c.theta_e_min = 0.40;
+  c.warmup_pct = 15;
+  c.K = 4;
+  c.theta_fb = 0.40;
+  c.clip_lo = 0.20;
+  c.clip_hi = 0.98;
+  c.eta_bar = 1.5;
+  c.eta_mode = 0;
+  c.flags = CAI_POS_FACTOR | (preset == CAI_PRESET_LLADA ? CAI_GATING : 0u);
+  *cfg = c;
+  return CAI_OK;
+}
+
+int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) {
+  if (!cfg || !W || !out) return CAI_ERR_ARG;
+  *out = nullptr;
+  int r = validate(cfg);
+  if (r != CAI_OK) return r;
+  if (reinterpret_cast<uintptr_t>(W) % 16 != 0) return CAI_ERR_ARG;
+
+  int dev = 0, major = 0, minor = 0, sms = 0, smem_optin = 0;
+  if (cudaGetDevice(&dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&major, cudaDevAttrComputeCapabilityMajor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&minor, cudaDevAttrComputeCapabilityMinor, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&sms, cudaDevAttrMultiProcessorCount, dev) != cudaSuccess ||
+      cudaDeviceGetAttribute(&smem_optin, cudaDevAttrMaxSharedMemoryPerBlockOptin, dev) !=
+          cudaSuccess) {
+    cudaGetLastError();
+    return CAI_ERR_CUDA;
+  }
+  if (major != 10 || minor != 3) return CAI_ERR_UNSUPPORTED;
+
+  cai_ctx* c = new (std::nothrow) cai_ctx();
+  if (!c) return CAI_ERR_NOMEM;
+  c->cfg = *cfg;
+  c->L = cfg->n_blocks * cfg->P;
+  c->BP = cfg->B * cfg->P;
+  c->rows_cap = round_up(c->BP, 16);
+
+  // LM-head launch shape: N chunk, tensor-memory columns, pipeline depth.
+  c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
+  c->acc_stride = round_up(c->n_max, 32);
+  c->tmem_cols = next_pow2(2 * c->acc_stride < 32 ? 32 : 2 * c->acc_stride);
+  c->b_stage_bytes = c->n_max * 128;
+  int stages = 12;
+  while (stages > 2 && head_smem_bytes(stages, c->b_stage_bytes, c->acc_stride) >
+                           static_cast<size_t>(smem_optin))
+    --stages;
+  c->n_stages = stages;
+  c->head_smem = head_smem_bytes(stages, c->b_stage_bytes, c->acc_stride);
+  const int units = (cfg->V + kUnitRows - 1) / kUnitRows;
+  c->G = units < sms ? units : sms;
+  const int glim = g_head_grid_limit.load();
+  if (glim > 0 && c->G > glim) c->G = glim;
+
+  const size_t BL = static_cast<size_t>(cfg->B) * c->L;
+  const size_t BN = static_cast<size_t>(cfg->B) * cfg->n_blocks;
+  void* p;
+#define CAI_ALLOC(field, type, count)                                  \
+  if ((r = alloc_into(c, &p, sizeof(type) * (count))) != CAI_OK) {    \
+    release(c);                                                        \
+    delete c;                                                          \
+    return r;                                                          \
+  }                                                                    \
+  field = static_cast<type*>(p);
+  CAI_ALLOC(c->st.tok, int, BL)
+  CAI_ALLOC(c->st.conf, float, BL)
+  CAI_ALLOC(c->st.s0, float, BL)
+  CAI_ALLOC(c->st.budget, uint8_t, BL)
+  CAI_ALLOC(c->st.cstep, int16_t, BL)
+  CAI_ALLOC(c->st.cand, int, BL)
+  CAI_ALLOC(c->st.ell, int, cfg->B)
+  CAI_ALLOC(c->st.eta, int, cfg->B)
+  CAI_ALLOC(c->st.exit_reason, int, BN)
+  CAI_ALLOC(c->st.exit_step, int, BN)
+  CAI_ALLOC(c->st.unresolved, int, BN)
+  CAI_ALLOC(c->st.m_hist, int, static_cast<size_t>(cfg->n_blocks) * cfg->T)
+  CAI_ALLOC(c->list, int, c->BP)
+  CAI_ALLOC(c->row_of, int, c->BP)
+  CAI_ALLOC(c->d_M, int, 1)
+  CAI_ALLOC(c->ticket, unsigned, 1)
+  CAI_ALLOC(c->err, uint32_t, 1)
+  CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
+  CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * 4 * c->G)
+  CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
+  if (!is_device_ptr(W)) {
+    CAI_ALLOC(c->W_owned, uint8_t, static_cast<size_t>(cfg->V) * cfg->H * 2)
+    if (cudaMemcpy(c->W_owned, W, static_cast<size_t>(cfg->V) * cfg->H * 2,
+                   cudaMemcpyHostToDevice) != cudaSuccess) {
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    c->W = c->W_owned;
+  } else {
+    c->W = W;
+  }
+#undef CAI_ALLOC
+  if (cudaHostAlloc(reinterpret_cast<void**>(&c->hf_host), sizeof(HostFlag), cudaHostAllocMapped) !=
+          cudaSuccess ||
+      cudaHostGetDevicePointer(reinterpret_cast<void**>(&c->hf_dev), c->hf_host, 0) != cudaSuccess) {
+    cudaGetLastError();
+    release(c);
+    delete c;
+    return CAI_ERR_NOMEM;
+  }
+  std::memset(c->hf_host, 0, sizeof(HostFlag));
+  reinterpret_cast<volatile HostFlag*>(c->hf_host)->seq = -1;
+  // A 128-row tile is only used when a CTA owns two 64-row units, so V >= 128.
+  if (!make_map(&c->tm_w128, c->W, cfg->V, cfg->H, cfg->V >= 128 ? 128 : 64) ||
+      !make_map(&c->tm_w64, c->W, cfg->V, cfg->H, 64) ||
+      !make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB)) {
+    release(c);
+    delete c;
+    return CAI_ERR_CUDA;
+  }
+  if (cudaFuncSetAttribute(lm_head_softmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                           static_cast<int>(c->head_smem)) != cudaSuccess) {
+    cudaGetLastError();
+    release(c);
+    delete c;
+    return CAI_ERR_CUDA;
+  }
+  c->stats.grid = c->G;
+  c->stats.stages = c->n_stages;
+  c->stats.n_max = c->n_max;
+  r = cai_reset(c, stream);
+  if (r != CAI_OK) {
+    release(c);
+    delete c;
+    return r;
+  }
+  *out = c;
+  return CAI_OK;
+}
+
+int cai_reset(cai_ctx* c, void* stream_v) {
+  if (!c) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  cudaStream_t s = static_cast<cudaStream_t>(stream_v);
+  const cai_config& cfg = c->cfg;
+  const size_t BL = static_cast<size_t>(cfg.B) * c->L;
+  const size_t BN = static_cast<size_t>(cfg.B) * cfg.n_blocks;
+  bool ok = cudaMemsetAsync(c->st.tok, 0xFF, BL * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.conf, 0, BL * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.s0, 0, BL * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.budget, 0, BL, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.cstep, 0xFF, BL * 2, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.cand, 0xFF, BL * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.ell, 0, cfg.B * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.eta, 0, cfg.B * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.exit_reason, 0, BN * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.exit_step, 0xFF, BN * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.unresolved, 0, BN * 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.m_hist, 0, static_cast<size_t>(cfg.n_blocks) * cfg.T * 4, s) ==
+                cudaSuccess &&
+            cudaMemsetAsync(c->ticket, 0, 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->err, 0, 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->d_M, 0, 4, s) == cudaSuccess;
+  if (!ok) return fail(c, CAI_ERR_CUDA);
+  // Step ids keep increasing across resets, so a host-flag write still in
+  // flight from the previous generation never satisfies a poll of this one.
+  c->blk = 0;
+  c->t_next = 0;
+  c->block_done_seen = false;
+  return CAI_OK;
+}
+
+int cai_first_step(cai_ctx* c, const void* hidden, void* stream) {
+  if (!c || !hidden) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (reinterpret_cast<uintptr_t>(hidden) % 16 != 0) return CAI_ERR_ARG;
+  if (c->t_next != 0) return CAI_ERR_ORDER;
+  c->block_done_seen = false;
+  return step(c, hidden, stream, true);
+}
+
+int cai_denoise_step(cai_ctx* c, const void* hidden, void* stream) {
+  if (!c || !hidden) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (reinterpret_cast<uintptr_t>(hidden) % 16 != 0) return CAI_ERR_ARG;
+  if (c->t_next < 1 || c->t_next >= c->cfg.T || c->block_done_seen) return CAI_ERR_ORDER;
+  return step(c, hidden, stream, false);
+}
+
+int cai_block_advance(cai_ctx* c, void* stream) {
+  (void)stream;
+  if (!c) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (c->t_next < 1 || c->blk + 1 >= c->cfg.n_blocks) return CAI_ERR_ORDER;
+  c->blk += 1;
+  c->t_next = 0;
+  c->block_done_seen = false;
+  return CAI_OK;
+}
+
+int cai_poll(cai_ctx* c, int32_t lag, int32_t timeout_ms, int32_t* all_done) {
+  if (!c || !all_done || lag < 0) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  *all_done = 0;
+  const int64_t target = c->last_step_id - lag;
+  if (target < 0) return CAI_OK;
+  volatile HostFlag* hf = c->hf_host;
+  const auto t0 = std::chrono::steady_clock::now();
+  for (uint32_t it = 0;; ++it) {
+    const int32_t seq = hf->seq;
+    if (seq >= target) break;
+    if (hf->err) return fail(c, CAI_ERR_DEVICE);
+    if ((it & 255u) == 255u) {
+      const auto dt = std::chrono::steady_clock::now() - t0;
+      if (std::chrono::duration_cast<std::chrono::milliseconds>(dt).count() >= timeout_ms)
+        return CAI_ERR_TIMEOUT;
+      std::this_thread::yield();
+    }
+  }
+  std::atomic_thread_fence(std::memory_order_acquire);
+  if (hf->err) return fail(c, CAI_ERR_DEVICE);
+  if (hf->blk == c->blk && hf->all_done) {
+    *all_done = 1;
+    c->block_done_seen = true;
+  }
+  return CAI_OK;
+}
+
+int cai_get_state(cai_ctx* c, cai_state_view* v) {
+  if (!c || !v) return CAI_ERR_ARG;
+  v->tok = c->st.tok;
+  v->conf = c->st.conf;
+  v->s0 = c->st.s0;
+  v->budget = c->st.budget;
+  v->cstep = c->st.cstep;
+  v->cand = c->st.cand;
+  v->ell = c->st.ell;
+  v->eta = c->st.eta;
+  v->exit_reason = c->st.exit_reason;
+  v->exit_step = c->st.exit_step;
+  v->unresolved = c->st.unresolved;
+  v->m_hist = c->st.m_hist;
+  return CAI_OK;
+}
+
+static int transfer(cai_ctx* c, const cai_host_state* h, bool down) {
+  const cai_config& cfg = c->cfg;
+  const size_t BL = static_cast<size_t>(cfg.B) * c->L;
+  const size_t BN = static_cast<size_t>(cfg.B) * cfg.n_blocks;
+  struct F {
+    void* host;
+    void* dev;
+    size_t bytes;
+  } f[] = {
+      {h->tok, c->st.tok, BL * 4},         {h->conf, c->st.conf, BL * 4},
+      {h->s0, c->st.s0, BL * 4},           {h->budget, c->st.budget, BL},
+      {h->cstep, c->st.cstep, BL * 2},     {h->cand, c->st.cand, BL * 4},
+      {h->ell, c->st.ell, cfg.B * 4u},     {h->eta, c->st.eta, cfg.B * 4u},
+      {h->exit_reason, c->st.exit_reason, BN * 4}, {h->exit_step, c->st.exit_step, BN * 4},
+      {h->unresolved, c->st.unresolved, BN * 4},
+      {h->m_hist, c->st.m_hist, static_cast<size_t>(cfg.n_blocks) * cfg.T * 4},
+  };
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+  for (const F& x : f) {
+    if (!x.host) continue;
+    cudaError_t e = down ? cudaMemcpy(x.host, x.dev, x.bytes, cudaMemcpyDeviceToHost)
+                         : cudaMemcpy(x.dev, x.host, x.bytes, cudaMemcpyHostToDevice);
+    if (e != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+  }
+  return CAI_OK;
+}
+
+int cai_state_download(cai_ctx* c, cai_host_state* dst) {
+  if (!c || !dst) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  int r = transfer(c, dst, true);
+  if (r != CAI_OK) return r;
+  dst->blk = c->blk;
+  dst->t_next = c->t_next;
+  if (reinterpret_cast<volatile HostFlag*>(c->hf_host)->err) return fail(c, CAI_ERR_DEVICE);
+  return CAI_OK;
+}
+
+int cai_state_upload(cai_ctx* c, const cai_host_state* src) {
+  if (!c || !src) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (src->blk < 0 || src->blk >= c->cfg.n_blocks || src->t_next < 0 || src->t_next > c->cfg.T)
+    return CAI_ERR_ARG;
+  int r = transfer(c, src, false);
+  if (r != CAI_OK) return r;
+  c->blk = src->blk;
+  c->t_next = src->t_next;
+  c->block_done_seen = false;
+  ListParams lp{};
+  lp.tok = c->st.tok;
+  lp.exit_reason = c->st.exit_reason;
+  lp.list = c->list;
+  lp.row_of = c->row_of;
+  lp.d_M = c->d_M;
+  lp.B = c->cfg.B;
+  lp.P = c->cfg.P;
+  lp.L = c->L;
+  lp.n_blocks = c->cfg.n_blocks;
+  lp.blk = c->blk;
+  rebuild_list_kernel<<<1, kCommitThreads>>>(lp);
+  c->stats.launches++;
+  r = check_launch(c);
+  if (r != CAI_OK) return r;
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+  return CAI_OK;
+}
+
+int cai_read_tokens(cai_ctx* c, int32_t* host_tokens, void* stream) {
+  if (!c || !host_tokens) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (cudaMemcpyAsync(host_tokens, c->st.tok, static_cast<size_t>(c->cfg.B) * c->L * 4,
+                      cudaMemcpyDeviceToHost, static_cast<cudaStream_t>(stream)) != cudaSuccess)
+    return fail(c, CAI_ERR_CUDA);
+  return CAI_OK;
+}
+
+int cai_profile(cai_ctx* c, int32_t enable) {
+  if (!c) return CAI_ERR_ARG;
+  c->profiling = enable != 0;
+  return CAI_OK;
+}
+
+int cai_get_stats(cai_ctx* c, cai_stats* out) {
+  if (!c || !out) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  double ms = 0.0;
+  for (size_t i = 0; i < c->ev_used; i += 2) {
+    if (cudaEventSynchronize(c->ev_pool[i + 1]) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+    float m = 0.f;
+    if (cudaEventElapsedTime(&m, c->ev_pool[i], c->ev_pool[i + 1]) != cudaSuccess)
+      return fail(c, CAI_ERR_CUDA);
+    ms += m;
+  }
+  c->stats.head_ms += ms;
+  c->stats.head_profiled += static_cast<int64_t>(c->ev_used / 2);
+  c->ev_used = 0;
+  *out = c->stats;
+  return CAI_OK;
+}
+
+void cai_free(cai_ctx* c) {
+  if (!c) return;
+  cudaDeviceSynchronize();
+  release(c);
+  delete c;
+}
+
+const char* cai_strerror(int s) {
+  switch (s) {
+    case CAI_OK: return "ok";
+    case CAI_ERR_ARG: return "invalid argument";
+    case CAI_ERR_SHAPE: return "unsupported shape";
+    case CAI_ERR_ORDER: return "call out of order";
+    case CAI_ERR_CUDA: return "CUDA runtime error";
+    case CAI_ERR_TIMEOUT: return "timed out waiting for the device";
+    case CAI_ERR_DEVICE: return "a kernel gave up a bounded wait";
+    case CAI_ERR_UNSUPPORTED: return "device is not compute capability 10.3";
+    case CAI_ERR_NOMEM: return "out of memory";
+    default: return "unknown status";
+  }
+}
+
+int cai_test_head_grid_limit(int32_t n) {
+  if (n < 0) return CAI_ERR_ARG;
+  g_head_grid_limit.store(n);
+  return CAI_OK;
+}
+
+int cai_test_fail_alloc_after(int32_t n) {
+  if (n < 0) return CAI_ERR_ARG;
+  g_fail_alloc_after.store(n);
+  return CAI_OK;
+}
+
+}  // extern "C"

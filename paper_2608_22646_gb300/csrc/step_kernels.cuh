@@ -1,0 +1,311 @@
+// The two light kernels around the LM head in one denoising step:
+//   gather_rows_kernel    copies the hidden rows of the step's masked
+//                         positions into the compact [rows_cap, H] operand;
+//   merge_commit_kernel   merges the per-CTA softmax partials into c_i and the
+//                         argmax, then runs the commit rule of Algorithm 1
+//                         (arXiv 2608.22646) for one sequence per CTA; the last
+//                         CTA to finish builds the next step's masked-row list.
+#pragma once
+
+#include <cuda_bf16.h>
+#include "head_kernel.cuh"
+
+namespace cai {
+
+constexpr int kMask = -1;
+enum : int { kRunning = 0, kExitDone = 1, kExitGrind = 2, kExitTmax = 3 };
+enum : uint32_t {
+  kFlagGating = 1u,
+  kFlagPosFactor = 2u,
+  kFlagFlush = 4u,
+  kFlagQuarterPos = 8u,
+  kFlagQuarterBlocks = 16u
+};
+constexpr int kMaxP = 256;
+constexpr int kGatherRowsPerCta = 4;
+constexpr int kGatherThreads = 256;
+constexpr int kCommitThreads = 256;
+
+// Host-visible record of the last committed step, in mapped pinned memory.
+struct HostFlag {
+  int32_t seq;       // step id of the last completed commit (-1: none)
+  int32_t blk;       // block of that step
+  int32_t all_done;  // every sequence has exited that block
+  int32_t m_next;    // masked rows the next step will decode
+  uint32_t err;      // copy of the device error word
+  int32_t pad[3];
+};
+
+struct StateArrays {
+  int* tok;
+  float* conf;
+  float* s0;
+  uint8_t* budget;
+  int16_t* cstep;
+  int* cand;
+  int* ell;
+  int* eta;
+  int* exit_reason;
+  int* exit_step;
+  int* unresolved;
+  int* m_hist;
+};
+
+// ------------------------------------------------------------ gather (K1) --
+
+struct GatherParams {
+  const __nv_bfloat16* hidden;  // [B P, H] hidden states of the current block
+  __nv_bfloat16* hc;            // [rows_cap, H] compact operand of the LM head
+  int* list;                    // [B P] token (b P + p) of each masked row
+  int* row_of;                  // [B P] row of each token in this step's list, -1
+  int* d_M;                     // masked rows of this step
+  int* m_hist;                  // [n_blocks, T]
+  int* ell;                     // [B] reset at step zero of a block
+  int hist_idx;
+  int B, BP, H;
+  int first;                    // step zero: every position of every sequence
+};
+
+__global__ void __launch_bounds__(kGatherThreads)
+    gather_rows_kernel(const GatherParams p) {
+  const int M = p.first ? p.BP : *p.d_M;
+  if (p.first) {
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < p.BP; i += gridDim.x * blockDim.x) {
+      p.list[i] = i;
+      p.row_of[i] = i;
+    }
+    if (blockIdx.x == 0) {
+      if (threadIdx.x == 0) *p.d_M = p.BP;
+      for (int b = threadIdx.x; b < p.B; b += blockDim.x) p.ell[b] = 0;
+    }
+  }
+  if (blockIdx.x == 0 && threadIdx.x == 0) p.m_hist[p.hist_idx] = M;
+  const int rows_pad = (M + 15) & ~15;
+  const int r = blockIdx.x * kGatherRowsPerCta + threadIdx.x / 64;
+  if (r >= rows_pad) return;
+  const int t = threadIdx.x & 63;
+  const int nvec = p.H / 8;  // 16-byte vectors per row
+  uint4* dst = reinterpret_cast<uint4*>(p.hc + static_cast<size_t>(r) * p.H);
+  if (r < M) {
+    const int src_row = p.first ? r : p.list[r];
+    const uint4* src = reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(src_row) * p.H);
+    for (int v = t; v < nvec; v += 64) dst[v] = __ldg(src + v);
+  } else {
+    for (int v = t; v < nvec; v += 64) dst[v] = make_uint4(0u, 0u, 0u, 0u);
+  }
+}
+
+// ------------------------------------------------------ list builder -----
+
+// Compact, in (b, p) order, the still-masked tokens of running sequences of
+// block blk into list / row_of; returns the count.  One CTA of
+// kCommitThreads threads.  Reads bypass L1: other CTAs wrote this state.
+__device__ int build_masked_list(const int* tok, const int* exit_reason, int* list, int* row_of,
+                                 int B, int P, int L, int n_blocks, int blk) {
+  __shared__ int s_wsum[kCommitThreads / 32];
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int BP = B * P;
+  int base = 0;
+  for (int i0 = 0; i0 < BP; i0 += kCommitThreads) {
+    const int i = i0 + tid;
+    bool mk = false;
+    if (i < BP) {
+      const int b = i / P, pp = i - b * P;
+      mk = __ldcg(&tok[static_cast<size_t>(b) * L + blk * P + pp]) == kMask &&
+           __ldcg(&exit_reason[b * n_blocks + blk]) == kRunning;
+    }
+    const unsigned bal = __ballot_sync(0xffffffffu, mk);
+    const int wpre = __popc(bal & ((1u << lane) - 1u));
+    if (lane == 0) s_wsum[warp] = __popc(bal);
+    __syncthreads();
+    int woff = 0, tot = 0;
+#pragma unroll
+    for (int w = 0; w < kCommitThreads / 32; ++w) {
+      const int c = s_wsum[w];
+      woff += (w < warp) ? c : 0;
+      tot += c;
+    }
+    if (i < BP) {
+      if (mk) {
+        list[base + woff + wpre] = i;
+        row_of[i] = base + woff + wpre;
+      } else {
+        row_of[i] = -1;
+      }
+    }
+    base += tot;
+    __syncthreads();
+  }
+  return base;
+}
+
+struct ListParams {
+  const int* tok;
+  const int* exit_reason;
+  int* list;
+  int* row_of;
+  int* d_M;
+  int B, P, L, n_blocks, blk;
+};
+
+// Rebuild the masked-row list from the state (after a state upload).
+__global__ void __launch_bounds__(kCommitThreads) rebuild_list_kernel(const ListParams p) {
+  const int n = build_masked_list(p.tok, p.exit_reason, p.list, p.row_of, p.B, p.P, p.L,
+                                  p.n_blocks, p.blk);
+  if (threadIdx.x == 0) *p.d_M = n;
+}
+
+// ------------------------------------------------------ merge + commit (K3) --
+
+struct CommitParams {
+  const float4* part;     // [rows_cap, n_part]
+  int n_part;             // partial slots per row (4 x LM-head CTAs)
+  StateArrays st;
+  int* list;
+  int* row_of;
+  int* d_M;
+  unsigned* ticket;       // zero between launches
+  HostFlag* hf;           // device alias of the mapped host record
+  uint32_t* err;
+  int B, P, L, n_blocks, T, blk, t, step_id;
+  int K;
+  int eta_mode;           // 0 count, 1 fraction of the generation length
+  float eta_bar;
+  float theta_fb;
+  int budget_half;        // Box 5 "p < 32" tier boundary
+  int budget_late;        // Box 5 "p >= 48" tier boundary
+  uint32_t flags;
+  float theta_tab[kMaxP]; // theta_i(t) per position (Box 6), from the host
+};
+
+__device__ __forceinline__ int budget_tier(float s, int p, int half, int late) {
+  if (s > 0.50f && p < half) return 8;
+  if (s < 0.25f || p >= late) return 64;
+  return 32;
+}
+
+__global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const CommitParams p) {
+  __shared__ int s_eta, s_left, s_reason, s_unres, s_last;
+  const int b = blockIdx.x;
+  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+  const int eb = b * p.n_blocks + p.blk;
+  const bool running = p.st.exit_reason[eb] == kRunning;
+  const bool gating = (p.flags & kFlagGating) != 0;
+  if (tid == 0) {
+    s_eta = 0;
+    s_left = 0;
+    s_reason = kRunning;
+    s_unres = 0;
+  }
+  __syncthreads();
+
+  if (running) {
+    // One warp per masked position: merge its partials, then the commit rule.
+    for (int pp = warp; pp < p.P; pp += kCommitThreads / 32) {
+      const size_t g = static_cast<size_t>(b) * p.L + p.blk * p.P + pp;
+      if (p.st.tok[g] != kMask) continue;
+      const int row = p.row_of[b * p.P + pp];
+      if (row < 0) {
+        if (lane == 0) atomicOr(p.err, kErrBadRow);
+        continue;
+      }
+      float m = kNegBig, s = 0.0f;
+      int ix = INT_MAX;
+      const float4* pr = p.part + static_cast<size_t>(row) * p.n_part;
+      for (int k = lane; k < p.n_part; k += 32) {
+        const float4 q = pr[k];
+        merge_tri(m, s, ix, q.x, q.y, __float_as_int(q.z));
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) {
+        const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+        const float so = __shfl_xor_sync(0xffffffffu, s, off);
+        const int io = __shfl_xor_sync(0xffffffffu, ix, off);
+        merge_tri(m, s, ix, mo, so, io);
+      }
+      if (lane == 0) {
+        const float c = 1.0f / s;  // max_v p_v = exp(m - LSE) = 1 / sum_v exp(z_v - m)
+        if (p.t == 0) {
+          p.st.s0[g] = c;
+          p.st.budget[g] = static_cast<uint8_t>(budget_tier(c, pp, p.budget_half, p.budget_late));
+        }
+        p.st.conf[g] = c;
+        p.st.cand[g] = ix;
+        const bool by_conf = c >= p.theta_tab[pp];
+        const bool by_budget = gating && p.t >= static_cast<int>(p.st.budget[g]);
+        if (by_conf || by_budget) {
+          p.st.tok[g] = ix;
+          p.st.cstep[g] = static_cast<int16_t>(p.t);
+          atomicAdd(&s_eta, 1);
+        } else {
+          atomicAdd(&s_left, 1);
+        }
+      }
+    }
+  }
+  __syncthreads();
+  if (running && tid == 0) {
+    const int eta = s_eta;
+    p.st.eta[b] = eta;
+    const bool low = p.eta_mode == 1
+                         ? (static_cast<double>(eta) / (static_cast<double>(p.n_blocks) * p.P) <
+                            static_cast<double>(p.eta_bar))
+                         : (static_cast<float>(eta) < p.eta_bar);
+    const int ell = low ? p.st.ell[b] + 1 : 0;
+    p.st.ell[b] = ell;
+    int reason = kRunning;
+    if (gating && ell >= p.K)
+      reason = kExitGrind;
+    else if (s_left == 0)
+      reason = kExitDone;
+    else if (p.t == p.T - 1)
+      reason = kExitTmax;
+    s_reason = reason;
+  }
+  __syncthreads();
+  const int reason = s_reason;
+  if (running && reason != kRunning) {
+    for (int pp = tid; pp < p.P; pp += kCommitThreads) {
+      const size_t g = static_cast<size_t>(b) * p.L + p.blk * p.P + pp;
+      if (p.st.tok[g] != kMask) continue;
+      if ((reason == kExitGrind && p.st.conf[g] > p.theta_fb) || (p.flags & kFlagFlush)) {
+        p.st.tok[g] = p.st.cand[g];
+        p.st.cstep[g] = static_cast<int16_t>(p.t);
+      } else {
+        atomicAdd(&s_unres, 1);
+      }
+    }
+    __syncthreads();
+    if (tid == 0) {
+      p.st.exit_reason[eb] = reason;
+      p.st.exit_step[eb] = p.t;
+      p.st.unresolved[eb] = s_unres;
+    }
+  }
+
+  // Last CTA to finish: next step's list and the host-visible record.
+  __syncthreads();
+  if (tid == 0) {
+    __threadfence();
+    s_last = atomicAdd(p.ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  const int n = build_masked_list(p.st.tok, p.st.exit_reason, p.list, p.row_of, p.B, p.P, p.L,
+                                  p.n_blocks, p.blk);
+  if (tid == 0) {
+    *p.d_M = n;
+    *p.ticket = 0u;
+    volatile HostFlag* hf = p.hf;
+    hf->blk = p.blk;
+    hf->all_done = n == 0 ? 1 : 0;
+    hf->m_next = n;
+    hf->err = *reinterpret_cast<volatile uint32_t*>(p.err);
+    __threadfence_system();
+    hf->seq = p.step_id;
+    __threadfence_system();
+  }
+}
+
+}  // namespace cai

@@ -1,0 +1,328 @@
+"""GPU parity: the sm_103a path through the C ABI against the oracle.
+
+Every test here runs the decoding head and commit rule on the GPU (gather,
+tcgen05 LM head with the online softmax epilogue, merge + commit) and checks
+each step teacher-forced against the fp64 oracle (``tests/parity.py``).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+import synth
+from tests import parity
+
+import paper_2608_22646_gb300 as cai
+
+pytestmark = pytest.mark.gpu
+
+
+def _ctx(B, P, H, V, T, n_blocks, preset=0, flags=None, W=None, seed=1234):
+    if W is None:
+        W = synth.lm_head_weight(V, H, seed=seed, device="cuda")
+    cfg = cai.cai_config_default(preset, B, P, H, V, T, n_blocks)
+    if flags is not None:
+        cfg.flags = flags
+    return cai.cai_init(cfg, W), W
+
+
+def _wl(name, **kw):
+    wl = synth.WORKLOADS[name]
+    return synth.Workload(**{**wl.__dict__, **kw})
+
+
+def test_toy_trajectory_every_step():
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows > wl.P * wl.n_blocks      # several steps per block
+        assert np.all(final["exit_reason"] != 0)
+        print(rep)
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_toy_literal_generator_grinds_at_t3():
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "literal")
+    try:
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert np.all(final["exit_reason"] == cai.CAI_EXIT_GRIND)
+        assert np.all(final["exit_step"] == 3)
+        assert np.all(final["tok"] == -1)
+    finally:
+        cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("shape,grid", [
+    # (B, P, H, V, T, n_blocks), LM-head CTA cap: ragged vocab tails (V % 64,
+    # V % 128), a single K stage (H = 64), M = 1, several MMA chunks (M > 256),
+    # B P not a multiple of 16, CTAs with several 128-row tiles and a 64-row one.
+    ((1, 1, 64, 64, 4, 2), 0),
+    ((3, 7, 128, 1000, 6, 2), 0),
+    ((3, 7, 128, 1000, 6, 2), 3),
+    ((2, 33, 192, 2112, 8, 2), 5),
+    ((2, 150, 64, 4160, 5, 1), 0),
+    ((2, 150, 64, 4160, 5, 1), 7),
+    ((5, 64, 256, 8192, 12, 2), 9),
+    ((1, 16, 256, 4096, 8, 4), 1),
+])
+def test_ragged_shapes_trajectory(shape, grid):
+    B, P, H, V, T, nb = shape
+    wl = synth.Workload("ragged", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    cai.cai_test_head_grid_limit(grid)
+    try:
+        ctx, W = _ctx(B, P, H, V, T, nb,
+                      flags=cai.CAI_GATING | cai.CAI_POS_FACTOR | cai.CAI_QUARTER_POS)
+    finally:
+        cai.cai_test_head_grid_limit(0)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=7)
+    try:
+        if grid:
+            assert cai.cai_get_stats(ctx)["grid"] == grid
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P
+    finally:
+        cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("preset,flags", [
+    (cai.CAI_PRESET_DREAM, None),  # gating OFF: budgets and grinding exit disabled
+    (cai.CAI_PRESET_LLADA, cai.CAI_GATING | cai.CAI_POS_FACTOR | cai.CAI_FLUSH_ON_EXIT),
+    (cai.CAI_PRESET_LLADA, cai.CAI_GATING | cai.CAI_QUARTER_BLOCKS),
+])
+def test_controller_variants(preset, flags):
+    wl = _wl("toy", B=4, a0="bimodal", gen_len=128)
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks, preset=preset, flags=flags)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=3)
+    try:
+        parity.run_checked_trajectory(ctx, W, hs)
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_fraction_eta_mode():
+    wl = _wl("toy", B=2)
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    cfg.eta_mode = 1
+    cfg.eta_bar = 0.015
+    ctx = cai.cai_init(cfg, W)
+    try:
+        parity.run_checked_trajectory(ctx, W, synth.HiddenStates(wl, W, "calibrated", seed=11))
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_all_commit_at_step_zero_and_noop_steps():
+    # Hidden rows equal to a scaled W row make every confidence ~1: every
+    # token commits at t = 0, the block exits DONE, and later steps decode nothing.
+    B, P, H, V, T = 2, 16, 256, 4096, 8
+    ctx, W = _ctx(B, P, H, V, T, 2)
+    try:
+        tgt = torch.arange(B * P, device="cuda") * 37 % V
+        h = (W[tgt].float() * 400.0).to(torch.bfloat16).reshape(B, P, H)
+        cai.cai_first_step(ctx, h)
+        assert cai.cai_poll(ctx, 0, 5000)
+        st = cai.cai_state_download(ctx)
+        assert np.array_equal(st["tok"][:, :P].reshape(-1), tgt.cpu().numpy())
+        assert np.all(st["exit_reason"][:, 0] == cai.CAI_EXIT_DONE)
+        assert np.all(st["exit_step"][:, 0] == 0)
+        with pytest.raises(cai.CaiError) as e:      # poll saw the block end
+            cai.cai_denoise_step(ctx, h)
+        assert e.value.status == cai.CAI_ERR_ORDER
+        cai.cai_block_advance(ctx)
+        cai.cai_first_step(ctx, h)
+        cai.cai_denoise_step(ctx, h)                # issued before a poll: decodes nothing
+        torch.cuda.synchronize()
+        st = cai.cai_state_download(ctx)
+        assert st["m_hist"][1, 0] == B * P and st["m_hist"][1, 1] == 0
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_teacher_forced_random_states():
+    # Random mid-block states uploaded into the context, then one step.
+    wl = _wl("toy", B=6, P=16, gen_len=32, T=20)
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=5)
+    ocfg = parity.oracle_config(ctx.cfg)
+    rng = np.random.default_rng(0)
+    try:
+        for trial in range(6):
+            blk = int(rng.integers(0, wl.n_blocks))
+            t = int(rng.integers(1, wl.T))
+            st = cai.cai_state_download(ctx)
+            for k in ("tok", "cstep", "cand", "budget", "conf", "s0"):
+                st[k][:] = 0
+            st["tok"][:] = -1
+            st["cstep"][:] = -1
+            sl = slice(blk * wl.P, (blk + 1) * wl.P)
+            committed = rng.random((wl.B, wl.P)) < 0.4
+            st["tok"][:, sl] = np.where(committed, rng.integers(0, wl.V, (wl.B, wl.P)), -1)
+            st["cstep"][:, sl] = np.where(committed, rng.integers(0, t, (wl.B, wl.P)), -1)
+            st["budget"][:, sl] = rng.choice([8, 32, 64], (wl.B, wl.P))
+            st["ell"][:] = rng.integers(0, 4, wl.B)
+            st["exit_reason"][:] = 0
+            st["exit_reason"][:, blk] = np.where(rng.random(wl.B) < 0.2, 1, 0)
+            st["exit_step"][:] = -1
+            st["unresolved"][:] = 0
+            st["m_hist"][:] = 0
+            st["blk"], st["t_next"] = blk, t
+            cai.cai_state_upload(ctx, st)
+            pre = cai.cai_state_download(ctx)
+            h = hs(blk, t)
+            cai.cai_denoise_step(ctx, h)
+            torch.cuda.synchronize()
+            post = cai.cai_state_download(ctx)
+            parity.check_step(ocfg, oracle.bf16_bits(W), h, pre, post, blk, t)
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_host_hidden_and_host_weight_match_device():
+    wl = synth.WORKLOADS["toy"]
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    a = cai.cai_init(cfg, W)
+    Wh = W.cpu().pin_memory()
+    b = cai.cai_init(cfg, Wh)
+    try:
+        for blk in range(2):
+            if blk:
+                cai.cai_block_advance(a)
+                cai.cai_block_advance(b)
+            for t in range(wl.T):
+                h = hs(blk, t)
+                step = cai.cai_first_step if t == 0 else cai.cai_denoise_step
+                step(a, h)
+                step(b, h.cpu().pin_memory())
+                torch.cuda.synchronize()
+        sa, sb = cai.cai_state_download(a), cai.cai_state_download(b)
+        for k in ("tok", "conf", "cand", "exit_reason", "m_hist"):
+            assert np.array_equal(sa[k], sb[k]), k
+        out = torch.empty((wl.B, wl.n_blocks * wl.P), dtype=torch.int32).pin_memory()
+        cai.cai_read_tokens(a, out)
+        torch.cuda.synchronize()
+        assert np.array_equal(out.numpy(), sa["tok"])
+    finally:
+        cai.cai_free(a)
+        cai.cai_free(b)
+
+
+def test_order_errors_and_poll():
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, 2)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        h = hs(0, 0)
+        with pytest.raises(cai.CaiError) as e:        # misaligned hidden pointer
+            cai.cai_first_step(ctx, h.data_ptr() + 2)
+        assert e.value.status == cai.CAI_ERR_ARG
+        for fn in (lambda: cai.cai_denoise_step(ctx, h), lambda: cai.cai_block_advance(ctx)):
+            with pytest.raises(cai.CaiError) as e:
+                fn()
+            assert e.value.status == cai.CAI_ERR_ORDER
+        assert not cai.cai_poll(ctx, 0, 100)          # nothing issued yet
+        cai.cai_first_step(ctx, h)
+        with pytest.raises(cai.CaiError) as e:
+            cai.cai_first_step(ctx, h)
+        assert e.value.status == cai.CAI_ERR_ORDER
+        for t in range(1, wl.T):
+            cai.cai_denoise_step(ctx, hs(0, t))
+        with pytest.raises(cai.CaiError) as e:        # t would reach T
+            cai.cai_denoise_step(ctx, h)
+        assert e.value.status == cai.CAI_ERR_ORDER
+        assert cai.cai_poll(ctx, 0, 5000)             # t = T - 1 always ends the block
+        cai.cai_block_advance(ctx)
+        cai.cai_first_step(ctx, h)
+        with pytest.raises(cai.CaiError) as e:        # already at the last block
+            cai.cai_block_advance(ctx)
+        assert e.value.status == cai.CAI_ERR_ORDER
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_alloc_failure_injection_leaks_nothing():
+    wl = synth.WORKLOADS["toy"]
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    torch.cuda.synchronize()
+    free0 = torch.cuda.mem_get_info()[0]
+    for n in (1, 5, 12, 20):
+        cai.cai_test_fail_alloc_after(n)
+        with pytest.raises(cai.CaiError) as e:
+            cai.cai_init(cfg, W)
+        assert e.value.status == cai.CAI_ERR_NOMEM
+    cai.cai_test_fail_alloc_after(0)
+    ctx = cai.cai_init(cfg, W)
+    cai.cai_free(ctx)
+    torch.cuda.synchronize()
+    assert abs(torch.cuda.mem_get_info()[0] - free0) < (8 << 20)
+
+
+def test_profile_and_stats():
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        cai.cai_profile(ctx, True)
+        cai.cai_first_step(ctx, hs(0, 0))
+        cai.cai_denoise_step(ctx, hs(0, 1))
+        s = cai.cai_get_stats(ctx)
+        assert s["steps"] == 2 and s["head_launches"] == 2 and s["launches"] == 6
+        assert s["head_profiled"] == 2 and s["head_ms"] > 0
+        assert s["grid"] == 64 and s["n_max"] == 16
+    finally:
+        cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("name", ["llada", "dream"])
+def test_full_size_first_step_sampled(name):
+    # Full LLaDA/Dream shapes: one step-zero decode of the whole block, then
+    # the oracle recomputes a sample of positions one by one.
+    wl = synth.WORKLOADS[name]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        h = hs(0, 0)
+        cai.cai_first_step(ctx, h)
+        torch.cuda.synchronize()
+        st = cai.cai_state_download(ctx)
+        sample = [0, 5, 17, wl.P - 1]
+        rows = oracle.bf16_bits(h.reshape(-1, wl.H))[sample]
+        o = oracle.head_rows(W, rows)
+        for k, p in enumerate(sample):
+            assert abs(st["s0"][0, p] - o["conf"][k]) <= parity.CONF_TOL
+            if o["gap"][k] > parity.GAP_TOL:
+                assert st["cand"][0, p] == o["idx"][k]
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_batched_multi_chunk_step_sampled():
+    # B = 64 sequences, 2048 masked rows (8 MMA chunks of 256) at full LLaDA
+    # width; sampled rows across chunks against the oracle.
+    wl = synth.WORKLOADS["llada_batched"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        h = hs(0, 0)
+        cai.cai_first_step(ctx, h)
+        torch.cuda.synchronize()
+        st = cai.cai_state_download(ctx)
+        flat = [0, 255, 256, 1023, 1500, 2047]
+        rows = oracle.bf16_bits(h.reshape(-1, wl.H))[flat]
+        o = oracle.head_rows(W, rows)
+        for k, i in enumerate(flat):
+            b, p = divmod(i, wl.P)
+            assert abs(st["s0"][b, p] - o["conf"][k]) <= parity.CONF_TOL
+            if o["gap"][k] > parity.GAP_TOL:
+                assert st["cand"][b, p] == o["idx"][k]
+        assert st["m_hist"][0, 0] == wl.B * wl.P
+    finally:
+        cai.cai_free(ctx)

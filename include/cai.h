@@ -19,7 +19,11 @@
  *
  * Execution model.  Every call that takes a stream is asynchronous on that
  * stream (a CUDA stream handle, or NULL for the legacy default stream); the
- * library never synchronises the device on the step path.  The batch runs
+ * library never synchronises the device on the step path.  The step kernels
+ * use programmatic dependent launch: each may be scheduled while the kernel
+ * before it in the stream still runs, and waits for that kernel to complete
+ * before touching anything it produces (setting CAI_PDL=0 in the environment
+ * before cai_init launches them plainly instead).  The batch runs
  * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
  * per sequence) and contribute no rows afterwards.  A context is not thread
  * safe; use one context per host thread.
@@ -74,7 +78,8 @@ extern "C" {
  * theta_fb, w (warmup_pct / 100), K, eta_bar.
  *
  * Shape limits (else CAI_ERR_SHAPE): B >= 1; 1 <= P <= 256; H % 64 == 0 and
- * 64 <= H <= 16384; V >= 64; 1 <= T <= 32767; n_blocks >= 1; B * P <= 65536.
+ * 64 <= H <= 16384; V >= 64; 1 <= T <= 32767; 1 <= n_blocks <= 32767;
+ * B * P <= 65536.
  */
 typedef struct cai_config {
   int32_t B;           /* sequences in the batch                                  */

@@ -10,9 +10,11 @@
 #include <chrono>
 #include <cmath>
 #include <cstdio>
+#include <cstdlib>
 #include <cstring>
 #include <new>
 #include <thread>
+#include <utility>
 #include <vector>
 
 #include "cai.h"
@@ -24,6 +26,13 @@ namespace {
 
 std::atomic<int> g_fail_alloc_after{0};
 std::atomic<int> g_head_grid_limit{0};
+
+// Programmatic dependent launch between the step's kernels; CAI_PDL=0 in the
+// environment turns it off (read once per context at cai_init).
+bool pdl_enabled() {
+  const char* e = std::getenv("CAI_PDL");
+  return !(e && e[0] == '0');
+}
 
 int dev_alloc(void** p, size_t bytes) {
   *p = nullptr;
@@ -84,6 +93,26 @@ int next_pow2(int x) {
   return p;
 }
 
+// Launch with programmatic stream serialization: the kernel may be scheduled
+// while the previous kernel in the stream is still running; every kernel of
+// this library waits for its predecessor (griddepcontrol.wait) before it
+// reads or writes anything that predecessor produces or consumes.
+template <typename... KArgs, typename... Args>
+cudaError_t launch_pdl(bool pdl, void (*kernel)(KArgs...), int grid, int block, size_t smem,
+                       cudaStream_t stream, Args&&... args) {
+  cudaLaunchConfig_t cfg = {};
+  cfg.gridDim = dim3(static_cast<unsigned>(grid));
+  cfg.blockDim = dim3(static_cast<unsigned>(block));
+  cfg.dynamicSmemBytes = smem;
+  cfg.stream = stream;
+  cudaLaunchAttribute attr[1];
+  attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+  attr[0].val.programmaticStreamSerializationAllowed = 1;
+  cfg.attrs = attr;
+  cfg.numAttrs = pdl ? 1 : 0;
+  return cudaLaunchKernelEx(&cfg, kernel, std::forward<Args>(args)...);
+}
+
 bool is_device_ptr(const void* p) {
   cudaPointerAttributes a;
   if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
@@ -120,6 +149,7 @@ struct cai_ctx {
   int sticky = CAI_OK;
   cai_stats stats{};
   bool profiling = false;
+  bool pdl = true;
   std::vector<cudaEvent_t> ev_pool;  // pairs (start, stop)
   size_t ev_used = 0;                // events recorded since the last stats call
   std::vector<void*> allocs;
@@ -145,7 +175,7 @@ int validate(const cai_config* c) {
   if (c->B < 1 || c->P < 1 || c->P > kMaxP || c->H < 64 || c->H > 16384 || (c->H % 64) != 0 ||
       c->V < 64 || c->T < 1 || c->T > 32767 || c->n_blocks < 1 ||
       static_cast<int64_t>(c->B) * c->P > 65536 ||
-      static_cast<int64_t>(c->n_blocks) * c->P > (1 << 24))
+      c->n_blocks > 32767 || static_cast<int64_t>(c->n_blocks) * c->P > (1 << 24))
     return CAI_ERR_SHAPE;
   if (c->warmup_pct < 0 || c->warmup_pct > 100 || c->K < 1 || (c->eta_mode != 0 && c->eta_mode != 1) ||
       !(c->clip_lo <= c->clip_hi) || (c->flags & ~31u) != 0)
@@ -215,19 +245,18 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   gp.list = c->list;
   gp.row_of = c->row_of;
   gp.d_M = c->d_M;
-  gp.m_hist = c->st.m_hist;
-  gp.ell = c->st.ell;
-  gp.hist_idx = c->blk * cfg.T + t;
   gp.B = cfg.B;
   gp.BP = c->BP;
   gp.H = cfg.H;
   gp.first = first ? 1 : 0;
   const int g_grid = c->rows_cap / kGatherRowsPerCta;
-  gather_rows_kernel<<<g_grid, kGatherThreads, 0, stream>>>(gp);
+  if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) != cudaSuccess)
+    return check_launch(c);
   c->stats.launches++;
 
   HeadParams hp{};
   hp.d_M = c->d_M;
+  hp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
   hp.part = c->part;
   hp.err = c->err;
   hp.V = cfg.V;
@@ -251,15 +280,16 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     c->ev_used += 2;
     cudaEventRecord(e0, stream);
   }
-  lm_head_softmax_kernel<<<c->G, kHeadThreads, c->head_smem, stream>>>(c->tm_w128, c->tm_w64,
-                                                                       c->tm_h, hp);
+  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream, c->tm_w128,
+                 c->tm_w64, c->tm_h, hp) != cudaSuccess)
+    return check_launch(c);
   if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.launches++;
   c->stats.head_launches++;
 
   CommitParams cp{};
   cp.part = c->part;
-  cp.n_part = 4 * c->G;
+  cp.n_part = c->G;
   cp.st = c->st;
   cp.list = c->list;
   cp.row_of = c->row_of;
@@ -289,7 +319,9 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     th = th > cfg.clip_hi ? cfg.clip_hi : th;
     cp.theta_tab[p] = static_cast<float>(th);
   }
-  merge_commit_kernel<<<cfg.B, kCommitThreads, 0, stream>>>(cp);
+  const int commit_threads = cfg.P < kCommitThreads / 32 ? 32 * cfg.P : kCommitThreads;
+  if (launch_pdl(c->pdl, merge_commit_kernel, cfg.B, commit_threads, 0, stream, cp) != cudaSuccess)
+    return check_launch(c);
   c->stats.launches++;
   c->stats.steps++;
   int r = check_launch(c);
@@ -354,6 +386,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->L = cfg->n_blocks * cfg->P;
   c->BP = cfg->B * cfg->P;
   c->rows_cap = round_up(c->BP, 16);
+  c->pdl = pdl_enabled();
 
   // LM-head launch shape: N chunk, tensor-memory columns, pipeline depth.
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
@@ -399,7 +432,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->ticket, unsigned, 1)
   CAI_ALLOC(c->err, uint32_t, 1)
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
-  CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * 4 * c->G)
+  CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * c->G)
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
   if (!is_device_ptr(W)) {
     CAI_ALLOC(c->W_owned, uint8_t, static_cast<size_t>(cfg->V) * cfg->H * 2)
@@ -423,7 +456,6 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     return CAI_ERR_NOMEM;
   }
   std::memset(c->hf_host, 0, sizeof(HostFlag));
-  reinterpret_cast<volatile HostFlag*>(c->hf_host)->seq = -1;
   // A 128-row tile is only used when a CTA owns two 64-row units, so V >= 128.
   if (!make_map(&c->tm_w128, c->W, cfg->V, cfg->H, cfg->V >= 128 ? 128 : 64) ||
       !make_map(&c->tm_w64, c->W, cfg->V, cfg->H, 64) ||
@@ -518,12 +550,15 @@ int cai_poll(cai_ctx* c, int32_t lag, int32_t timeout_ms, int32_t* all_done) {
   *all_done = 0;
   const int64_t target = c->last_step_id - lag;
   if (target < 0) return CAI_OK;
-  volatile HostFlag* hf = c->hf_host;
+  volatile unsigned long long* word = &c->hf_host->word;
   const auto t0 = std::chrono::steady_clock::now();
+  unsigned long long w = 0;
   for (uint32_t it = 0;; ++it) {
-    const int32_t seq = hf->seq;
-    if (seq >= target) break;
-    if (hf->err) return fail(c, CAI_ERR_DEVICE);
+    w = *word;
+    // The word holds step id + 1 (ids are kept since cai_init); 0 means "none yet".
+    const bool seen = static_cast<int64_t>(w & 0xFFFFFFFFull) - 1 >= target;
+    if ((w >> 33) & 1ull) return fail(c, CAI_ERR_DEVICE);
+    if (seen) break;
     if ((it & 255u) == 255u) {
       const auto dt = std::chrono::steady_clock::now() - t0;
       if (std::chrono::duration_cast<std::chrono::milliseconds>(dt).count() >= timeout_ms)
@@ -531,9 +566,8 @@ int cai_poll(cai_ctx* c, int32_t lag, int32_t timeout_ms, int32_t* all_done) {
       std::this_thread::yield();
     }
   }
-  std::atomic_thread_fence(std::memory_order_acquire);
-  if (hf->err) return fail(c, CAI_ERR_DEVICE);
-  if (hf->blk == c->blk && hf->all_done) {
+  const int blk = static_cast<int>((w >> 34) & 0x7FFFull);
+  if (blk == (c->blk & 0x7FFF) && ((w >> 32) & 1ull)) {
     *all_done = 1;
     c->block_done_seen = true;
   }
@@ -591,7 +625,9 @@ int cai_state_download(cai_ctx* c, cai_host_state* dst) {
   if (r != CAI_OK) return r;
   dst->blk = c->blk;
   dst->t_next = c->t_next;
-  if (reinterpret_cast<volatile HostFlag*>(c->hf_host)->err) return fail(c, CAI_ERR_DEVICE);
+  uint32_t err = 0;
+  if (cudaMemcpy(&err, c->err, 4, cudaMemcpyDeviceToHost) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+  if (err) return fail(c, CAI_ERR_DEVICE);
   return CAI_OK;
 }
 

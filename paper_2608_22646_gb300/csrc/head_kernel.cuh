@@ -8,8 +8,9 @@
 // rows in units of 64 rows, streams it once from HBM through a TMA ring of
 // K = 64 stages, and keeps the logits in tensor memory: they are never
 // written anywhere.  The epilogue reduces every accumulator tile to a running
-// (max, sum of exponentials, argmax) per position in the log2 domain, and each
-// epilogue warp writes one partial triple per position, [M, 4 gridDim.x].
+// (max, sum of exponentials, argmax) per position in the log2 domain; the four
+// epilogue warps merge their slices through shared memory and each CTA writes
+// one partial triple per position, [M, gridDim.x].
 //
 // Warp roles (192 threads, one CTA per SM):
 //   warp 0      TMA producer (one lane): W tile + hidden tile per stage
@@ -34,7 +35,8 @@ constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows t
 
 struct HeadParams {
   const int* d_M;     // masked rows of this step (device)
-  float4* part;       // [rows_cap, 4 G] partial (m2, S, idx bits, 0) per epilogue warp
+  int* m_hist_slot;   // where this step's M is recorded
+  float4* part;       // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
   uint32_t* err;      // error word
   int V, H;
   int units;          // ceil(V / 64)
@@ -116,19 +118,20 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, uint3
 struct HeadSmem {
   uint8_t* a;       // n_stages x 16 KiB
   uint8_t* b;       // n_stages x b_stage_bytes
+  float4* epi;      // [2][4][acc_stride] cross-warp merge, double-buffered by chunk
   uint64_t* full;   // n_stages
   uint64_t* empty;  // n_stages
   uint64_t* accf;   // 2
   uint64_t* acce;   // 2
   uint64_t* drain;  // 1
+  uint64_t* epib;   // 2: the four epilogue warps have written epi[buffer]
   uint32_t* tmem_slot;
   volatile int* abort;
 };
 
 __host__ __device__ inline size_t head_smem_bytes(int n_stages, int b_stage_bytes, int acc_stride) {
-  (void)acc_stride;
-  return 1024 + (size_t)n_stages * (kATileBytes + b_stage_bytes) + (size_t)(2 * n_stages + 5) * 8 +
-         16;
+  return 1024 + (size_t)n_stages * (kATileBytes + b_stage_bytes) + (size_t)8 * acc_stride * 16 +
+         (size_t)(2 * n_stages + 7) * 8 + 16;
 }
 
 __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
@@ -137,12 +140,14 @@ __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
                                              ~static_cast<uintptr_t>(1023));
   s.a = base;
   s.b = s.a + (size_t)p.n_stages * kATileBytes;
-  s.full = reinterpret_cast<uint64_t*>(s.b + (size_t)p.n_stages * p.b_stage_bytes);
+  s.epi = reinterpret_cast<float4*>(s.b + (size_t)p.n_stages * p.b_stage_bytes);
+  s.full = reinterpret_cast<uint64_t*>(s.epi + 8 * p.acc_stride);
   s.empty = s.full + p.n_stages;
   s.accf = s.empty + p.n_stages;
   s.acce = s.accf + 2;
   s.drain = s.acce + 2;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
+  s.epib = s.drain + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.epib + 2);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   return s;
 }
@@ -152,8 +157,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                            const __grid_constant__ CUtensorMap tm_w64,
                            const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
   extern __shared__ uint8_t smem_raw[];
-  const int M = *p.d_M;
-  if (M <= 0) return;  // every sequence has exited: nothing to decode
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
   HeadSmem sm = carve(smem_raw, p);
@@ -163,9 +166,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   const int u0 = static_cast<int>((static_cast<long long>(cta) * p.units) / G);
   const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.units) / G);
   const int n_tiles = (u1 - u0 + 1) >> 1;
-  const int n_chunks = (M + kChunkN - 1) / kChunkN;
   const int KB = p.H / kBlockK;
 
+  // Prologue (overlaps the previous kernel under programmatic dependent launch).
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.n_stages; ++s) {
       mbar_init(&sm.full[s], 1);
@@ -176,8 +179,11 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
       mbar_init(&sm.acce[a], 4);
     }
     mbar_init(sm.drain, 1);
+    mbar_init(&sm.epib[0], 4);
+    mbar_init(&sm.epib[1], 4);
     *sm.abort = 0;
     fence_mbar_init();
+    grid_launch_dependents();
   }
   if (warp == 0 && lane == 0) {
     prefetch_tmap(&tm_w128);
@@ -193,11 +199,28 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   tc_fence_after();
   const uint32_t tmem_base = *sm.tmem_slot;
 
+  // The weight does not depend on the previous kernels: the producer starts
+  // streaming the first ring of W tiles before waiting for them.  Everything
+  // that does (the masked-row count, the gathered rows, the partial buffer)
+  // is touched only after grid_dependency_wait().
+  const int n_pre = min(p.n_stages, n_tiles * KB);
+
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------ producer --
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_h = policy_evict_last();
+      for (int i = 0; i < n_pre; ++i) {
+        const int j = i / KB, kb = i - j * KB;
+        const int ut = u0 + 2 * j;
+        const int rows = (u1 - ut >= 2) ? 128 : 64;
+        mbar_expect_tx(&sm.full[i], static_cast<uint32_t>(rows * 128));
+        tma_load_2d(sm.a + (size_t)i * kATileBytes, rows == 128 ? &tm_w128 : &tm_w64, &sm.full[i],
+                    kb * kBlockK, ut * kUnitRows, pol_w);
+      }
+      grid_dependency_wait();
+      const int M = *p.d_M;
+      const int n_chunks = (M + kChunkN - 1) / kChunkN;
       int stage = 0;
       uint32_t phase = 0;
       long long issued = 0;
@@ -210,15 +233,18 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
           const int rows = (u1 - ut >= 2) ? 128 : 64;
           const int r0 = ut * kUnitRows;
           const CUtensorMap* tw = rows == 128 ? &tm_w128 : &tm_w64;
-          const uint32_t bytes = static_cast<uint32_t>(rows * 128 + nq * 128);
           for (int kb = 0; kb < KB; ++kb) {
-            if (!mbar_wait(&sm.empty[stage], phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
+            const bool pre = issued < n_pre;  // A already in flight for this stage
+            if (!pre &&
+                !mbar_wait(&sm.empty[stage], phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(&sm.full[stage], bytes);
-            tma_load_2d(sm.a + (size_t)stage * kATileBytes, tw, &sm.full[stage], kb * kBlockK, r0,
-                        pol_w);
+            mbar_arrive_expect_tx(&sm.full[stage],
+                                  static_cast<uint32_t>((pre ? 0 : rows * 128) + nq * 128));
+            if (!pre)
+              tma_load_2d(sm.a + (size_t)stage * kATileBytes, tw, &sm.full[stage], kb * kBlockK,
+                          r0, pol_w);
             uint8_t* bdst = sm.b + (size_t)stage * p.b_stage_bytes;
             for (int i = 0; i < nq / kBoxRowsB; ++i)
               tma_load_2d(bdst + i * kBoxRowsB * 128, &tm_h, &sm.full[stage], kb * kBlockK,
@@ -230,6 +256,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
           }
         }
+      }
+      if (issued < n_pre) {
+        // Nothing to decode (M = 0) or an abort before the prefetched stages
+        // were claimed: complete their phases so the W copies can be drained.
+        for (long long i = issued; i < n_pre; ++i) mbar_arrive(&sm.full[i]);
+        for (long long i = issued; i < n_pre; ++i) mbar_drain(&sm.full[i], 0, p.err);
       }
       if (!ok) {
         // Abort path: let the copies already in flight land before exit.
@@ -243,6 +275,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------------------------------------------- MMA issuer --
+      grid_dependency_wait();
+      const int M = *p.d_M;
+      const int n_chunks = (M + kChunkN - 1) / kChunkN;
       int stage = 0;
       uint32_t phase = 0;
       int acc = 0;
@@ -293,7 +328,11 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     __syncwarp();
   } else {
     // --------------------------------------------------------- epilogue --
-    const int ew = warp - 2;       // 0..3: partial slot of this warp
+    grid_dependency_wait();
+    const int M = *p.d_M;
+    const int n_chunks = (M + kChunkN - 1) / kChunkN;
+    if (threadIdx.x == 64 && cta == 0) *p.m_hist_slot = M;
+    const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
     int acc = 0;
@@ -342,15 +381,36 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         if (acc == 0) acc_phase ^= 1u;
       }
       if (!ok) break;
-      // One partial per (position, CTA, epilogue warp): no cross-warp barrier,
-      // the merge kernel combines the 4 G slots of each position.
-      const int ncols = min(nq, M - n0);
+      // Cross-warp merge of the four 32-row slices of every column, then one
+      // partial per (position, CTA).  The buffer alternates by chunk: a warp
+      // writes buffer q & 1 again only after every warp arrived for chunk q + 1,
+      // which each does after reading chunk q.
+      const int buf = q & 1;
+      float4* epi = sm.epi + buf * 4 * p.acc_stride;
 #pragma unroll
       for (int g = 0; g < 8; ++g) {
-        const int col = 32 * g + lane;
-        if (g < ngroups && col < ncols)
-          p.part[static_cast<size_t>(n0 + col) * (4 * G) + 4 * cta + ew] =
+        if (g < ngroups)
+          epi[ew * p.acc_stride + 32 * g + lane] =
               make_float4(rm[g], rs[g], __int_as_float(ri[g]), 0.0f);
+      }
+      __syncwarp();
+      if (lane == 0) mbar_arrive(&sm.epib[buf]);
+      if (!mbar_wait(&sm.epib[buf], static_cast<uint32_t>((q >> 1) & 1), sm.abort, p.err,
+                     kErrWaitEpi)) {
+        ok = false;
+        break;
+      }
+      const int ncols = min(nq, M - n0);
+      for (int col = ew * 32 + lane; col < ncols; col += 128) {
+        const float4 a = epi[col];
+        float m = a.x, s = a.y;
+        int i = __float_as_int(a.z);
+#pragma unroll
+        for (int w = 1; w < 4; ++w) {
+          const float4 b = epi[w * p.acc_stride + col];
+          merge_tri(m, s, i, b.x, b.y, __float_as_int(b.z));
+        }
+        p.part[static_cast<size_t>(n0 + col) * G + cta] = make_float4(m, s, __int_as_float(i), 0.0f);
       }
     }
   }

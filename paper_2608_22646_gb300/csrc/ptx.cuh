@@ -21,6 +21,7 @@ enum : uint32_t {
   kErrWaitAccEmpty = 1u << 3,// MMA issuer waiting for a drained accumulator
   kErrDrain = 1u << 4,       // drain of in-flight copies on the abort path
   kErrBadRow = 1u << 5,      // a masked token had no row in this step's list
+  kErrWaitEpi = 1u << 6,     // epilogue warps waiting for each other's slices
 };
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
@@ -47,6 +48,13 @@ __device__ __forceinline__ void fence_mbar_init() {
 
 __device__ __forceinline__ void mbar_arrive_expect_tx(uint64_t* bar, uint32_t bytes) {
   asm volatile("mbarrier.arrive.expect_tx.shared::cta.b64 _, [%0], %1;" ::"r"(smem_addr(bar)),
+               "r"(bytes)
+               : "memory");
+}
+
+// Add transaction bytes to the current phase without arriving.
+__device__ __forceinline__ void mbar_expect_tx(uint64_t* bar, uint32_t bytes) {
+  asm volatile("mbarrier.expect_tx.relaxed.cta.shared::cta.b64 [%0], %1;" ::"r"(smem_addr(bar)),
                "r"(bytes)
                : "memory");
 }
@@ -85,6 +93,20 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
       }
     }
   }
+}
+
+// ---------------------------------------------- programmatic dependent launch --
+
+// Wait until the grids this launch depends on (the previous kernel in the
+// stream) have completed and their memory operations are visible.
+__device__ __forceinline__ void grid_dependency_wait() {
+  asm volatile("griddepcontrol.wait;" ::: "memory");
+}
+
+// Allow the next kernel in the stream to be scheduled before this one ends;
+// it still waits for this grid's completion before reading what it wrote.
+__device__ __forceinline__ void grid_launch_dependents() {
+  asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 
 // ------------------------------------------------------------------ TMA --

@@ -128,7 +128,6 @@ struct cai_ctx {
   cai_config cfg{};
   int L = 0, BP = 0, rows_cap = 0;
   const void* W = nullptr;
-  void* W_owned = nullptr;
   StateArrays st{};
   int* list = nullptr;
   int* row_of = nullptr;
@@ -140,7 +139,8 @@ struct cai_ctx {
   void* hidden_stage = nullptr;
   HostFlag* hf_host = nullptr;
   HostFlag* hf_dev = nullptr;
-  CUtensorMap tm_w128{}, tm_w64{}, tm_h{};
+  void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
+  CUtensorMap tm_h{};
   int G = 0, n_stages = 0, n_max = 0, acc_stride = 0, tmem_cols = 0, b_stage_bytes = 0;
   size_t head_smem = 0;
   int blk = 0, t_next = 0;
@@ -255,6 +255,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   c->stats.launches++;
 
   HeadParams hp{};
+  hp.wpk = static_cast<const uint8_t*>(c->wpk);
   hp.d_M = c->d_M;
   hp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
   hp.part = c->part;
@@ -280,8 +281,8 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     c->ev_used += 2;
     cudaEventRecord(e0, stream);
   }
-  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream, c->tm_w128,
-                 c->tm_w64, c->tm_h, hp) != cudaSuccess)
+  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream, c->tm_h,
+                 hp) != cudaSuccess)
     return check_launch(c);
   if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.launches++;
@@ -434,18 +435,39 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
   CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * c->G)
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
+  CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * 128 * cfg->H)
+  const void* w_src = W;
+  void* w_tmp = nullptr;
   if (!is_device_ptr(W)) {
-    CAI_ALLOC(c->W_owned, uint8_t, static_cast<size_t>(cfg->V) * cfg->H * 2)
-    if (cudaMemcpy(c->W_owned, W, static_cast<size_t>(cfg->V) * cfg->H * 2,
-                   cudaMemcpyHostToDevice) != cudaSuccess) {
+    if ((r = dev_alloc(&w_tmp, static_cast<size_t>(cfg->V) * cfg->H * 2)) != CAI_OK) {
+      release(c);
+      delete c;
+      return r;
+    }
+    if (cudaMemcpy(w_tmp, W, static_cast<size_t>(cfg->V) * cfg->H * 2, cudaMemcpyHostToDevice) !=
+        cudaSuccess) {
+      cudaFree(w_tmp);
       release(c);
       delete c;
       return CAI_ERR_CUDA;
     }
-    c->W = c->W_owned;
-  } else {
-    c->W = W;
+    w_src = w_tmp;
   }
+  {
+    const long long n_chunks = static_cast<long long>(units) * 64 * cfg->H / 8;
+    pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+        static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
+        n_chunks);
+    const cudaError_t e1 = cudaGetLastError();
+    const cudaError_t e2 = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
+    if (w_tmp) cudaFree(w_tmp);
+    if (e1 != cudaSuccess || e2 != cudaSuccess) {
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+  }
+  c->W = W;
 #undef CAI_ALLOC
   if (cudaHostAlloc(reinterpret_cast<void**>(&c->hf_host), sizeof(HostFlag), cudaHostAllocMapped) !=
           cudaSuccess ||
@@ -456,10 +478,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     return CAI_ERR_NOMEM;
   }
   std::memset(c->hf_host, 0, sizeof(HostFlag));
-  // A 128-row tile is only used when a CTA owns two 64-row units, so V >= 128.
-  if (!make_map(&c->tm_w128, c->W, cfg->V, cfg->H, cfg->V >= 128 ? 128 : 64) ||
-      !make_map(&c->tm_w64, c->W, cfg->V, cfg->H, 64) ||
-      !make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB)) {
+  if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB)) {
     release(c);
     delete c;
     return CAI_ERR_CUDA;

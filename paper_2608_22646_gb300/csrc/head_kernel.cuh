@@ -5,17 +5,18 @@
 // run with A and B swapped: the vocabulary fills the MMA M dimension (128 rows
 // of W per accumulator tile) and the positions form the N dimension
 // (16..256 columns, rounded up to 16).  Each CTA owns a contiguous range of W
-// rows in units of 64 rows, streams it once from HBM through a TMA ring of
+// rows in units of 64 rows and streams it once from HBM through a ring of
 // K = 64 stages, and keeps the logits in tensor memory: they are never
-// written anywhere.  The epilogue reduces every accumulator tile to a running
-// (max, sum of exponentials, argmax) per position in the log2 domain; the four
-// epilogue warps merge their slices through shared memory and each CTA writes
-// one partial triple per position, [M, gridDim.x].
+// written anywhere.
 //
-// Warp roles (192 threads, one CTA per SM):
-//   warp 0      TMA producer (one lane): W tile + hidden tile per stage
-//   warp 1      TMEM allocator; one lane issues tcgen05.mma
-//   warps 2..5  epilogue: tcgen05.ld, transposing warp reduction, partials
+// W is read from a packed copy made once per context (pack_weight_kernel) in
+// exactly the order the CTAs consume it: CTA c owns rows [64 u0, 64 u1) and
+// the bytes [128 H u0, 128 H u1) of the packed copy, laid out tile by tile and
+// k block by k block, each stage already in the 128-byte-swizzled K-major
+// layout the MMA descriptors expect.  Every CTA therefore streams one
+// contiguous region front to back with one bulk copy per stage; contiguous
+// copies keep DRAM pages open, the strided 128-byte rows of a 2-D tensor box
+// do not.
 #pragma once
 
 #include <climits>
@@ -34,6 +35,7 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows to 0
 
 struct HeadParams {
+  const uint8_t* wpk; // packed W (see pack_weight_kernel)
   const int* d_M;     // masked rows of this step (device)
   int* m_hist_slot;   // where this step's M is recorded
   float4* part;       // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
@@ -104,6 +106,51 @@ __device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool
   oi = ix[0];
 }
 
+// First 64-row unit of CTA c when `units` units are split over G CTAs.
+__host__ __device__ inline int unit_begin(int c, int units, int G) {
+  return static_cast<int>((static_cast<long long>(c) * units) / G);
+}
+
+// Byte offset in the packed weight of the stage (tile j, k block kb) of a CTA
+// whose range starts at unit u0; rows = 128, or 64 for a final half tile.
+__host__ __device__ inline size_t packed_stage(int u0, int j, int kb, int rows, int H) {
+  return static_cast<size_t>(u0) * 128 * H + static_cast<size_t>(j) * 256 * H +
+         static_cast<size_t>(kb) * rows * 128;
+}
+
+// Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` 64-row
+// units.  Inside a stage block, row r's 16-byte chunk c (k = 8c..8c+7 of the
+// block's 64) sits at r * 128 + ((c ^ (r & 7)) * 16): the 128-byte swizzle of
+// 8-row, 1024-byte atoms.  Rows >= V are zero.  One thread per destination
+// 16-byte chunk; n_chunks = units * 64 * H / 8.
+__global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
+                                   int H, int units, int G, long long n_chunks) {
+  const long long unit_bytes = 128ll * H;
+  for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
+       d += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long byte = d * 16;
+    const int u = static_cast<int>(byte / unit_bytes);
+    // CTA owning unit u: the largest c with unit_begin(c) <= u.
+    int c = static_cast<int>((static_cast<long long>(u) * G) / units);
+    while (c + 1 < G && unit_begin(c + 1, units, G) <= u) ++c;
+    while (c > 0 && unit_begin(c, units, G) > u) --c;
+    const int u0 = unit_begin(c, units, G), u1 = unit_begin(c + 1, units, G);
+    const long long off = byte - static_cast<long long>(u0) * unit_bytes;
+    const int j = static_cast<int>(off / (2 * unit_bytes));
+    const long long rem = off - static_cast<long long>(j) * 2 * unit_bytes;
+    const int ut = u0 + 2 * j;
+    const int rows = (u1 - ut >= 2) ? 128 : 64;
+    const int kb = static_cast<int>(rem / (rows * 128));
+    const int inblk = static_cast<int>(rem - static_cast<long long>(kb) * rows * 128);
+    const int r = inblk >> 7;
+    const int cl = ((inblk >> 4) & 7) ^ (r & 7);
+    const long long v = static_cast<long long>(ut) * 64 + r;
+    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
+    out[d] = val;
+  }
+}
+
 // Wait used only on the abort path, for copies this CTA already issued.
 __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, uint32_t* err) {
   const uint64_t t0 = global_timer_ns();
@@ -152,10 +199,15 @@ __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
   return s;
 }
 
+// Stage (tile j, k block kb) of this CTA's packed range: one contiguous copy.
+__device__ __forceinline__ void load_w_stage(uint8_t* dst, const uint8_t* wpk, int u0, int j,
+                                             int rows, int kb, int H, uint64_t* bar, uint64_t pol) {
+  bulk_load(dst, wpk + packed_stage(u0, j, kb, rows, H), static_cast<uint32_t>(rows * 128), bar,
+            pol);
+}
+
 __global__ void __launch_bounds__(kHeadThreads, 1)
-    lm_head_softmax_kernel(const __grid_constant__ CUtensorMap tm_w128,
-                           const __grid_constant__ CUtensorMap tm_w64,
-                           const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
+    lm_head_softmax_kernel(const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -163,8 +215,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
   const int G = gridDim.x;
   const int cta = blockIdx.x;
-  const int u0 = static_cast<int>((static_cast<long long>(cta) * p.units) / G);
-  const int u1 = static_cast<int>((static_cast<long long>(cta + 1) * p.units) / G);
+  const int u0 = unit_begin(cta, p.units, G);
+  const int u1 = unit_begin(cta + 1, p.units, G);
   const int n_tiles = (u1 - u0 + 1) >> 1;
   const int KB = p.H / kBlockK;
 
@@ -185,11 +237,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     fence_mbar_init();
     grid_launch_dependents();
   }
-  if (warp == 0 && lane == 0) {
-    prefetch_tmap(&tm_w128);
-    prefetch_tmap(&tm_w64);
-    prefetch_tmap(&tm_h);
-  }
+  if (warp == 0 && lane == 0) prefetch_tmap(&tm_h);
   if (warp == 1) {
     tmem_alloc(sm.tmem_slot, static_cast<uint32_t>(p.tmem_cols));
     tmem_relinquish();
@@ -215,8 +263,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         const int ut = u0 + 2 * j;
         const int rows = (u1 - ut >= 2) ? 128 : 64;
         mbar_expect_tx(&sm.full[i], static_cast<uint32_t>(rows * 128));
-        tma_load_2d(sm.a + (size_t)i * kATileBytes, rows == 128 ? &tm_w128 : &tm_w64, &sm.full[i],
-                    kb * kBlockK, ut * kUnitRows, pol_w);
+        load_w_stage(sm.a + (size_t)i * kATileBytes, p.wpk, u0, j, rows, kb, p.H, &sm.full[i],
+                     pol_w);
       }
       grid_dependency_wait();
       const int M = *p.d_M;
@@ -231,8 +279,6 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         for (int j = 0; j < n_tiles && ok; ++j) {
           const int ut = u0 + 2 * j;
           const int rows = (u1 - ut >= 2) ? 128 : 64;
-          const int r0 = ut * kUnitRows;
-          const CUtensorMap* tw = rows == 128 ? &tm_w128 : &tm_w64;
           for (int kb = 0; kb < KB; ++kb) {
             const bool pre = issued < n_pre;  // A already in flight for this stage
             if (!pre &&
@@ -243,8 +289,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             mbar_arrive_expect_tx(&sm.full[stage],
                                   static_cast<uint32_t>((pre ? 0 : rows * 128) + nq * 128));
             if (!pre)
-              tma_load_2d(sm.a + (size_t)stage * kATileBytes, tw, &sm.full[stage], kb * kBlockK,
-                          r0, pol_w);
+              load_w_stage(sm.a + (size_t)stage * kATileBytes, p.wpk, u0, j, rows, kb, p.H,
+                           &sm.full[stage], pol_w);
             uint8_t* bdst = sm.b + (size_t)stage * p.b_stage_bytes;
             for (int i = 0; i < nq / kBoxRowsB; ++i)
               tma_load_2d(bdst + i * kBoxRowsB * 128, &tm_h, &sm.full[stage], kb * kBlockK,

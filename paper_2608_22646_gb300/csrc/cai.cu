@@ -34,6 +34,14 @@ bool pdl_enabled() {
   return !(e && e[0] == '0');
 }
 
+// Optional caps on the LM head's W ring depth (CAI_HEAD_STAGES) and tile
+// group size (CAI_HEAD_GMAX), read once per context at cai_init; 0 or unset
+// keeps the defaults.  Tuning knobs only: results do not depend on them.
+int env_int(const char* name) {
+  const char* e = std::getenv(name);
+  return e ? std::atoi(e) : 0;
+}
+
 int dev_alloc(void** p, size_t bytes) {
   *p = nullptr;
   int n = g_fail_alloc_after.load();
@@ -141,7 +149,8 @@ struct cai_ctx {
   HostFlag* hf_dev = nullptr;
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
   CUtensorMap tm_h{};
-  int G = 0, n_stages = 0, n_max = 0, acc_stride = 0, tmem_cols = 0, b_stage_bytes = 0;
+  int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
+  int b_slot_bytes = 0;
   size_t head_smem = 0;
   int blk = 0, t_next = 0;
   int64_t last_step_id = -1;
@@ -264,8 +273,10 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.H = cfg.H;
   hp.units = (cfg.V + kUnitRows - 1) / kUnitRows;
   hp.n_stages = c->n_stages;
-  hp.b_stage_bytes = c->b_stage_bytes;
-  hp.acc_stride = c->acc_stride;
+  hp.n_bslots = c->n_bslots;
+  hp.b_slot_bytes = c->b_slot_bytes;
+  hp.slot_cols = c->slot_cols;
+  hp.gmax = c->gmax;
   hp.tmem_cols = c->tmem_cols;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
   if (c->profiling) {
@@ -389,21 +400,44 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->rows_cap = round_up(c->BP, 16);
   c->pdl = pdl_enabled();
 
-  // LM-head launch shape: N chunk, tensor-memory columns, pipeline depth.
+  // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
+  // at most one per 64-row unit), tile group size (tiles sharing one hidden
+  // stage; two group buffers of gmax * slot_cols tensor-memory columns fit in
+  // 512), ring depths within the opt-in shared memory.
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
-  c->acc_stride = round_up(c->n_max, 32);
-  c->tmem_cols = next_pow2(2 * c->acc_stride < 32 ? 32 : 2 * c->acc_stride);
-  c->b_stage_bytes = c->n_max * 128;
-  int stages = 12;
-  while (stages > 2 && head_smem_bytes(stages, c->b_stage_bytes, c->acc_stride) >
-                           static_cast<size_t>(smem_optin))
-    --stages;
-  c->n_stages = stages;
-  c->head_smem = head_smem_bytes(stages, c->b_stage_bytes, c->acc_stride);
+  c->slot_cols = round_up(c->n_max, 32);
   const int units = (cfg->V + kUnitRows - 1) / kUnitRows;
   c->G = units < sms ? units : sms;
   const int glim = g_head_grid_limit.load();
   if (glim > 0 && c->G > glim) c->G = glim;
+  const int max_units = (units + c->G - 1) / c->G;
+  const int max_tiles = (max_units + 1) / 2;
+  // Default: as many tiles per group as two group buffers of tensor memory
+  // allow (all of a CTA's tiles for N <= 32).  Every tile of a group is an
+  // independent accumulation chain, and at small N a single chain is bound by
+  // MMA latency rather than HBM; interleaving the chains of the group hides
+  // it.  CAI_HEAD_GMAX overrides (bounded by the tensor memory).
+  c->gmax = max_tiles;
+  const int gset = env_int("CAI_HEAD_GMAX");
+  if (gset > 0) c->gmax = gset;
+  if (c->gmax > 256 / c->slot_cols) c->gmax = 256 / c->slot_cols;
+  if (c->gmax < 1) c->gmax = 1;
+  c->tmem_cols = next_pow2(2 * c->gmax * c->slot_cols < 32 ? 32 : 2 * c->gmax * c->slot_cols);
+  c->b_slot_bytes = c->n_max * 128;
+  auto bslots_for = [&](int stages) {
+    // One hidden stage serves a group of tiles; keep enough of them in flight
+    // to cover the W ring (groups may be one tile smaller than gmax).
+    const int per = c->gmax > 1 ? c->gmax - 1 : 1;
+    return c->gmax == 1 ? stages : (stages + per - 1) / per + 1;
+  };
+  const int scap = env_int("CAI_HEAD_STAGES");
+  int stages = scap >= 2 && scap < 12 ? scap : 12;
+  while (stages > 2 && head_smem_bytes(stages, bslots_for(stages), c->b_slot_bytes,
+                                       c->slot_cols) > static_cast<size_t>(smem_optin))
+    --stages;
+  c->n_stages = stages;
+  c->n_bslots = bslots_for(stages);
+  c->head_smem = head_smem_bytes(stages, c->n_bslots, c->b_slot_bytes, c->slot_cols);
 
   const size_t BL = static_cast<size_t>(cfg->B) * c->L;
   const size_t BN = static_cast<size_t>(cfg->B) * cfg->n_blocks;
@@ -457,7 +491,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     const long long n_chunks = static_cast<long long>(units) * 64 * cfg->H / 8;
     pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
-        n_chunks);
+        c->gmax, n_chunks);
     const cudaError_t e1 = cudaGetLastError();
     const cudaError_t e2 = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
     if (w_tmp) cudaFree(w_tmp);

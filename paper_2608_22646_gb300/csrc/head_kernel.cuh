@@ -5,18 +5,34 @@
 // run with A and B swapped: the vocabulary fills the MMA M dimension (128 rows
 // of W per accumulator tile) and the positions form the N dimension
 // (16..256 columns, rounded up to 16).  Each CTA owns a contiguous range of W
-// rows in units of 64 rows and streams it once from HBM through a ring of
-// K = 64 stages, and keeps the logits in tensor memory: they are never
-// written anywhere.
+// rows in units of 64 rows and reads it once from HBM; the logits stay in
+// tensor memory and are never written anywhere.  The epilogue reduces every
+// accumulator tile to a running (max, sum of exponentials, argmax) per
+// position in the log2 domain; the four epilogue warps merge their slices
+// through shared memory and each CTA writes one partial triple per position,
+// [M, gridDim.x].
+//
+// Tiles are processed in groups (up to `gmax` tiles of 128 rows): for each
+// K block the hidden-state stage (B) is loaded once and used by every tile of
+// the group, each tile accumulating into its own tensor-memory slot.  The B
+// operand is thus read from L2 once per group instead of once per tile, and
+// the group's tiles form independent accumulation chains whose MMAs overlap:
+// at small N one chain alone is bound by MMA latency, not by HBM.  Two group
+// buffers let the epilogue of one group overlap the MMAs of the next.
 //
 // W is read from a packed copy made once per context (pack_weight_kernel) in
 // exactly the order the CTAs consume it: CTA c owns rows [64 u0, 64 u1) and
-// the bytes [128 H u0, 128 H u1) of the packed copy, laid out tile by tile and
-// k block by k block, each stage already in the 128-byte-swizzled K-major
-// layout the MMA descriptors expect.  Every CTA therefore streams one
-// contiguous region front to back with one bulk copy per stage; contiguous
-// copies keep DRAM pages open, the strided 128-byte rows of a 2-D tensor box
-// do not.
+// the bytes [128 H u0, 128 H u1) of the packed copy, laid out group by group,
+// K block by K block, tile by tile, each stage already in the
+// 128-byte-swizzled K-major layout the MMA descriptors expect.  Every CTA thus
+// streams one contiguous region front to back with one bulk copy per stage;
+// contiguous copies keep DRAM pages open, the strided 128-byte rows of a 2-D
+// tensor box do not.
+//
+// Warp roles (192 threads, one CTA per SM):
+//   warp 0      producer (one lane): W stages (bulk copies), hidden stages (TMA)
+//   warp 1      TMEM allocator; one lane issues tcgen05.mma
+//   warps 2..5  epilogue: tcgen05.ld, transposing warp reduction, partials
 #pragma once
 
 #include <climits>
@@ -35,18 +51,97 @@ constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows to 0
 
 struct HeadParams {
-  const uint8_t* wpk; // packed W (see pack_weight_kernel)
-  const int* d_M;     // masked rows of this step (device)
-  int* m_hist_slot;   // where this step's M is recorded
-  float4* part;       // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
-  uint32_t* err;      // error word
+  const uint8_t* wpk;  // packed W (see pack_weight_kernel)
+  const int* d_M;      // masked rows of this step (device)
+  int* m_hist_slot;    // where this step's M is recorded
+  float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
+  uint32_t* err;       // error word
   int V, H;
-  int units;          // ceil(V / 64)
-  int n_stages;
-  int b_stage_bytes;  // n_max * 128
-  int acc_stride;     // tensor-memory columns per accumulator buffer
-  int tmem_cols;      // allocated tensor-memory columns
+  int units;           // ceil(V / 64)
+  int n_stages;        // depth of the W ring (16 KiB slots)
+  int n_bslots;        // depth of the hidden-state ring
+  int b_slot_bytes;    // n_max * 128
+  int slot_cols;       // tensor-memory columns per tile accumulator (round32(n_max))
+  int gmax;            // largest tile group
+  int tmem_cols;       // allocated tensor-memory columns (>= 2 gmax slot_cols)
 };
+
+// ------------------------------------------------------------ CTA plan --
+
+// First 64-row unit of CTA c when `units` units are split over G CTAs.
+__host__ __device__ inline int unit_begin(int c, int units, int G) {
+  return static_cast<int>((static_cast<long long>(c) * units) / G);
+}
+
+// The work of one CTA: units [u0, u1) as tiles of 128 rows (the last may be
+// 64), grouped gsz = min(gmax, tiles) tiles at a time.
+struct CtaPlan {
+  int u0, u1, n_tiles, gsz, n_groups;
+  __host__ __device__ int tile_rows(int t) const { return (u1 - (u0 + 2 * t) >= 2) ? 128 : 64; }
+  __host__ __device__ int group_first(int g) const { return g * gsz; }
+  __host__ __device__ int group_count(int g) const {
+    const int n = n_tiles - g * gsz;
+    return n < gsz ? n : gsz;
+  }
+  __host__ __device__ int group_rows(int g) const {
+    const int t0 = group_first(g), n = group_count(g);
+    return 128 * (n - 1) + tile_rows(t0 + n - 1);
+  }
+  // Byte offset in the packed weight of W stage (group g, K block kb, tile t).
+  __host__ __device__ size_t stage_offset(int g, int kb, int t, int H) const {
+    return static_cast<size_t>(u0) * 128 * H + static_cast<size_t>(g) * gsz * 256 * H +
+           static_cast<size_t>(kb) * group_rows(g) * 128 +
+           static_cast<size_t>(t - group_first(g)) * kATileBytes;
+  }
+};
+
+__host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
+  CtaPlan p;
+  p.u0 = unit_begin(c, units, G);
+  p.u1 = unit_begin(c + 1, units, G);
+  p.n_tiles = (p.u1 - p.u0 + 1) >> 1;
+  const int g = gmax < p.n_tiles ? gmax : p.n_tiles;
+  p.gsz = g < 1 ? 1 : g;
+  p.n_groups = (p.n_tiles + p.gsz - 1) / p.gsz;
+  return p;
+}
+
+// Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` 64-row
+// units and groups of up to gmax tiles.  Inside a stage block, row r's
+// 16-byte chunk c (k = 8c..8c+7 of the block's 64) sits at
+// r * 128 + ((c ^ (r & 7)) * 16): the 128-byte swizzle of 8-row, 1024-byte
+// atoms.  Rows >= V are zero.  One thread per destination 16-byte chunk;
+// n_chunks = units * 64 * H / 8.
+__global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
+                                   int H, int units, int G, int gmax, long long n_chunks) {
+  const long long unit_bytes = 128ll * H;
+  for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
+       d += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long byte = d * 16;
+    const int u = static_cast<int>(byte / unit_bytes);
+    // CTA owning unit u: the largest c with unit_begin(c) <= u.
+    int c = static_cast<int>((static_cast<long long>(u) * G) / units);
+    while (c + 1 < G && unit_begin(c + 1, units, G) <= u) ++c;
+    while (c > 0 && unit_begin(c, units, G) > u) --c;
+    const CtaPlan pl = cta_plan(c, units, G, gmax);
+    const long long off = byte - static_cast<long long>(pl.u0) * unit_bytes;
+    const int g = static_cast<int>(off / (static_cast<long long>(pl.gsz) * 2 * unit_bytes));
+    const long long rem = off - static_cast<long long>(g) * pl.gsz * 2 * unit_bytes;
+    const int grow = pl.group_rows(g);
+    const int kb = static_cast<int>(rem / (grow * 128));
+    const int rem2 = static_cast<int>(rem - static_cast<long long>(kb) * grow * 128);
+    const int t = pl.group_first(g) + rem2 / kATileBytes;
+    const int inblk = rem2 % kATileBytes;
+    const int r = inblk >> 7;
+    const int cl = ((inblk >> 4) & 7) ^ (r & 7);
+    const long long v = static_cast<long long>(pl.u0 + 2 * t) * 64 + r;
+    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
+    out[d] = val;
+  }
+}
+
+// ------------------------------------------------------------ reduction --
 
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
@@ -67,20 +162,12 @@ __device__ __forceinline__ void merge_tri(float& m, float& s, int& i, float mo, 
   i = in;
 }
 
-// 32 rows (one per lane) x 32 columns (one register each) -> lane l holds the
-// (max, sum, argmax) of column l over the 32 rows.  Five halving steps: at
+// 32 lanes x 32 columns of online-softmax triples -> lane l holds the merge of
+// column l over the 32 lanes, in m[0], s[0], ix[0].  Five halving steps: at
 // width w each lane keeps half of its live columns and receives the partner's
 // copy of the same columns (31 merges per lane, one exponential each).
-__device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
-                                                   int lane, float& om, float& os, int& oi) {
-  float m[32], s[32];
-  int ix[32];
-#pragma unroll
-  for (int c = 0; c < 32; ++c) {
-    m[c] = valid ? __uint_as_float(v[c]) * kLog2e : kNegBig;
-    s[c] = valid ? 1.0f : 0.0f;
-    ix[c] = valid ? vrow : INT_MAX;
-  }
+__device__ __forceinline__ void transpose_merge32(float (&m)[32], float (&s)[32], int (&ix)[32],
+                                                  int lane) {
 #pragma unroll
   for (int w = 16; w >= 1; w >>= 1) {
     const bool up = (lane & w) != 0;
@@ -101,54 +188,36 @@ __device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool
       ix[c] = ki;
     }
   }
+}
+
+// 32 rows (one per lane) x 32 columns of logits -> lane l holds the
+// (max, sum, argmax) of column l over the 32 rows.
+__device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
+                                                   int lane, float& om, float& os, int& oi) {
+  float m[32], s[32];
+  int ix[32];
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    m[c] = valid ? __uint_as_float(v[c]) * kLog2e : kNegBig;
+    s[c] = valid ? 1.0f : 0.0f;
+    ix[c] = valid ? vrow : INT_MAX;
+  }
+  transpose_merge32(m, s, ix, lane);
   om = m[0];
   os = s[0];
   oi = ix[0];
 }
 
-// First 64-row unit of CTA c when `units` units are split over G CTAs.
-__host__ __device__ inline int unit_begin(int c, int units, int G) {
-  return static_cast<int>((static_cast<long long>(c) * units) / G);
-}
-
-// Byte offset in the packed weight of the stage (tile j, k block kb) of a CTA
-// whose range starts at unit u0; rows = 128, or 64 for a final half tile.
-__host__ __device__ inline size_t packed_stage(int u0, int j, int kb, int rows, int H) {
-  return static_cast<size_t>(u0) * 128 * H + static_cast<size_t>(j) * 256 * H +
-         static_cast<size_t>(kb) * rows * 128;
-}
-
-// Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` 64-row
-// units.  Inside a stage block, row r's 16-byte chunk c (k = 8c..8c+7 of the
-// block's 64) sits at r * 128 + ((c ^ (r & 7)) * 16): the 128-byte swizzle of
-// 8-row, 1024-byte atoms.  Rows >= V are zero.  One thread per destination
-// 16-byte chunk; n_chunks = units * 64 * H / 8.
-__global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
-                                   int H, int units, int G, long long n_chunks) {
-  const long long unit_bytes = 128ll * H;
-  for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
-       d += static_cast<long long>(gridDim.x) * blockDim.x) {
-    const long long byte = d * 16;
-    const int u = static_cast<int>(byte / unit_bytes);
-    // CTA owning unit u: the largest c with unit_begin(c) <= u.
-    int c = static_cast<int>((static_cast<long long>(u) * G) / units);
-    while (c + 1 < G && unit_begin(c + 1, units, G) <= u) ++c;
-    while (c > 0 && unit_begin(c, units, G) > u) --c;
-    const int u0 = unit_begin(c, units, G), u1 = unit_begin(c + 1, units, G);
-    const long long off = byte - static_cast<long long>(u0) * unit_bytes;
-    const int j = static_cast<int>(off / (2 * unit_bytes));
-    const long long rem = off - static_cast<long long>(j) * 2 * unit_bytes;
-    const int ut = u0 + 2 * j;
-    const int rows = (u1 - ut >= 2) ? 128 : 64;
-    const int kb = static_cast<int>(rem / (rows * 128));
-    const int inblk = static_cast<int>(rem - static_cast<long long>(kb) * rows * 128);
-    const int r = inblk >> 7;
-    const int cl = ((inblk >> 4) & 7) ^ (r & 7);
-    const long long v = static_cast<long long>(ut) * 64 + r;
-    uint4 val = make_uint4(0u, 0u, 0u, 0u);
-    if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
-    out[d] = val;
-  }
+// Fold one logit z (log2 units) of vocabulary row `row` into a running
+// triple.  Rows arrive in increasing order, so only a strictly larger value
+// replaces the argmax (ties keep the lower index).
+__device__ __forceinline__ void online_update(float& m, float& s, int& i, float z, int row) {
+  const float d = z - m;
+  const float e = fast_exp2(-fabsf(d));
+  const bool up = d > 0.0f;
+  s = up ? fmaf(s, e, 1.0f) : s + e;
+  m = up ? z : m;
+  i = up ? row : i;
 }
 
 // Wait used only on the abort path, for copies this CTA already issued.
@@ -162,23 +231,29 @@ __device__ __forceinline__ void mbar_drain(uint64_t* bar, uint32_t parity, uint3
   }
 }
 
+// ------------------------------------------------------------- smem map --
+
 struct HeadSmem {
-  uint8_t* a;       // n_stages x 16 KiB
-  uint8_t* b;       // n_stages x b_stage_bytes
-  float4* epi;      // [2][4][acc_stride] cross-warp merge, double-buffered by chunk
-  uint64_t* full;   // n_stages
-  uint64_t* empty;  // n_stages
-  uint64_t* accf;   // 2
-  uint64_t* acce;   // 2
-  uint64_t* drain;  // 1
-  uint64_t* epib;   // 2: the four epilogue warps have written epi[buffer]
+  uint8_t* a;        // n_stages x 16 KiB (W)
+  uint8_t* b;        // n_bslots x b_slot_bytes (hidden rows)
+  float4* epi;       // [2][4][slot_cols] cross-warp merge, double-buffered by chunk
+  uint64_t* full_a;  // n_stages
+  uint64_t* empty_a; // n_stages
+  uint64_t* full_b;  // n_bslots
+  uint64_t* empty_b; // n_bslots
+  uint64_t* accf;    // 2: group accumulators ready
+  uint64_t* acce;    // 2: group accumulators drained by the epilogue
+  uint64_t* drain;   // 1
+  uint64_t* epib;    // 2: the four epilogue warps have written epi[buffer]
   uint32_t* tmem_slot;
   volatile int* abort;
 };
 
-__host__ __device__ inline size_t head_smem_bytes(int n_stages, int b_stage_bytes, int acc_stride) {
-  return 1024 + (size_t)n_stages * (kATileBytes + b_stage_bytes) + (size_t)8 * acc_stride * 16 +
-         (size_t)(2 * n_stages + 7) * 8 + 16;
+__host__ __device__ inline size_t head_smem_bytes(int n_stages, int n_bslots, int b_slot_bytes,
+                                                  int slot_cols) {
+  return 1024 + static_cast<size_t>(n_stages) * kATileBytes +
+         static_cast<size_t>(n_bslots) * b_slot_bytes + static_cast<size_t>(8) * slot_cols * 16 +
+         static_cast<size_t>(2 * n_stages + 2 * n_bslots + 7) * 8 + 16;
 }
 
 __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
@@ -186,11 +261,13 @@ __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   s.a = base;
-  s.b = s.a + (size_t)p.n_stages * kATileBytes;
-  s.epi = reinterpret_cast<float4*>(s.b + (size_t)p.n_stages * p.b_stage_bytes);
-  s.full = reinterpret_cast<uint64_t*>(s.epi + 8 * p.acc_stride);
-  s.empty = s.full + p.n_stages;
-  s.accf = s.empty + p.n_stages;
+  s.b = s.a + static_cast<size_t>(p.n_stages) * kATileBytes;
+  s.epi = reinterpret_cast<float4*>(s.b + static_cast<size_t>(p.n_bslots) * p.b_slot_bytes);
+  s.full_a = reinterpret_cast<uint64_t*>(s.epi + 8 * p.slot_cols);
+  s.empty_a = s.full_a + p.n_stages;
+  s.full_b = s.empty_a + p.n_stages;
+  s.empty_b = s.full_b + p.n_bslots;
+  s.accf = s.empty_b + p.n_bslots;
   s.acce = s.accf + 2;
   s.drain = s.acce + 2;
   s.epib = s.drain + 1;
@@ -199,12 +276,19 @@ __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
   return s;
 }
 
-// Stage (tile j, k block kb) of this CTA's packed range: one contiguous copy.
-__device__ __forceinline__ void load_w_stage(uint8_t* dst, const uint8_t* wpk, int u0, int j,
-                                             int rows, int kb, int H, uint64_t* bar, uint64_t pol) {
-  bulk_load(dst, wpk + packed_stage(u0, j, kb, rows, H), static_cast<uint32_t>(rows * 128), bar,
-            pol);
-}
+// Ring position: slot index and the parity of its current phase.
+struct Ring {
+  int slot = 0;
+  uint32_t phase = 0;
+  __device__ void next(int n) {
+    if (++slot == n) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+// ---------------------------------------------------------------- kernel --
 
 __global__ void __launch_bounds__(kHeadThreads, 1)
     lm_head_softmax_kernel(const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
@@ -215,24 +299,25 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
   const int G = gridDim.x;
   const int cta = blockIdx.x;
-  const int u0 = unit_begin(cta, p.units, G);
-  const int u1 = unit_begin(cta + 1, p.units, G);
-  const int n_tiles = (u1 - u0 + 1) >> 1;
+  const CtaPlan pl = cta_plan(cta, p.units, G, p.gmax);
   const int KB = p.H / kBlockK;
 
   // Prologue (overlaps the previous kernel under programmatic dependent launch).
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.n_stages; ++s) {
-      mbar_init(&sm.full[s], 1);
-      mbar_init(&sm.empty[s], 1);
+      mbar_init(&sm.full_a[s], 1);
+      mbar_init(&sm.empty_a[s], 1);
+    }
+    for (int s = 0; s < p.n_bslots; ++s) {
+      mbar_init(&sm.full_b[s], 1);
+      mbar_init(&sm.empty_b[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&sm.accf[a], 1);
       mbar_init(&sm.acce[a], 4);
+      mbar_init(&sm.epib[a], 4);
     }
     mbar_init(sm.drain, 1);
-    mbar_init(&sm.epib[0], 4);
-    mbar_init(&sm.epib[1], 4);
     *sm.abort = 0;
     fence_mbar_init();
     grid_launch_dependents();
@@ -246,74 +331,89 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   __syncthreads();
   tc_fence_after();
   const uint32_t tmem_base = *sm.tmem_slot;
+  const int group_cols = p.gmax * p.slot_cols;  // tensor-memory columns per group buffer
 
   // The weight does not depend on the previous kernels: the producer starts
-  // streaming the first ring of W tiles before waiting for them.  Everything
+  // streaming the first ring of W stages before waiting for them.  Everything
   // that does (the masked-row count, the gathered rows, the partial buffer)
   // is touched only after grid_dependency_wait().
-  const int n_pre = min(p.n_stages, n_tiles * KB);
+  const int n_pre = min(p.n_stages, pl.n_tiles * KB);
 
   if (warp == 0) {
     if (lane == 0) {
       // ------------------------------------------------------ producer --
       const uint64_t pol_w = policy_evict_first();
       const uint64_t pol_h = policy_evict_last();
-      for (int i = 0; i < n_pre; ++i) {
-        const int j = i / KB, kb = i - j * KB;
-        const int ut = u0 + 2 * j;
-        const int rows = (u1 - ut >= 2) ? 128 : 64;
-        mbar_expect_tx(&sm.full[i], static_cast<uint32_t>(rows * 128));
-        load_w_stage(sm.a + (size_t)i * kATileBytes, p.wpk, u0, j, rows, kb, p.H, &sm.full[i],
-                     pol_w);
+      {
+        int i = 0;
+        for (int g = 0; g < pl.n_groups && i < n_pre; ++g)
+          for (int kb = 0; kb < KB && i < n_pre; ++kb)
+            for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g) && i < n_pre;
+                 ++t, ++i) {
+              const uint32_t bytes = static_cast<uint32_t>(pl.tile_rows(t) * 128);
+              mbar_expect_tx(&sm.full_a[i], bytes);
+              bulk_load(sm.a + static_cast<size_t>(i) * kATileBytes,
+                        p.wpk + pl.stage_offset(g, kb, t, p.H), bytes, &sm.full_a[i], pol_w);
+            }
       }
       grid_dependency_wait();
       const int M = *p.d_M;
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
-      int stage = 0;
-      uint32_t phase = 0;
-      long long issued = 0;
+      Ring ra, rb;
+      long long a_issued = 0, b_issued = 0;
       bool ok = true;
       for (int q = 0; q < n_chunks && ok; ++q) {
         const int n0 = q * kChunkN;
         const int nq = (min(kChunkN, M - n0) + 15) & ~15;
-        for (int j = 0; j < n_tiles && ok; ++j) {
-          const int ut = u0 + 2 * j;
-          const int rows = (u1 - ut >= 2) ? 128 : 64;
-          for (int kb = 0; kb < KB; ++kb) {
-            const bool pre = issued < n_pre;  // A already in flight for this stage
-            if (!pre &&
-                !mbar_wait(&sm.empty[stage], phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
+        for (int g = 0; g < pl.n_groups && ok; ++g) {
+          for (int kb = 0; kb < KB && ok; ++kb) {
+            if (!mbar_wait(&sm.empty_b[rb.slot], rb.phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
               ok = false;
               break;
             }
-            mbar_arrive_expect_tx(&sm.full[stage],
-                                  static_cast<uint32_t>((pre ? 0 : rows * 128) + nq * 128));
-            if (!pre)
-              load_w_stage(sm.a + (size_t)stage * kATileBytes, p.wpk, u0, j, rows, kb, p.H,
-                           &sm.full[stage], pol_w);
-            uint8_t* bdst = sm.b + (size_t)stage * p.b_stage_bytes;
+            mbar_arrive_expect_tx(&sm.full_b[rb.slot], static_cast<uint32_t>(nq * 128));
+            uint8_t* bdst = sm.b + static_cast<size_t>(rb.slot) * p.b_slot_bytes;
             for (int i = 0; i < nq / kBoxRowsB; ++i)
-              tma_load_2d(bdst + i * kBoxRowsB * 128, &tm_h, &sm.full[stage], kb * kBlockK,
+              tma_load_2d(bdst + i * kBoxRowsB * 128, &tm_h, &sm.full_b[rb.slot], kb * kBlockK,
                           n0 + i * kBoxRowsB, pol_h);
-            ++issued;
-            if (++stage == p.n_stages) {
-              stage = 0;
-              phase ^= 1u;
+            ++b_issued;
+            rb.next(p.n_bslots);
+            for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
+              if (a_issued < n_pre) {
+                mbar_arrive(&sm.full_a[ra.slot]);  // copy already in flight
+              } else {
+                if (!mbar_wait(&sm.empty_a[ra.slot], ra.phase ^ 1u, sm.abort, p.err,
+                               kErrWaitEmpty)) {
+                  ok = false;
+                  break;
+                }
+                const uint32_t bytes = static_cast<uint32_t>(pl.tile_rows(t) * 128);
+                mbar_arrive_expect_tx(&sm.full_a[ra.slot], bytes);
+                bulk_load(sm.a + static_cast<size_t>(ra.slot) * kATileBytes,
+                          p.wpk + pl.stage_offset(g, kb, t, p.H), bytes, &sm.full_a[ra.slot],
+                          pol_w);
+              }
+              ++a_issued;
+              ra.next(p.n_stages);
             }
           }
         }
       }
-      if (issued < n_pre) {
+      if (a_issued < n_pre) {
         // Nothing to decode (M = 0) or an abort before the prefetched stages
         // were claimed: complete their phases so the W copies can be drained.
-        for (long long i = issued; i < n_pre; ++i) mbar_arrive(&sm.full[i]);
-        for (long long i = issued; i < n_pre; ++i) mbar_drain(&sm.full[i], 0, p.err);
+        for (long long i = a_issued; i < n_pre; ++i) mbar_arrive(&sm.full_a[i]);
+        for (long long i = a_issued; i < n_pre; ++i) mbar_drain(&sm.full_a[i], 0, p.err);
       }
       if (!ok) {
         // Abort path: let the copies already in flight land before exit.
-        const long long first = issued > p.n_stages ? issued - p.n_stages : 0;
-        for (long long i = first; i < issued; ++i)
-          mbar_drain(&sm.full[i % p.n_stages], static_cast<uint32_t>((i / p.n_stages) & 1),
+        const long long fa = a_issued > p.n_stages ? a_issued - p.n_stages : 0;
+        for (long long i = fa; i < a_issued; ++i)
+          mbar_drain(&sm.full_a[i % p.n_stages], static_cast<uint32_t>((i / p.n_stages) & 1),
+                     p.err);
+        const long long fb = b_issued > p.n_bslots ? b_issued - p.n_bslots : 0;
+        for (long long i = fb; i < b_issued; ++i)
+          mbar_drain(&sm.full_b[i % p.n_bslots], static_cast<uint32_t>((i / p.n_bslots) & 1),
                      p.err);
       }
     }
@@ -324,45 +424,52 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
       grid_dependency_wait();
       const int M = *p.d_M;
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
-      int stage = 0;
-      uint32_t phase = 0;
-      int acc = 0;
-      uint32_t acc_phase = 0;
+      Ring ra, rb, racc;
       bool ok = true;
       for (int q = 0; q < n_chunks && ok; ++q) {
         const int n0 = q * kChunkN;
         const int nq = (min(kChunkN, M - n0) + 15) & ~15;
         const uint32_t idesc = idesc_bf16_f32(kRowsPerTile, static_cast<uint32_t>(nq));
-        for (int j = 0; j < n_tiles && ok; ++j) {
-          if (!mbar_wait(&sm.acce[acc], acc_phase ^ 1u, sm.abort, p.err, kErrWaitAccEmpty)) {
+        for (int g = 0; g < pl.n_groups && ok; ++g) {
+          if (!mbar_wait(&sm.acce[racc.slot], racc.phase ^ 1u, sm.abort, p.err,
+                         kErrWaitAccEmpty)) {
             ok = false;
             break;
           }
           tc_fence_after();
-          const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * p.acc_stride);
-          for (int kb = 0; kb < KB; ++kb) {
-            if (!mbar_wait(&sm.full[stage], phase, sm.abort, p.err, kErrWaitFull)) {
+          const uint32_t d_group = tmem_base + static_cast<uint32_t>(racc.slot * group_cols);
+          for (int kb = 0; kb < KB && ok; ++kb) {
+            if (!mbar_wait(&sm.full_b[rb.slot], rb.phase, sm.abort, p.err, kErrWaitFull)) {
               ok = false;
               break;
             }
-            tc_fence_after();
-            const uint32_t a_addr = smem_addr(sm.a + (size_t)stage * kATileBytes);
-            const uint32_t b_addr = smem_addr(sm.b + (size_t)stage * p.b_stage_bytes);
+            const uint32_t b_addr =
+                smem_addr(sm.b + static_cast<size_t>(rb.slot) * p.b_slot_bytes);
+            for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
+              if (!mbar_wait(&sm.full_a[ra.slot], ra.phase, sm.abort, p.err, kErrWaitFull)) {
+                ok = false;
+                break;
+              }
+              tc_fence_after();
+              const uint32_t a_addr =
+                  smem_addr(sm.a + static_cast<size_t>(ra.slot) * kATileBytes);
+              const uint32_t d_tmem =
+                  d_group + static_cast<uint32_t>((t - pl.group_first(g)) * p.slot_cols);
 #pragma unroll
-            for (int kk = 0; kk < kBlockK / 16; ++kk) {
-              mma_bf16(d_tmem, sdesc_k_sw128(a_addr + kk * 32), sdesc_k_sw128(b_addr + kk * 32),
-                       idesc, (kb | kk) != 0 ? 1u : 0u);
+              for (int kk = 0; kk < kBlockK / 16; ++kk) {
+                mma_bf16(d_tmem, sdesc_k_sw128(a_addr + kk * 32), sdesc_k_sw128(b_addr + kk * 32),
+                         idesc, (kb | kk) != 0 ? 1u : 0u);
+              }
+              mma_commit(&sm.empty_a[ra.slot]);
+              ra.next(p.n_stages);
             }
-            mma_commit(&sm.empty[stage]);
-            if (++stage == p.n_stages) {
-              stage = 0;
-              phase ^= 1u;
-            }
+            if (!ok) break;
+            mma_commit(&sm.empty_b[rb.slot]);
+            rb.next(p.n_bslots);
           }
           if (!ok) break;
-          mma_commit(&sm.accf[acc]);
-          acc ^= 1;
-          if (acc == 0) acc_phase ^= 1u;
+          mma_commit(&sm.accf[racc.slot]);
+          racc.next(2);
         }
       }
       if (!ok) {
@@ -381,8 +488,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
-    int acc = 0;
-    uint32_t acc_phase = 0;
+    Ring racc;
     bool ok = true;
     for (int q = 0; q < n_chunks && ok; ++q) {
       const int n0 = q * kChunkN;
@@ -391,40 +497,88 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
       float rm[8], rs[8];
       int ri[8];
 #pragma unroll
-      for (int g = 0; g < 8; ++g) {
-        rm[g] = kNegBig;
-        rs[g] = 0.0f;
-        ri[g] = INT_MAX;
+      for (int c = 0; c < 8; ++c) {
+        rm[c] = kNegBig;
+        rs[c] = 0.0f;
+        ri[c] = INT_MAX;
       }
-      for (int j = 0; j < n_tiles; ++j) {
-        const int ut = u0 + 2 * j;
-        const int rows = (u1 - ut >= 2) ? 128 : 64;
-        const int row_local = quarter * 32 + lane;
-        const int vrow = ut * kUnitRows + row_local;
-        const bool valid = row_local < rows && vrow < p.V;
-        if (!mbar_wait(&sm.accf[acc], acc_phase, sm.abort, p.err, kErrWaitAccFull)) {
-          ok = false;
-          break;
-        }
-        tc_fence_after();
-        const uint32_t tcol = tmem_base + lane_base + static_cast<uint32_t>(acc * p.acc_stride);
+      if (ngroups == 1) {
+        // Up to 32 positions: each lane folds its own row of every tile into a
+        // running triple per column (one exponential per logit, no shuffles);
+        // the 32 lanes are merged once, after the last tile.
+        float lm[32], ls[32];
+        int li[32];
 #pragma unroll
-        for (int g = 0; g < 8; ++g) {
-          if (g < ngroups) {
-            uint32_t v[32];
-            tmem_ld_32cols(tcol + 32 * g, v);
-            tmem_ld_wait();
-            float m, s;
-            int i;
-            transpose_reduce32(v, valid, vrow, lane, m, s, i);
-            merge_tri(rm[g], rs[g], ri[g], m, s, i);
-          }
+        for (int c = 0; c < 32; ++c) {
+          lm[c] = kNegBig;
+          ls[c] = 0.0f;
+          li[c] = INT_MAX;
         }
-        tc_fence_before();
-        __syncwarp();
-        if (lane == 0) mbar_arrive(&sm.acce[acc]);
-        acc ^= 1;
-        if (acc == 0) acc_phase ^= 1u;
+        for (int g = 0; g < pl.n_groups; ++g) {
+          if (!mbar_wait(&sm.accf[racc.slot], racc.phase, sm.abort, p.err, kErrWaitAccFull)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t tgroup =
+              tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
+          for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
+            const int row_local = quarter * 32 + lane;
+            const int vrow = (pl.u0 + 2 * t) * kUnitRows + row_local;
+            const bool valid = row_local < pl.tile_rows(t) && vrow < p.V;
+            uint32_t v[32];
+            tmem_ld_32cols(tgroup + static_cast<uint32_t>((t - pl.group_first(g)) * p.slot_cols),
+                           v);
+            tmem_ld_wait();
+            if (valid) {
+#pragma unroll
+              for (int c = 0; c < 32; ++c)
+                online_update(lm[c], ls[c], li[c], __uint_as_float(v[c]) * kLog2e, vrow);
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.acce[racc.slot]);
+          racc.next(2);
+        }
+        if (!ok) break;
+        transpose_merge32(lm, ls, li, lane);
+        rm[0] = lm[0];
+        rs[0] = ls[0];
+        ri[0] = li[0];
+      } else {
+        for (int g = 0; g < pl.n_groups; ++g) {
+          if (!mbar_wait(&sm.accf[racc.slot], racc.phase, sm.abort, p.err, kErrWaitAccFull)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t tgroup =
+              tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
+          for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
+            const int row_local = quarter * 32 + lane;
+            const int vrow = (pl.u0 + 2 * t) * kUnitRows + row_local;
+            const bool valid = row_local < pl.tile_rows(t) && vrow < p.V;
+            const uint32_t tcol =
+                tgroup + static_cast<uint32_t>((t - pl.group_first(g)) * p.slot_cols);
+#pragma unroll
+            for (int c = 0; c < 8; ++c) {
+              if (c < ngroups) {
+                uint32_t v[32];
+                tmem_ld_32cols(tcol + 32 * c, v);
+                tmem_ld_wait();
+                float m, s;
+                int i;
+                transpose_reduce32(v, valid, vrow, lane, m, s, i);
+                merge_tri(rm[c], rs[c], ri[c], m, s, i);
+              }
+            }
+          }
+          tc_fence_before();
+          __syncwarp();
+          if (lane == 0) mbar_arrive(&sm.acce[racc.slot]);
+          racc.next(2);
+        }
       }
       if (!ok) break;
       // Cross-warp merge of the four 32-row slices of every column, then one
@@ -432,12 +586,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
       // writes buffer q & 1 again only after every warp arrived for chunk q + 1,
       // which each does after reading chunk q.
       const int buf = q & 1;
-      float4* epi = sm.epi + buf * 4 * p.acc_stride;
+      float4* epi = sm.epi + buf * 4 * p.slot_cols;
 #pragma unroll
-      for (int g = 0; g < 8; ++g) {
-        if (g < ngroups)
-          epi[ew * p.acc_stride + 32 * g + lane] =
-              make_float4(rm[g], rs[g], __int_as_float(ri[g]), 0.0f);
+      for (int c = 0; c < 8; ++c) {
+        if (c < ngroups)
+          epi[ew * p.slot_cols + 32 * c + lane] =
+              make_float4(rm[c], rs[c], __int_as_float(ri[c]), 0.0f);
       }
       __syncwarp();
       if (lane == 0) mbar_arrive(&sm.epib[buf]);
@@ -453,7 +607,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         int i = __float_as_int(a.z);
 #pragma unroll
         for (int w = 1; w < 4; ++w) {
-          const float4 b = epi[w * p.acc_stride + col];
+          const float4 b = epi[w * p.slot_cols + col];
           merge_tri(m, s, i, b.x, b.y, __float_as_int(b.z));
         }
         p.part[static_cast<size_t>(n0 + col) * G + cta] = make_float4(m, s, __int_as_float(i), 0.0f);

@@ -25,7 +25,7 @@ constexpr int kMaxP = 256;
 constexpr int kGatherRowsPerCta = 4;
 constexpr int kGatherThreads = 256;
 constexpr int kCommitThreads = 256;  // merge kernel: small enough to share an SM with the LM head
-constexpr int kPosPerWarp = 4;       // positions whose partials a warp loads at once
+constexpr int kPosPerWarp = 2;       // positions whose partials a warp loads at once
 constexpr int kPartPerLane = 5;      // partial slots a lane loads per position (G <= 160)
 
 // Host-visible record of the last committed step, one 64-bit word in mapped

@@ -173,6 +173,19 @@ def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0):
                       f"fp64, one thread per row), {dt:.1f} s"}
 
 
+def aggregate(ms: float, positions: int, dist=None, device=None):
+    """Whole-job figures over ranks: the slowest rank's time and the sum of
+    every rank's decoded positions (each rank decodes its own batch)."""
+    if dist is None:
+        return ms, positions
+    import torch
+    t = torch.tensor([ms], dtype=torch.float64, device=device)
+    n = torch.tensor([positions], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    dist.all_reduce(n, op=dist.ReduceOp.SUM)
+    return float(t.item()), int(n.item())
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -275,11 +288,7 @@ def main():
         head_launches = stats2["head_launches"] - stats1["head_launches"]
         head_ms = stats2["head_ms"] - stats1["head_ms"]
 
-    if dist:
-        t = torch.tensor([ms], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        ms = float(t.item())
-    total_positions = positions * args.steps * world
+    ms, total_positions = aggregate(ms, positions * args.steps, dist, dev)
     value = total_positions / (ms / 1e3)
 
     # Roofline of the dominant kernel (LM head): algorithmic bytes of every
@@ -299,6 +308,9 @@ def main():
                 "frac": round(achieved / hbm, 4),
                 "traffic": (tr["dram_bytes_per_launch"] if tr and tr.get("workload") == wl.name
                             else None),
+                "traffic_basis": ("ncu dram read+write of one full-mask launch; algorithmic bytes "
+                                  "of that launch %d" % tr["algorithmic_bytes_of_profiled_launch"])
+                                 if tr and tr.get("workload") == wl.name else None,
                 "algorithmic_bytes_per_launch": round(alg_bytes / max(1, head_launches)),
                 "kernel": "lm_head_softmax_kernel", "peak_source": f"{peak_kind} hbm_gbs",
                 "head_launches": head_launches, "head_ms_total": round(head_ms, 3),
@@ -365,14 +377,8 @@ def e2e_run(cai, ctx, hs, wl, args, dist, dev):
     dt = time.perf_counter() - t0
     st = cai.cai_state_download(ctx)
     n_step_calls = (cai.cai_get_stats(ctx)["steps"] - s0) / steps
-    world = 1
-    if dist:
-        t = torch.tensor([dt], device=dev)
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-        dt = float(t.item())
-        world = dist.get_world_size()
-    positions = int(st["m_hist"].sum())
-    return {"value": round(positions * steps * world / dt, 1), "unit": UNIT,
+    dt_ms, positions = aggregate(dt * 1e3, int(st["m_hist"].sum()) * steps, dist, dev)
+    return {"value": round(positions / (dt_ms / 1e3), 1), "unit": UNIT,
             "h2d_bytes_per_step": int(n_step_calls * wl.B * wl.P * wl.H * 2),
             "d2h_bytes_per_step": int(wl.B * wl.n_blocks * wl.P * 4 + n_step_calls * 32),
             "timing": "host wall clock around whole generations, pinned host inputs"}

@@ -61,6 +61,8 @@ WORKLOADS = {
 # (kappa, gamma) per (V, H), written by oracle/calibrate_synth.py.
 CALIBRATED: dict[tuple[int, int], tuple[float, float]] = {
     (4096, 256): (12.494524, 3.125000),
+    (126464, 4096): (3.612477, 0.781250),
+    (152064, 3584): (3.891420, 0.835191),
 }
 
 

@@ -1,0 +1,136 @@
+"""The C ABI on a machine without a GPU: the library loads, exports exactly
+what include/cai.h declares, its structs have the header's layout, and
+argument / shape validation answers before any CUDA call."""
+import ctypes
+import os
+import re
+import subprocess
+import tempfile
+
+import pytest
+
+import paper_2608_22646_gb300 as cai
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "cai.h")
+
+
+@pytest.fixture(scope="module", autouse=True)
+def built():
+    from paper_2608_22646_gb300 import build
+    build.build()
+
+
+def _declared():
+    src = open(HEADER).read()
+    src = re.sub(r"/\*.*?\*/", "", src, flags=re.S)
+    return sorted(set(re.findall(r"\b(cai_[a-z0-9_]+)\s*\(", src)))
+
+
+def test_exports_match_header():
+    names = _declared()
+    assert names == sorted(cai.EXPORTS), (names, sorted(cai.EXPORTS))
+    lib = cai.lib()
+    for n in names:
+        assert hasattr(lib, n), n
+    out = subprocess.run(["nm", "-D", "--defined-only", cai.LIB_PATH], capture_output=True,
+                         text=True, check=True).stdout
+    exported = set(re.findall(r"\bT (cai_[a-z0-9_]+)$", out, flags=re.M))
+    assert set(names) <= exported
+
+
+def _c_layout():
+    """sizeof/offsetof of the ABI structs as a C compiler sees the header."""
+    prog = r'''
+#include <stddef.h>
+#include <stdio.h>
+#include "cai.h"
+#define F(T, f) printf(#T "." #f " %zu\n", offsetof(T, f));
+int main(void) {
+  printf("cai_config %zu\ncai_state_view %zu\ncai_host_state %zu\ncai_stats %zu\n",
+         sizeof(cai_config), sizeof(cai_state_view), sizeof(cai_host_state), sizeof(cai_stats));
+  F(cai_config, theta_s) F(cai_config, warmup_pct) F(cai_config, theta_fb) F(cai_config, eta_bar)
+  F(cai_config, eta_mode) F(cai_config, flags)
+  F(cai_host_state, m_hist) F(cai_host_state, blk) F(cai_host_state, t_next)
+  F(cai_stats, head_ms) F(cai_stats, grid) F(cai_stats, n_max)
+  return 0;
+}
+'''
+    with tempfile.TemporaryDirectory() as d:
+        c = os.path.join(d, "l.c")
+        open(c, "w").write(prog)
+        exe = os.path.join(d, "l")
+        subprocess.check_call(["gcc", "-std=c99", "-I", os.path.dirname(HEADER), c, "-o", exe])
+        out = subprocess.run([exe], capture_output=True, text=True, check=True).stdout
+    return dict(line.rsplit(" ", 1) for line in out.strip().splitlines())
+
+
+def test_struct_layout_matches_binding():
+    lay = {k: int(v) for k, v in _c_layout().items()}
+    assert lay["cai_config"] == ctypes.sizeof(cai.cai_config)
+    assert lay["cai_state_view"] == ctypes.sizeof(cai.cai_state_view)
+    assert lay["cai_host_state"] == ctypes.sizeof(cai.cai_host_state)
+    assert lay["cai_stats"] == ctypes.sizeof(cai.cai_stats)
+    for key, v in lay.items():
+        if "." in key:
+            s, f = key.split(".")
+            assert getattr(getattr(cai, s), f).offset == v, key
+
+
+def test_config_default_values():
+    c = cai.cai_config_default(cai.CAI_PRESET_LLADA, 1, 32, 4096, 126464, 32, 8)
+    assert (c.theta_s, c.theta_e1, c.theta_e_step, c.theta_e_min) == (0.9, 0.7, 0.1, 0.4)
+    assert (c.warmup_pct, c.K, c.theta_fb, c.clip_lo, c.clip_hi, c.eta_bar) == \
+        (15, 4, 0.4, 0.2, 0.98, 1.5)
+    assert c.flags == cai.CAI_GATING | cai.CAI_POS_FACTOR
+    d = cai.cai_config_default(cai.CAI_PRESET_DREAM, 1, 32, 3584, 152064, 32, 8)
+    assert d.flags == cai.CAI_POS_FACTOR
+    with pytest.raises(cai.CaiError) as e:
+        cai.cai_config_default(7, 1, 1, 64, 64, 1, 1)
+    assert e.value.status == cai.CAI_ERR_ARG
+
+
+@pytest.mark.parametrize("field,value,status", [
+    ("H", 100, cai.CAI_ERR_SHAPE),      # H % 64 != 0
+    ("P", 300, cai.CAI_ERR_SHAPE),      # P > 256
+    ("V", 32, cai.CAI_ERR_SHAPE),       # V < 64
+    ("B", 0, cai.CAI_ERR_SHAPE),
+    ("T", 0, cai.CAI_ERR_SHAPE),
+    ("n_blocks", 40000, cai.CAI_ERR_SHAPE),
+    ("K", 0, cai.CAI_ERR_ARG),
+    ("eta_mode", 2, cai.CAI_ERR_ARG),
+    ("flags", 1 << 7, cai.CAI_ERR_ARG),
+])
+def test_init_validates_before_any_cuda_call(field, value, status):
+    c = cai.cai_config_default(0, 1, 16, 256, 4096, 8, 4)
+    setattr(c, field, value)
+    w = (ctypes.c_uint16 * 16)()
+    h = ctypes.c_void_p()
+    assert cai.lib().cai_init(ctypes.byref(c), ctypes.addressof(w), None, ctypes.byref(h)) == status
+    assert not h.value
+
+
+def test_null_and_status_strings():
+    lib = cai.lib()
+    h = ctypes.c_void_p()
+    assert lib.cai_init(None, None, None, ctypes.byref(h)) == cai.CAI_ERR_ARG
+    for fn in ("cai_first_step", "cai_denoise_step"):
+        assert getattr(lib, fn)(None, None, None) == cai.CAI_ERR_ARG
+    assert lib.cai_block_advance(None, None) == cai.CAI_ERR_ARG
+    lib.cai_free(None)
+    for s in range(-8, 1):
+        assert cai.cai_strerror(s) != "unknown status"
+    assert cai.cai_strerror(-99) == "unknown status"
+    assert lib.cai_test_fail_alloc_after(-1) == cai.CAI_ERR_ARG
+    assert lib.cai_test_head_grid_limit(-1) == cai.CAI_ERR_ARG
+
+
+def test_no_device_is_a_status_not_a_crash():
+    import torch
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present")
+    c = cai.cai_config_default(0, 1, 16, 256, 4096, 8, 4)
+    w = (ctypes.c_uint16 * (4096 * 256))()
+    h = ctypes.c_void_p()
+    r = cai.lib().cai_init(ctypes.byref(c), ctypes.addressof(w), None, ctypes.byref(h))
+    assert r in (cai.CAI_ERR_CUDA, cai.CAI_ERR_UNSUPPORTED) and not h.value

@@ -241,6 +241,34 @@ int cai_get_stats(cai_ctx* ctx, cai_stats* out);
  * NULL is a no-op. */
 void cai_free(cai_ctx* ctx);
 
+/*
+ * Decoding head over caller rows without allocating anything.  The paper has
+ * no counterpart: this is a convenience for callers that cannot call
+ * cudaMalloc where they need the head (a memory pool that owns the whole
+ * device, an allocator-free runtime that reserved everything up front, a
+ * region where an allocation would synchronise the device).  No context is
+ * needed and nothing is allocated: no cudaMalloc, cudaFree or allocating
+ * library call.
+ *
+ * For each of the M rows of `rows` ([M, H] bf16, device), computes
+ * conf[i] = max_v softmax(W rows[i])_v and argmax[i] = the lowest v reaching
+ * that maximum, against the caller's W ([V, H] bf16 row-major, device, read in
+ * place).  conf (float) and argmax (int32) are device arrays of M entries.
+ * Asynchronous on `stream`.  Limits: 1 <= M <= 256, V >= 128, H % 64 == 0 and
+ * 64 <= H <= 16384; pointers 16-byte aligned (else CAI_ERR_SHAPE / CAI_ERR_ARG).
+ *
+ * Scratch: a fixed file-scope device array of 256 x 160 partial triples
+ * (640 KiB) plus an error word, held by every GPU that loads this library until
+ * the process exits, shared by all calls and keeping the last call's
+ * contents.  Calls that overlap on the GPU (on different streams, or from
+ * different threads) race on it.  The first call on each device looks up the
+ * array's device address and sets the kernel's shared-memory limit, with that
+ * device current; make that first call before any stream capture.  If a
+ * kernel-side bounded wait gives up, that call's outputs are NaN / -1.
+ */
+int cai_head_rows_static(const void* W, int32_t V, int32_t H, const void* rows, int32_t M,
+                         float* conf, int32_t* argmax, void* stream);
+
 /* Static string for a status code. */
 const char* cai_strerror(int status);
 

@@ -46,7 +46,8 @@ CAI_RUNNING, CAI_EXIT_DONE, CAI_EXIT_GRIND, CAI_EXIT_TMAX = 0, 1, 2, 3
 EXPORTS = ("cai_config_default", "cai_init", "cai_first_step", "cai_denoise_step",
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
-           "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit")
+           "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
+           "cai_head_rows_static")
 
 
 class CaiError(RuntimeError):
@@ -110,6 +111,7 @@ def _load():
         "cai_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
         "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
+        "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -273,6 +275,16 @@ def cai_test_fail_alloc_after(n: int) -> None:
 
 def cai_test_head_grid_limit(n: int) -> None:
     _check(lib().cai_test_head_grid_limit(n), "cai_test_head_grid_limit")
+
+
+def cai_head_rows_static(W, rows, conf, argmax, stream=None) -> None:
+    """Confidence and argmax of every row of ``rows`` [M, H] against ``W`` [V, H]
+    into the device arrays ``conf`` (float32 [M]) and ``argmax`` (int32 [M]),
+    allocating nothing (see include/cai.h)."""
+    V, H = W.shape
+    M = rows.shape[0]
+    _check(lib().cai_head_rows_static(_ptr(W), V, H, _ptr(rows), M, _ptr(conf), _ptr(argmax),
+                                      _stream(stream)), "cai_head_rows_static")
 
 
 def config_from_dict(d: dict) -> cai_config:

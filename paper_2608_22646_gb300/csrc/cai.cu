@@ -781,3 +781,6 @@ int cai_test_fail_alloc_after(int32_t n) {
 }
 
 }  // extern "C"
+
+// The allocation-free decoding head (cai_head_rows_static).
+#include "static_head.cuh"

@@ -291,19 +291,28 @@ def main():
     ms, total_positions = aggregate(ms, positions * args.steps, dist, dev)
     value = total_positions / (ms / 1e3)
 
-    # Roofline of the dominant kernel (LM head): algorithmic bytes of every
-    # launch = W once (2 V H, only when it decodes rows) + the masked rows (2 M H).
+    # Roofline of the dominant kernel (LM head), launch by launch: a launch
+    # that decodes M rows reads 2 V H + 2 M H bytes (W once, the rows once) and
+    # does 2 M V H flops; its roof is the slower of the two at the measured
+    # peaks.  Launches of empty steps (M = 0) have no algorithmic work.
     hbm, tf_burst, tf_sus, peak_kind = _peaks()
-    alg_bytes = args.steps * (nonzero_launch * 2.0 * wl.V * wl.H + positions * 2.0 * wl.H)
-    alg_flops = args.steps * positions * 2.0 * wl.V * wl.H
-    head_s = max(head_ms, 1e-9) / 1e3
-    mean_m = positions / max(1, nonzero_launch)
-    # ridge: a launch reads 2 V H bytes and does 2 M V H flops, so it is
-    # HBM-bound while M < tensor peak / HBM peak (about 280 positions)
-    bound = "hbm" if mean_m < tf_burst * 1e12 / (hbm * 1e9) else "tensor"
+    tf = tf_sus or tf_burst
+    m_t = [int(x) for x in st0["m_hist"].reshape(-1) if x > 0]
+    bytes_t = [2.0 * wl.V * wl.H + 2.0 * m * wl.H for m in m_t]
+    flops_t = [2.0 * m * wl.V * wl.H for m in m_t]
+    t_hbm = sum(b / (hbm * 1e9) for b in bytes_t)
+    t_tc = sum(f / (tf * 1e12) for f in flops_t)
+    t_roof = sum(max(b / (hbm * 1e9), f / (tf * 1e12)) for b, f in zip(bytes_t, flops_t))
+    head_s = max(head_ms, 1e-9) / 1e3 / args.steps       # LM-head time per generation
     tr = _traffic_record(os.path.join(ROOT, "paper_2608_22646_gb300", "csrc", "head_kernel.cuh"))
-    if bound == "hbm":
-        achieved = alg_bytes / head_s / 1e9
+    per_launch = max(1, head_launches // max(1, args.steps))
+    common = {"kernel": "lm_head_softmax_kernel", "head_launches": head_launches,
+              "head_ms_total": round(head_ms, 3),
+              "roofline_time_frac": round(t_roof / head_s, 4),
+              "timing": "CUDA events around every LM-head launch, second pass of the same "
+                        "K generations"}
+    if t_hbm >= t_tc:
+        achieved = sum(bytes_t) / head_s / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(achieved / hbm, 4),
                 "traffic": (tr["dram_bytes_per_launch"] if tr and tr.get("workload") == wl.name
@@ -311,20 +320,14 @@ def main():
                 "traffic_basis": ("ncu dram read+write of one full-mask launch; algorithmic bytes "
                                   "of that launch %d" % tr["algorithmic_bytes_of_profiled_launch"])
                                  if tr and tr.get("workload") == wl.name else None,
-                "algorithmic_bytes_per_launch": round(alg_bytes / max(1, head_launches)),
-                "kernel": "lm_head_softmax_kernel", "peak_source": f"{peak_kind} hbm_gbs",
-                "head_launches": head_launches, "head_ms_total": round(head_ms, 3),
-                "timing": "CUDA events around every LM-head launch, second pass of the same "
-                          "K generations"}
+                "algorithmic_bytes_per_launch": round(sum(bytes_t) / per_launch),
+                "peak_source": f"{peak_kind} hbm_gbs", **common}
     else:
-        achieved = alg_flops / head_s / 1e12
-        pk = tf_sus or tf_burst
-        roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": pk, "unit": "TFLOP/s",
-                "frac": round(achieved / pk, 4), "traffic": None,
-                "kernel": "lm_head_softmax_kernel", "peak_source": f"{peak_kind} bf16 sustained",
-                "head_launches": head_launches, "head_ms_total": round(head_ms, 3),
-                "timing": "CUDA events around every LM-head launch, second pass of the same "
-                          "K generations"}
+        achieved = sum(flops_t) / head_s / 1e12
+        roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": tf,
+                "unit": "TFLOP/s", "frac": round(achieved / tf, 4), "traffic": None,
+                "algorithmic_flops_per_launch": round(sum(flops_t) / per_launch),
+                "peak_source": f"{peak_kind} bf16 sustained", **common}
 
     line = {
         "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,

@@ -156,7 +156,7 @@ typedef struct cai_stats {
   int32_t grid;             /* CTAs of the LM-head kernel                          */
   int32_t stages;           /* pipeline stages of the LM-head kernel               */
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
-  int32_t reserved;
+  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 256), else 3          */
 } cai_stats;
 
 /* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")

@@ -85,7 +85,8 @@ class cai_stats(ctypes.Structure):
     _fields_ = [("steps", ctypes.c_int64), ("launches", ctypes.c_int64),
                 ("head_launches", ctypes.c_int64), ("head_ms", ctypes.c_double),
                 ("head_profiled", ctypes.c_int64), ("grid", ctypes.c_int32),
-                ("stages", ctypes.c_int32), ("n_max", ctypes.c_int32), ("reserved", ctypes.c_int32)]
+                ("stages", ctypes.c_int32), ("n_max", ctypes.c_int32),
+                ("kernels_per_step", ctypes.c_int32)]
 
 
 def _load():

@@ -148,7 +148,10 @@ struct cai_ctx {
   HostFlag* hf_host = nullptr;
   HostFlag* hf_dev = nullptr;
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
-  CUtensorMap tm_h{};
+  CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
+  CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
+  const void* hid_mapped = nullptr;
+  bool fused = false;    // single-kernel step (B P <= 256)
   int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
   int b_slot_bytes = 0;
   size_t head_smem = 0;
@@ -235,77 +238,17 @@ double pos_factor_of(const cai_config& c, int p) {
   return p < q1 ? 0.80 : p < q2 ? 0.90 : p < q3 ? 1.05 : 1.10;
 }
 
-int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
-  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   const cai_config& cfg = c->cfg;
-  const void* hid = hidden;
-  if (!is_device_ptr(hidden)) {
-    if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
-                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
-      return fail(c, CAI_ERR_CUDA);
-    hid = c->hidden_stage;
-  }
-  const int t = c->t_next;
-  const int64_t step_id = c->last_step_id + 1;
-
-  GatherParams gp{};
-  gp.hidden = static_cast<const __nv_bfloat16*>(hid);
-  gp.hc = c->hc;
-  gp.list = c->list;
-  gp.row_of = c->row_of;
-  gp.d_M = c->d_M;
-  gp.B = cfg.B;
-  gp.BP = c->BP;
-  gp.H = cfg.H;
-  gp.first = first ? 1 : 0;
-  const int g_grid = c->rows_cap / kGatherRowsPerCta;
-  if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) != cudaSuccess)
-    return check_launch(c);
-  c->stats.launches++;
-
-  HeadParams hp{};
-  hp.wpk = static_cast<const uint8_t*>(c->wpk);
-  hp.d_M = c->d_M;
-  hp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
-  hp.part = c->part;
-  hp.err = c->err;
-  hp.V = cfg.V;
-  hp.H = cfg.H;
-  hp.units = (cfg.V + kUnitRows - 1) / kUnitRows;
-  hp.n_stages = c->n_stages;
-  hp.n_bslots = c->n_bslots;
-  hp.b_slot_bytes = c->b_slot_bytes;
-  hp.slot_cols = c->slot_cols;
-  hp.gmax = c->gmax;
-  hp.tmem_cols = c->tmem_cols;
-  cudaEvent_t e0 = nullptr, e1 = nullptr;
-  if (c->profiling) {
-    if (c->ev_used + 2 > c->ev_pool.size()) {
-      for (int k = 0; k < 2; ++k) {
-        cudaEvent_t e;
-        if (cudaEventCreate(&e) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
-        c->ev_pool.push_back(e);
-      }
-    }
-    e0 = c->ev_pool[c->ev_used];
-    e1 = c->ev_pool[c->ev_used + 1];
-    c->ev_used += 2;
-    cudaEventRecord(e0, stream);
-  }
-  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream, c->tm_h,
-                 hp) != cudaSuccess)
-    return check_launch(c);
-  if (c->profiling) cudaEventRecord(e1, stream);
-  c->stats.launches++;
-  c->stats.head_launches++;
-
   CommitParams cp{};
   cp.part = c->part;
   cp.n_part = c->G;
+  cp.identity_rows = c->fused ? 1 : 0;
   cp.st = c->st;
   cp.list = c->list;
   cp.row_of = c->row_of;
   cp.d_M = c->d_M;
+  cp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
   cp.ticket = c->ticket;
   cp.hf = c->hf_dev;
   cp.err = c->err;
@@ -331,10 +274,95 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     th = th > cfg.clip_hi ? cfg.clip_hi : th;
     cp.theta_tab[p] = static_cast<float>(th);
   }
-  const int commit_threads = cfg.P < kCommitThreads / 32 ? 32 * cfg.P : kCommitThreads;
-  if (launch_pdl(c->pdl, merge_commit_kernel, cfg.B, commit_threads, 0, stream, cp) != cudaSuccess)
+  return cp;
+}
+
+// One denoising step.  Single-kernel step (B P <= 256): the LM-head kernel
+// reads the hidden states in place and its last CTA commits.  Otherwise:
+// gather -> LM head -> merge + commit.
+int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  const cai_config& cfg = c->cfg;
+  const void* hid = hidden;
+  if (!is_device_ptr(hidden)) {
+    if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
+                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
+      return fail(c, CAI_ERR_CUDA);
+    hid = c->hidden_stage;
+  }
+  const int t = c->t_next;
+  const int64_t step_id = c->last_step_id + 1;
+
+  if (!c->fused) {
+    GatherParams gp{};
+    gp.hidden = static_cast<const __nv_bfloat16*>(hid);
+    gp.hc = c->hc;
+    gp.list = c->list;
+    gp.row_of = c->row_of;
+    gp.d_M = c->d_M;
+    gp.B = cfg.B;
+    gp.BP = c->BP;
+    gp.H = cfg.H;
+    gp.first = first ? 1 : 0;
+    const int g_grid = c->rows_cap / kGatherRowsPerCta;
+    if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) !=
+        cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
+  } else if (hid != c->hid_mapped) {
+    // The single-kernel step reads the caller's [B P, H] rows through TMA.
+    if (!make_map(&c->tm_hid, hid, c->BP, cfg.H, kBoxRowsB)) return CAI_ERR_ARG;
+    c->hid_mapped = hid;
+  }
+
+  HeadParams hp{};
+  hp.wpk = static_cast<const uint8_t*>(c->wpk);
+  hp.d_M = c->d_M;
+  hp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
+  hp.fused = c->fused ? 1 : 0;
+  hp.M_fixed = c->BP;
+  hp.first = first ? 1 : 0;
+  hp.part = c->part;
+  hp.err = c->err;
+  hp.V = cfg.V;
+  hp.H = cfg.H;
+  hp.units = (cfg.V + kUnitRows - 1) / kUnitRows;
+  hp.n_stages = c->n_stages;
+  hp.n_bslots = c->n_bslots;
+  hp.b_slot_bytes = c->b_slot_bytes;
+  hp.slot_cols = c->slot_cols;
+  hp.gmax = c->gmax;
+  hp.tmem_cols = c->tmem_cols;
+  const CommitParams cp = commit_params(c, t, step_id);
+  if (c->fused) hp.cp = cp;
+  cudaEvent_t e0 = nullptr, e1 = nullptr;
+  if (c->profiling) {
+    if (c->ev_used + 2 > c->ev_pool.size()) {
+      for (int k = 0; k < 2; ++k) {
+        cudaEvent_t e;
+        if (cudaEventCreate(&e) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+        c->ev_pool.push_back(e);
+      }
+    }
+    e0 = c->ev_pool[c->ev_used];
+    e1 = c->ev_pool[c->ev_used + 1];
+    c->ev_used += 2;
+    cudaEventRecord(e0, stream);
+  }
+  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream,
+                 c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
     return check_launch(c);
+  if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.launches++;
+  c->stats.head_launches++;
+
+  if (!c->fused) {
+    const int commit_threads = cfg.P < kCommitThreads / 32 ? 32 * cfg.P : kCommitThreads;
+    if (launch_pdl(c->pdl, merge_commit_kernel, cfg.B, commit_threads, 0, stream, cp) !=
+        cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
+  }
   c->stats.steps++;
   int r = check_launch(c);
   if (r != CAI_OK) return r;
@@ -399,6 +427,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->BP = cfg->B * cfg->P;
   c->rows_cap = round_up(c->BP, 16);
   c->pdl = pdl_enabled();
+  c->fused = c->BP <= kChunkN;
 
   // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
   // at most one per 64-row unit), tile group size (tiles sharing one hidden
@@ -407,7 +436,11 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
   c->slot_cols = round_up(c->n_max, 32);
   const int units = (cfg->V + kUnitRows - 1) / kUnitRows;
-  c->G = units < sms ? units : sms;
+  // Single-kernel step: one SM is left to the CTA that commits the step, so
+  // the next step's CTAs all find a free SM instead of one of them waiting
+  // for the commit to finish (and becoming the next step's straggler).
+  const int usable_sms = c->fused && sms > 1 ? sms - 1 : sms;
+  c->G = units < usable_sms ? units : usable_sms;
   const int glim = g_head_grid_limit.load();
   if (glim > 0 && c->G > glim) c->G = glim;
   const int max_units = (units + c->G - 1) / c->G;
@@ -430,10 +463,18 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     const int per = c->gmax > 1 ? c->gmax - 1 : 1;
     return c->gmax == 1 ? stages : (stages + per - 1) / per + 1;
   };
+  // Dynamic shared memory may use what the kernel's static shared memory leaves.
+  cudaFuncAttributes head_attr{};
+  if (cudaFuncGetAttributes(&head_attr, lm_head_softmax_kernel) != cudaSuccess) {
+    cudaGetLastError();
+    delete c;
+    return CAI_ERR_CUDA;
+  }
+  const size_t dyn_limit = static_cast<size_t>(smem_optin) - head_attr.sharedSizeBytes;
   const int scap = env_int("CAI_HEAD_STAGES");
   int stages = scap >= 2 && scap < 12 ? scap : 12;
   while (stages > 2 && head_smem_bytes(stages, bslots_for(stages), c->b_slot_bytes,
-                                       c->slot_cols) > static_cast<size_t>(smem_optin))
+                                       c->slot_cols) > dyn_limit)
     --stages;
   c->n_stages = stages;
   c->n_bslots = bslots_for(stages);
@@ -517,8 +558,19 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     delete c;
     return CAI_ERR_CUDA;
   }
+  // All step kernels ask for the same (largest) shared-memory carveout, so the
+  // small gather and merge CTAs can be resident on an SM beside an LM-head
+  // CTA; under programmatic dependent launch they then start, and wait, while
+  // the neighbouring kernel still runs.
   if (cudaFuncSetAttribute(lm_head_softmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                           static_cast<int>(c->head_smem)) != cudaSuccess) {
+                           static_cast<int>(c->head_smem)) != cudaSuccess ||
+      cudaFuncSetAttribute(lm_head_softmax_kernel,
+                           cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess ||
+      cudaFuncSetAttribute(gather_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess ||
+      cudaFuncSetAttribute(merge_commit_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                           cudaSharedmemCarveoutMaxShared) != cudaSuccess) {
     cudaGetLastError();
     release(c);
     delete c;
@@ -527,6 +579,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->stats.grid = c->G;
   c->stats.stages = c->n_stages;
   c->stats.n_max = c->n_max;
+  c->stats.kernels_per_step = c->fused ? 1 : 3;
   r = cai_reset(c, stream);
   if (r != CAI_OK) {
     release(c);

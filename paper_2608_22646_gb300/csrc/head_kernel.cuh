@@ -29,6 +29,14 @@
 // contiguous copies keep DRAM pages open, the strided 128-byte rows of a 2-D
 // tensor box do not.
 //
+// Single-kernel step (fused = 1, used when B P <= 256): the kernel decodes all
+// B P rows straight from the caller's hidden states (no gather; at N <= 256 a
+// step reads W once whatever N is), and the last CTA to finish (atomic
+// ticket, no waiting) merges the partials and applies the commit rule for
+// every sequence (commit.cuh).  A step is then one launch, and under
+// programmatic dependent launch the next step's prologue and first W stages
+// overlap this step's commit.
+//
 // Warp roles (192 threads, one CTA per SM):
 //   warp 0      producer (one lane): W stages (bulk copies), hidden stages (TMA)
 //   warp 1      TMEM allocator; one lane issues tcgen05.mma
@@ -36,7 +44,9 @@
 #pragma once
 
 #include <climits>
+#include "commit.cuh"
 #include "ptx.cuh"
+#include "softmax.cuh"
 
 namespace cai {
 
@@ -47,13 +57,14 @@ constexpr int kChunkN = 256;       // largest MMA N (positions per pass over W)
 constexpr int kBoxRowsB = 16;      // rows per TMA box of the hidden tile
 constexpr int kHeadThreads = 192;
 constexpr int kATileBytes = kRowsPerTile * kBlockK * 2;  // 16 KiB
-constexpr float kLog2e = 1.4426950408889634f;
-constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows to 0
 
 struct HeadParams {
   const uint8_t* wpk;  // packed W (see pack_weight_kernel)
-  const int* d_M;      // masked rows of this step (device)
-  int* m_hist_slot;    // where this step's M is recorded
+  const int* d_M;      // masked rows of this step (device; multi-kernel step)
+  int* m_hist_slot;    // where this step's M is recorded (multi-kernel step)
+  int fused;           // 1: single-kernel step (see below), 0: gather / head / merge kernels
+  int M_fixed;         // rows decoded by the single-kernel step (all B P positions)
+  int first;           // the step is a block's step zero (every position masked)
   float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
   uint32_t* err;       // error word
   int V, H;
@@ -64,6 +75,7 @@ struct HeadParams {
   int slot_cols;       // tensor-memory columns per tile accumulator (round32(n_max))
   int gmax;            // largest tile group
   int tmem_cols;       // allocated tensor-memory columns (>= 2 gmax slot_cols)
+  CommitParams cp;     // commit rule, run by the last CTA of a single-kernel step
 };
 
 // ------------------------------------------------------------ CTA plan --
@@ -94,6 +106,16 @@ struct CtaPlan {
            static_cast<size_t>(t - group_first(g)) * kATileBytes;
   }
 };
+
+// Rows this launch decodes.  Multi-kernel step: the masked rows the gather
+// kernel compacted.  Single-kernel step: all B P rows, unless the previous
+// step left nothing masked in a running sequence (and this is not a block's
+// step zero), in which case there is nothing to decode.  Read after
+// grid_dependency_wait().
+__device__ __forceinline__ int rows_to_decode(const int* d_M, int fused, int first, int M_fixed) {
+  if (!fused) return *d_M;
+  return (first || *d_M > 0) ? M_fixed : 0;
+}
 
 __host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
   CtaPlan p;
@@ -139,85 +161,6 @@ __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restric
     if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
     out[d] = val;
   }
-}
-
-// ------------------------------------------------------------ reduction --
-
-__device__ __forceinline__ float fast_exp2(float x) {
-  float y;
-  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-  return y;
-}
-
-// Merge two online-softmax triples (m in log2 units, S = sum 2^(z - m), idx).
-// The larger maximum keeps weight 1; ties keep the lower vocabulary index.
-__device__ __forceinline__ void merge_tri(float& m, float& s, int& i, float mo, float so,
-                                          int io) {
-  const float e = fast_exp2(-fabsf(m - mo));
-  const bool mine = m >= mo;
-  const float sn = mine ? fmaf(so, e, s) : fmaf(s, e, so);
-  const int in = (m > mo) ? i : ((mo > m) ? io : min(i, io));
-  m = fmaxf(m, mo);
-  s = sn;
-  i = in;
-}
-
-// 32 lanes x 32 columns of online-softmax triples -> lane l holds the merge of
-// column l over the 32 lanes, in m[0], s[0], ix[0].  Five halving steps: at
-// width w each lane keeps half of its live columns and receives the partner's
-// copy of the same columns (31 merges per lane, one exponential each).
-__device__ __forceinline__ void transpose_merge32(float (&m)[32], float (&s)[32], int (&ix)[32],
-                                                  int lane) {
-#pragma unroll
-  for (int w = 16; w >= 1; w >>= 1) {
-    const bool up = (lane & w) != 0;
-#pragma unroll
-    for (int c = 0; c < w; ++c) {
-      float km = up ? m[c + w] : m[c];
-      float ks = up ? s[c + w] : s[c];
-      int ki = up ? ix[c + w] : ix[c];
-      const float sm = up ? m[c] : m[c + w];
-      const float ss = up ? s[c] : s[c + w];
-      const int si = up ? ix[c] : ix[c + w];
-      const float rm = __shfl_xor_sync(0xffffffffu, sm, w);
-      const float rs = __shfl_xor_sync(0xffffffffu, ss, w);
-      const int ri = __shfl_xor_sync(0xffffffffu, si, w);
-      merge_tri(km, ks, ki, rm, rs, ri);
-      m[c] = km;
-      s[c] = ks;
-      ix[c] = ki;
-    }
-  }
-}
-
-// 32 rows (one per lane) x 32 columns of logits -> lane l holds the
-// (max, sum, argmax) of column l over the 32 rows.
-__device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
-                                                   int lane, float& om, float& os, int& oi) {
-  float m[32], s[32];
-  int ix[32];
-#pragma unroll
-  for (int c = 0; c < 32; ++c) {
-    m[c] = valid ? __uint_as_float(v[c]) * kLog2e : kNegBig;
-    s[c] = valid ? 1.0f : 0.0f;
-    ix[c] = valid ? vrow : INT_MAX;
-  }
-  transpose_merge32(m, s, ix, lane);
-  om = m[0];
-  os = s[0];
-  oi = ix[0];
-}
-
-// Fold one logit z (log2 units) of vocabulary row `row` into a running
-// triple.  Rows arrive in increasing order, so only a strictly larger value
-// replaces the argmax (ties keep the lower index).
-__device__ __forceinline__ void online_update(float& m, float& s, int& i, float z, int row) {
-  const float d = z - m;
-  const float e = fast_exp2(-fabsf(d));
-  const bool up = d > 0.0f;
-  s = up ? fmaf(s, e, 1.0f) : s + e;
-  m = up ? z : m;
-  i = up ? row : i;
 }
 
 // Wait used only on the abort path, for copies this CTA already issued.
@@ -320,8 +263,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     mbar_init(sm.drain, 1);
     *sm.abort = 0;
     fence_mbar_init();
-    grid_launch_dependents();
   }
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
   if (warp == 0 && lane == 0) prefetch_tmap(&tm_h);
   if (warp == 1) {
     tmem_alloc(sm.tmem_slot, static_cast<uint32_t>(p.tmem_cols));
@@ -357,7 +300,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
       }
       grid_dependency_wait();
-      const int M = *p.d_M;
+      const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb;
       long long a_issued = 0, b_issued = 0;
@@ -422,7 +365,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     if (lane == 0) {
       // ---------------------------------------------------- MMA issuer --
       grid_dependency_wait();
-      const int M = *p.d_M;
+      const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb, racc;
       bool ok = true;
@@ -482,9 +425,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   } else {
     // --------------------------------------------------------- epilogue --
     grid_dependency_wait();
-    const int M = *p.d_M;
+    const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
     const int n_chunks = (M + kChunkN - 1) / kChunkN;
-    if (threadIdx.x == 64 && cta == 0) *p.m_hist_slot = M;
+    if (!p.fused && threadIdx.x == 64 && cta == 0) *p.m_hist_slot = M;
     const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
@@ -620,6 +563,27 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   if (warp == 1) {
     tc_fence_after();
     tmem_dealloc(tmem_base, static_cast<uint32_t>(p.tmem_cols));
+  }
+
+  if (p.fused) {
+    // Single-kernel step: the last CTA to finish commits the step.
+    __shared__ int s_last;
+    if (threadIdx.x == 0) {
+      __threadfence();
+      s_last = atomicAdd(p.cp.ticket, 1u) == static_cast<unsigned>(G - 1);
+    }
+    __syncthreads();
+    if (!s_last) return;
+    __threadfence();
+    int decoded = 0, remaining = 0;
+    for (int b = 0; b < p.cp.B; ++b) {
+      int left = 0;
+      // Every copy and MMA has completed: the W ring is free shared memory.
+      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), &left);
+      remaining += left;
+    }
+    if (threadIdx.x == 0) *p.cp.m_hist_slot = decoded;
+    finish_step(p.cp, remaining);
   }
 }
 

@@ -1,0 +1,93 @@
+// Online-softmax triples: (m, S, idx) with m the running maximum in log2 units,
+// S = sum of 2^(z - m) over the values seen, idx the lowest index reaching m.
+// Merging two triples or folding in one value is exact up to fp32 rounding, so
+// any split of the vocabulary reduces to max_v z, sum_v exp(z_v - max) and the
+// argmax (Box 1 of arXiv 2608.22646: c = exp(max - LSE) = 1 / S).
+#pragma once
+
+#include <climits>
+#include <cstdint>
+
+namespace cai {
+
+constexpr float kLog2e = 1.4426950408889634f;
+constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows to 0
+
+__device__ __forceinline__ float fast_exp2(float x) {
+  float y;
+  asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+  return y;
+}
+
+// Merge two online-softmax triples (m in log2 units, S = sum 2^(z - m), idx).
+// The larger maximum keeps weight 1; ties keep the lower vocabulary index.
+__device__ __forceinline__ void merge_tri(float& m, float& s, int& i, float mo, float so,
+                                          int io) {
+  const float e = fast_exp2(-fabsf(m - mo));
+  const bool mine = m >= mo;
+  const float sn = mine ? fmaf(so, e, s) : fmaf(s, e, so);
+  const int in = (m > mo) ? i : ((mo > m) ? io : min(i, io));
+  m = fmaxf(m, mo);
+  s = sn;
+  i = in;
+}
+
+// 32 lanes x 32 columns of online-softmax triples -> lane l holds the merge of
+// column l over the 32 lanes, in m[0], s[0], ix[0].  Five halving steps: at
+// width w each lane keeps half of its live columns and receives the partner's
+// copy of the same columns (31 merges per lane, one exponential each).
+__device__ __forceinline__ void transpose_merge32(float (&m)[32], float (&s)[32], int (&ix)[32],
+                                                  int lane) {
+#pragma unroll
+  for (int w = 16; w >= 1; w >>= 1) {
+    const bool up = (lane & w) != 0;
+#pragma unroll
+    for (int c = 0; c < w; ++c) {
+      float km = up ? m[c + w] : m[c];
+      float ks = up ? s[c + w] : s[c];
+      int ki = up ? ix[c + w] : ix[c];
+      const float sm = up ? m[c] : m[c + w];
+      const float ss = up ? s[c] : s[c + w];
+      const int si = up ? ix[c] : ix[c + w];
+      const float rm = __shfl_xor_sync(0xffffffffu, sm, w);
+      const float rs = __shfl_xor_sync(0xffffffffu, ss, w);
+      const int ri = __shfl_xor_sync(0xffffffffu, si, w);
+      merge_tri(km, ks, ki, rm, rs, ri);
+      m[c] = km;
+      s[c] = ks;
+      ix[c] = ki;
+    }
+  }
+}
+
+// 32 rows (one per lane) x 32 columns of logits -> lane l holds the
+// (max, sum, argmax) of column l over the 32 rows.
+__device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
+                                                   int lane, float& om, float& os, int& oi) {
+  float m[32], s[32];
+  int ix[32];
+#pragma unroll
+  for (int c = 0; c < 32; ++c) {
+    m[c] = valid ? __uint_as_float(v[c]) * kLog2e : kNegBig;
+    s[c] = valid ? 1.0f : 0.0f;
+    ix[c] = valid ? vrow : INT_MAX;
+  }
+  transpose_merge32(m, s, ix, lane);
+  om = m[0];
+  os = s[0];
+  oi = ix[0];
+}
+
+// Fold one logit z (log2 units) of vocabulary row `row` into a running
+// triple.  Rows arrive in increasing order, so only a strictly larger value
+// replaces the argmax (ties keep the lower index).
+__device__ __forceinline__ void online_update(float& m, float& s, int& i, float z, int row) {
+  const float d = z - m;
+  const float e = fast_exp2(-fabsf(d));
+  const bool up = d > 0.0f;
+  s = up ? fmaf(s, e, 1.0f) : s + e;
+  m = up ? z : m;
+  i = up ? row : i;
+}
+
+}  // namespace cai

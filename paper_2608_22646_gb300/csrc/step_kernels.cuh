@@ -12,52 +12,9 @@
 
 namespace cai {
 
-constexpr int kMask = -1;
-enum : int { kRunning = 0, kExitDone = 1, kExitGrind = 2, kExitTmax = 3 };
-enum : uint32_t {
-  kFlagGating = 1u,
-  kFlagPosFactor = 2u,
-  kFlagFlush = 4u,
-  kFlagQuarterPos = 8u,
-  kFlagQuarterBlocks = 16u
-};
-constexpr int kMaxP = 256;
 constexpr int kGatherRowsPerCta = 4;
 constexpr int kGatherThreads = 256;
 constexpr int kCommitThreads = 256;  // merge kernel: small enough to share an SM with the LM head
-constexpr int kPosPerWarp = 2;       // positions whose partials a warp loads at once
-constexpr int kPartPerLane = 5;      // partial slots a lane loads per position (G <= 160)
-
-// Host-visible record of the last committed step, one 64-bit word in mapped
-// pinned memory written by a single store (so the host never sees a torn
-// record): bits 0-31 step id + 1, bit 32 every sequence has exited the block,
-// bit 33 the device error word is non-zero, bits 34-48 the block index.
-struct HostFlag {
-  unsigned long long word;  // 0 = no step committed yet
-  unsigned long long pad;
-};
-__host__ __device__ inline unsigned long long host_flag_word(int step_id, bool all_done, bool err,
-                                                             int blk) {
-  return static_cast<unsigned long long>(static_cast<uint32_t>(step_id) + 1u) |
-         (static_cast<unsigned long long>(all_done ? 1u : 0u) << 32) |
-         (static_cast<unsigned long long>(err ? 1u : 0u) << 33) |
-         (static_cast<unsigned long long>(static_cast<uint32_t>(blk) & 0x7FFFu) << 34);
-}
-
-struct StateArrays {
-  int* tok;
-  float* conf;
-  float* s0;
-  uint8_t* budget;
-  int16_t* cstep;
-  int* cand;
-  int* ell;
-  int* eta;
-  int* exit_reason;
-  int* exit_step;
-  int* unresolved;
-  int* m_hist;
-};
 
 // ------------------------------------------------------------ gather (K1) --
 
@@ -73,7 +30,7 @@ struct GatherParams {
 
 __global__ void __launch_bounds__(kGatherThreads)
     gather_rows_kernel(const GatherParams p) {
-  if (threadIdx.x == 0) grid_launch_dependents();
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();  // the previous step's merge wrote list, row_of and d_M
   const int M = p.first ? p.BP : *p.d_M;
   if (p.first) {
@@ -98,49 +55,7 @@ __global__ void __launch_bounds__(kGatherThreads)
   }
 }
 
-// ------------------------------------------------------ list builder -----
-
-// Compact, in (b, p) order, the still-masked tokens of running sequences of
-// block blk into list / row_of; returns the count.  One CTA (blockDim.x a
-// multiple of 32, at most 1024).  Reads bypass L1: other CTAs wrote this state.
-__device__ int build_masked_list(const int* tok, const int* exit_reason, int* list, int* row_of,
-                                 int B, int P, int L, int n_blocks, int blk) {
-  __shared__ int s_wsum[32];
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nwarps = blockDim.x >> 5;
-  const int BP = B * P;
-  int base = 0;
-  for (int i0 = 0; i0 < BP; i0 += blockDim.x) {
-    const int i = i0 + tid;
-    bool mk = false;
-    if (i < BP) {
-      const int b = i / P, pp = i - b * P;
-      mk = __ldcg(&tok[static_cast<size_t>(b) * L + blk * P + pp]) == kMask &&
-           __ldcg(&exit_reason[b * n_blocks + blk]) == kRunning;
-    }
-    const unsigned bal = __ballot_sync(0xffffffffu, mk);
-    const int wpre = __popc(bal & ((1u << lane) - 1u));
-    if (lane == 0) s_wsum[warp] = __popc(bal);
-    __syncthreads();
-    int woff = 0, tot = 0;
-    for (int w = 0; w < nwarps; ++w) {
-      const int c = s_wsum[w];
-      woff += (w < warp) ? c : 0;
-      tot += c;
-    }
-    if (i < BP) {
-      if (mk) {
-        list[base + woff + wpre] = i;
-        row_of[i] = base + woff + wpre;
-      } else {
-        row_of[i] = -1;
-      }
-    }
-    base += tot;
-    __syncthreads();
-  }
-  return base;
-}
+// ------------------------------------------------------ list rebuild -----
 
 struct ListParams {
   const int* tok;
@@ -160,173 +75,17 @@ __global__ void __launch_bounds__(kCommitThreads) rebuild_list_kernel(const List
 
 // ------------------------------------------------------ merge + commit (K3) --
 
-struct CommitParams {
-  const float4* part;     // [rows_cap, n_part]
-  int n_part;             // partial slots per row (one per LM-head CTA)
-  StateArrays st;
-  int* list;
-  int* row_of;
-  int* d_M;
-  unsigned* ticket;       // zero between launches
-  HostFlag* hf;           // device alias of the mapped host record
-  uint32_t* err;
-  int B, P, L, n_blocks, T, blk, t, step_id;
-  int K;
-  int eta_mode;           // 0 count, 1 fraction of the generation length
-  float eta_bar;
-  float theta_fb;
-  int budget_half;        // Box 5 "p < 32" tier boundary
-  int budget_late;        // Box 5 "p >= 48" tier boundary
-  uint32_t flags;
-  float theta_tab[kMaxP]; // theta_i(t) per position (Box 6), from the host
-};
-
-__device__ __forceinline__ int budget_tier(float s, int p, int half, int late) {
-  if (s > 0.50f && p < half) return 8;
-  if (s < 0.25f || p >= late) return 64;
-  return 32;
-}
-
-// One CTA per sequence: warp w merges the partials of positions
-// w, w + 8, w + 16, ... (four at a time, all loads issued before any merge)
-// and lane 0 applies the commit rule to each.
+// One CTA per sequence: merge_commit_sequence for sequence blockIdx.x, then the
+// last CTA to finish (atomic ticket; none needed for a single CTA) builds the
+// next step's list and publishes the step.
 __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const CommitParams p) {
-  __shared__ int s_eta, s_left, s_reason, s_unres, s_last;
-  if (threadIdx.x == 0) grid_launch_dependents();
-  const int b = blockIdx.x;
-  const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
-  const int nwarps = blockDim.x >> 5;
-  if (tid == 0) {
-    s_eta = 0;
-    s_left = 0;
-    s_reason = kRunning;
-    s_unres = 0;
-  }
-  grid_dependency_wait();  // partials of this step, state of the previous one
-  __syncthreads();
-  const int eb = b * p.n_blocks + p.blk;
-  const bool running = p.st.exit_reason[eb] == kRunning;
-  const bool gating = (p.flags & kFlagGating) != 0;
-
-  if (running) {
-    for (int base = warp; base < p.P; base += nwarps * kPosPerWarp) {
-      int row[kPosPerWarp];
-      float4 q[kPosPerWarp][kPartPerLane];
-#pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
-        const int pp = base + j * nwarps;
-        row[j] = -1;
-        if (pp < p.P) {
-          const size_t g = static_cast<size_t>(b) * p.L + p.blk * p.P + pp;
-          if (p.st.tok[g] == kMask) {
-            row[j] = p.row_of[b * p.P + pp];
-            if (row[j] < 0) {
-              if (lane == 0) atomicOr(p.err, kErrBadRow);
-              row[j] = -2;
-            }
-          }
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
-        const float4* pr = p.part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * p.n_part;
-#pragma unroll
-        for (int u = 0; u < kPartPerLane; ++u) {
-          const int k = lane + 32 * u;
-          q[j][u] = (row[j] >= 0 && k < p.n_part)
-                        ? __ldcg(pr + k)
-                        : make_float4(kNegBig, 0.0f, __int_as_float(INT_MAX), 0.0f);
-        }
-      }
-#pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
-        if (row[j] < 0) continue;  // warp-uniform
-        const int pp = base + j * nwarps;
-        float m = kNegBig, s = 0.0f;
-        int ix = INT_MAX;
-#pragma unroll
-        for (int u = 0; u < kPartPerLane; ++u)
-          merge_tri(m, s, ix, q[j][u].x, q[j][u].y, __float_as_int(q[j][u].z));
-        for (int k = lane + 32 * kPartPerLane; k < p.n_part; k += 32) {
-          const float4 r = __ldcg(p.part + static_cast<size_t>(row[j]) * p.n_part + k);
-          merge_tri(m, s, ix, r.x, r.y, __float_as_int(r.z));
-        }
-#pragma unroll
-        for (int off = 16; off >= 1; off >>= 1) {
-          const float mo = __shfl_xor_sync(0xffffffffu, m, off);
-          const float so = __shfl_xor_sync(0xffffffffu, s, off);
-          const int io = __shfl_xor_sync(0xffffffffu, ix, off);
-          merge_tri(m, s, ix, mo, so, io);
-        }
-        if (lane == 0) {
-          const size_t g = static_cast<size_t>(b) * p.L + p.blk * p.P + pp;
-          const float c = 1.0f / s;  // max_v p_v = exp(m - LSE) = 1 / sum_v exp(z_v - m)
-          if (p.t == 0) {
-            p.st.s0[g] = c;
-            p.st.budget[g] =
-                static_cast<uint8_t>(budget_tier(c, pp, p.budget_half, p.budget_late));
-          }
-          p.st.conf[g] = c;
-          p.st.cand[g] = ix;
-          const bool by_conf = c >= p.theta_tab[pp];
-          const bool by_budget = gating && p.t >= static_cast<int>(p.st.budget[g]);
-          if (by_conf || by_budget) {
-            p.st.tok[g] = ix;
-            p.st.cstep[g] = static_cast<int16_t>(p.t);
-            atomicAdd(&s_eta, 1);
-          } else {
-            atomicAdd(&s_left, 1);
-          }
-        }
-      }
-    }
-  }
-  __syncthreads();
-  if (running && tid == 0) {
-    const int eta = s_eta;
-    p.st.eta[b] = eta;
-    const bool low = p.eta_mode == 1
-                         ? (static_cast<double>(eta) / (static_cast<double>(p.n_blocks) * p.P) <
-                            static_cast<double>(p.eta_bar))
-                         : (static_cast<float>(eta) < p.eta_bar);
-    // Algorithm 1 sets ell <- 0 before the block's first step.
-    const int ell = low ? (p.t == 0 ? 0 : p.st.ell[b]) + 1 : 0;
-    p.st.ell[b] = ell;
-    int reason = kRunning;
-    if (gating && ell >= p.K)
-      reason = kExitGrind;
-    else if (s_left == 0)
-      reason = kExitDone;
-    else if (p.t == p.T - 1)
-      reason = kExitTmax;
-    s_reason = reason;
-  }
-  __syncthreads();
-  const int reason = s_reason;
-  if (running && reason != kRunning) {
-    for (int pp = tid; pp < p.P; pp += blockDim.x) {
-      const size_t g = static_cast<size_t>(b) * p.L + p.blk * p.P + pp;
-      if (p.st.tok[g] != kMask) continue;
-      if ((reason == kExitGrind && p.st.conf[g] > p.theta_fb) || (p.flags & kFlagFlush)) {
-        p.st.tok[g] = p.st.cand[g];
-        p.st.cstep[g] = static_cast<int16_t>(p.t);
-      } else {
-        atomicAdd(&s_unres, 1);
-      }
-    }
-    __syncthreads();
-    if (tid == 0) {
-      p.st.exit_reason[eb] = reason;
-      p.st.exit_step[eb] = p.t;
-      p.st.unresolved[eb] = s_unres;
-    }
-  }
-
-  // Last CTA to finish: next step's list and the host-visible record.  With
-  // a single CTA there is nobody to wait for.
-  __syncthreads();
+  __shared__ int s_last;
+  __shared__ CommitSmem cs;
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // partials of this step, state of the previous one
+  merge_commit_sequence(p, blockIdx.x, cs);
   if (gridDim.x > 1) {
-    if (tid == 0) {
+    if (threadIdx.x == 0) {
       __threadfence();
       s_last = atomicAdd(p.ticket, 1u) == gridDim.x - 1;
     }
@@ -334,17 +93,7 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
     if (!s_last) return;
     __threadfence();
   }
-  const int n = build_masked_list(p.st.tok, p.st.exit_reason, p.list, p.row_of, p.B, p.P, p.L,
-                                  p.n_blocks, p.blk);
-  if (tid == 0) {
-    *p.d_M = n;
-    *p.ticket = 0u;
-    const bool err = *reinterpret_cast<volatile uint32_t*>(p.err) != 0u;
-    // The host uses this word only for control flow; it reads the state
-    // itself through stream-ordered copies, so no system fence is needed.
-    *reinterpret_cast<volatile unsigned long long*>(&p.hf->word) =
-        host_flag_word(p.step_id, n == 0, err, p.blk);
-  }
+  finish_step(p);
 }
 
 }  // namespace cai

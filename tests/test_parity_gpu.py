@@ -274,7 +274,8 @@ def test_profile_and_stats():
         cai.cai_first_step(ctx, hs(0, 0))
         cai.cai_denoise_step(ctx, hs(0, 1))
         s = cai.cai_get_stats(ctx)
-        assert s["steps"] == 2 and s["head_launches"] == 2 and s["launches"] == 6
+        assert s["steps"] == 2 and s["head_launches"] == 2
+        assert s["kernels_per_step"] == 1 and s["launches"] == 2    # B P = 16: one kernel
         assert s["head_profiled"] == 2 and s["head_ms"] > 0
         assert s["grid"] == 64 and s["n_max"] == 16
     finally:

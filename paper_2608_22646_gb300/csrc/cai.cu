@@ -430,7 +430,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->fused = c->BP <= kChunkN;
 
   // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
-  // at most one per 64-row unit), tile group size (tiles sharing one hidden
+  // at least kMinCtaRows vocabulary rows per CTA), tile group size (tiles sharing one hidden
   // stage; two group buffers of gmax * slot_cols tensor-memory columns fit in
   // 512), ring depths within the opt-in shared memory.
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
@@ -440,11 +440,15 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   // the next step's CTAs all find a free SM instead of one of them waiting
   // for the commit to finish (and becoming the next step's straggler).
   const int usable_sms = c->fused && sms > 1 ? sms - 1 : sms;
-  c->G = units < usable_sms ? units : usable_sms;
+  // V is split in units of one swizzle atom (kUnitRows rows), so any grid
+  // size balances the rows to within kUnitRows per CTA.
+  const int min_units = kMinCtaRows / kUnitRows;
+  const int g_rows = (units + min_units - 1) / min_units;
+  c->G = g_rows < usable_sms ? g_rows : usable_sms;
   const int glim = g_head_grid_limit.load();
   if (glim > 0 && c->G > glim) c->G = glim;
   const int max_units = (units + c->G - 1) / c->G;
-  const int max_tiles = (max_units + 1) / 2;
+  const int max_tiles = (max_units * kUnitRows + kRowsPerTile - 1) / kRowsPerTile;
   // Default: as many tiles per group as two group buffers of tensor memory
   // allow (all of a CTA's tiles for N <= 32).  Every tile of a group is an
   // independent accumulation chain, and at small N a single chain is bound by
@@ -510,7 +514,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
   CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * c->G)
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
-  CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * 128 * cfg->H)
+  CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   const void* w_src = W;
   void* w_tmp = nullptr;
   if (!is_device_ptr(W)) {
@@ -529,7 +533,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     w_src = w_tmp;
   }
   {
-    const long long n_chunks = static_cast<long long>(units) * 64 * cfg->H / 8;
+    const long long n_chunks = static_cast<long long>(units) * kUnitRows * cfg->H / 8;
     pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
         c->gmax, n_chunks);

@@ -5,7 +5,8 @@
 // run with A and B swapped: the vocabulary fills the MMA M dimension (128 rows
 // of W per accumulator tile) and the positions form the N dimension
 // (16..256 columns, rounded up to 16).  Each CTA owns a contiguous range of W
-// rows in units of 64 rows and reads it once from HBM; the logits stay in
+// rows (whole 8-row swizzle atoms, at least 64 rows, balanced over the grid
+// to within 8 rows) and reads it once from HBM; the logits stay in
 // tensor memory and are never written anywhere.  The epilogue reduces every
 // accumulator tile to a running (max, sum of exponentials, argmax) per
 // position in the log2 domain; the four epilogue warps merge their slices
@@ -21,8 +22,8 @@
 // buffers let the epilogue of one group overlap the MMAs of the next.
 //
 // W is read from a packed copy made once per context (pack_weight_kernel) in
-// exactly the order the CTAs consume it: CTA c owns rows [64 u0, 64 u1) and
-// the bytes [128 H u0, 128 H u1) of the packed copy, laid out group by group,
+// exactly the order the CTAs consume it: CTA c owns rows [8 u0, 8 u1) and
+// the bytes [16 H u0, 16 H u1) of the packed copy, laid out group by group,
 // K block by K block, tile by tile, each stage already in the
 // 128-byte-swizzled K-major layout the MMA descriptors expect.  Every CTA thus
 // streams one contiguous region front to back with one bulk copy per stage;
@@ -51,7 +52,8 @@
 namespace cai {
 
 constexpr int kRowsPerTile = 128;  // MMA M: vocabulary rows per accumulator
-constexpr int kUnitRows = 64;      // granularity of the per-CTA split of V
+constexpr int kUnitRows = 8;       // granularity of the per-CTA split of V (one swizzle atom)
+constexpr int kMinCtaRows = 64;    // fewest vocabulary rows the launch gives one CTA
 constexpr int kBlockK = 64;        // K per stage: one 128-byte swizzled row of bf16
 constexpr int kChunkN = 256;       // largest MMA N (positions per pass over W)
 constexpr int kBoxRowsB = 16;      // rows per TMA box of the hidden tile
@@ -68,7 +70,7 @@ struct HeadParams {
   float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
   uint32_t* err;       // error word
   int V, H;
-  int units;           // ceil(V / 64)
+  int units;           // ceil(V / kUnitRows)
   int n_stages;        // depth of the W ring (16 KiB slots)
   int n_bslots;        // depth of the hidden-state ring
   int b_slot_bytes;    // n_max * 128
@@ -80,16 +82,22 @@ struct HeadParams {
 
 // ------------------------------------------------------------ CTA plan --
 
-// First 64-row unit of CTA c when `units` units are split over G CTAs.
+// First unit (kUnitRows rows) of CTA c when `units` units are split over G CTAs.
 __host__ __device__ inline int unit_begin(int c, int units, int G) {
   return static_cast<int>((static_cast<long long>(c) * units) / G);
 }
 
-// The work of one CTA: units [u0, u1) as tiles of 128 rows (the last may be
-// 64), grouped gsz = min(gmax, tiles) tiles at a time.
+// The work of one CTA: units [u0, u1), i.e. vocabulary rows [row0, row0 +
+// rows), as tiles of 128 rows (the last may be shorter, by a multiple of
+// kUnitRows), grouped gsz = min(gmax, tiles) tiles at a time.
 struct CtaPlan {
   int u0, u1, n_tiles, gsz, n_groups;
-  __host__ __device__ int tile_rows(int t) const { return (u1 - (u0 + 2 * t) >= 2) ? 128 : 64; }
+  __host__ __device__ int row0() const { return u0 * kUnitRows; }
+  __host__ __device__ int rows() const { return (u1 - u0) * kUnitRows; }
+  __host__ __device__ int tile_rows(int t) const {
+    const int r = rows() - t * kRowsPerTile;
+    return r < kRowsPerTile ? r : kRowsPerTile;
+  }
   __host__ __device__ int group_first(int g) const { return g * gsz; }
   __host__ __device__ int group_count(int g) const {
     const int n = n_tiles - g * gsz;
@@ -97,11 +105,11 @@ struct CtaPlan {
   }
   __host__ __device__ int group_rows(int g) const {
     const int t0 = group_first(g), n = group_count(g);
-    return 128 * (n - 1) + tile_rows(t0 + n - 1);
+    return kRowsPerTile * (n - 1) + tile_rows(t0 + n - 1);
   }
   // Byte offset in the packed weight of W stage (group g, K block kb, tile t).
   __host__ __device__ size_t stage_offset(int g, int kb, int t, int H) const {
-    return static_cast<size_t>(u0) * 128 * H + static_cast<size_t>(g) * gsz * 256 * H +
+    return static_cast<size_t>(row0()) * 2 * H + static_cast<size_t>(g) * gsz * kRowsPerTile * 2 * H +
            static_cast<size_t>(kb) * group_rows(g) * 128 +
            static_cast<size_t>(t - group_first(g)) * kATileBytes;
   }
@@ -121,22 +129,22 @@ __host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
   CtaPlan p;
   p.u0 = unit_begin(c, units, G);
   p.u1 = unit_begin(c + 1, units, G);
-  p.n_tiles = (p.u1 - p.u0 + 1) >> 1;
+  p.n_tiles = (p.rows() + kRowsPerTile - 1) / kRowsPerTile;
   const int g = gmax < p.n_tiles ? gmax : p.n_tiles;
   p.gsz = g < 1 ? 1 : g;
   p.n_groups = (p.n_tiles + p.gsz - 1) / p.gsz;
   return p;
 }
 
-// Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` 64-row
-// units and groups of up to gmax tiles.  Inside a stage block, row r's
+// Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` units of
+// kUnitRows rows and groups of up to gmax tiles.  Inside a stage block, row r's
 // 16-byte chunk c (k = 8c..8c+7 of the block's 64) sits at
 // r * 128 + ((c ^ (r & 7)) * 16): the 128-byte swizzle of 8-row, 1024-byte
 // atoms.  Rows >= V are zero.  One thread per destination 16-byte chunk;
-// n_chunks = units * 64 * H / 8.
+// n_chunks = units * kUnitRows * H / 8.
 __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
                                    int H, int units, int G, int gmax, long long n_chunks) {
-  const long long unit_bytes = 128ll * H;
+  const long long unit_bytes = 2ll * kUnitRows * H;
   for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
        d += static_cast<long long>(gridDim.x) * blockDim.x) {
     const long long byte = d * 16;
@@ -147,8 +155,9 @@ __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restric
     while (c > 0 && unit_begin(c, units, G) > u) --c;
     const CtaPlan pl = cta_plan(c, units, G, gmax);
     const long long off = byte - static_cast<long long>(pl.u0) * unit_bytes;
-    const int g = static_cast<int>(off / (static_cast<long long>(pl.gsz) * 2 * unit_bytes));
-    const long long rem = off - static_cast<long long>(g) * pl.gsz * 2 * unit_bytes;
+    const long long group_bytes = static_cast<long long>(pl.gsz) * kRowsPerTile * 2 * H;
+    const int g = static_cast<int>(off / group_bytes);
+    const long long rem = off - static_cast<long long>(g) * group_bytes;
     const int grow = pl.group_rows(g);
     const int kb = static_cast<int>(rem / (grow * 128));
     const int rem2 = static_cast<int>(rem - static_cast<long long>(kb) * grow * 128);
@@ -156,7 +165,7 @@ __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restric
     const int inblk = rem2 % kATileBytes;
     const int r = inblk >> 7;
     const int cl = ((inblk >> 4) & 7) ^ (r & 7);
-    const long long v = static_cast<long long>(pl.u0 + 2 * t) * 64 + r;
+    const long long v = static_cast<long long>(pl.row0()) + t * kRowsPerTile + r;
     uint4 val = make_uint4(0u, 0u, 0u, 0u);
     if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
     out[d] = val;
@@ -467,7 +476,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
               tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
           for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
             const int row_local = quarter * 32 + lane;
-            const int vrow = (pl.u0 + 2 * t) * kUnitRows + row_local;
+            const int vrow = pl.row0() + t * kRowsPerTile + row_local;
             const bool valid = row_local < pl.tile_rows(t) && vrow < p.V;
             uint32_t v[32];
             tmem_ld_32cols(tgroup + static_cast<uint32_t>((t - pl.group_first(g)) * p.slot_cols),
@@ -500,7 +509,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
               tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
           for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
             const int row_local = quarter * 32 + lane;
-            const int vrow = (pl.u0 + 2 * t) * kUnitRows + row_local;
+            const int vrow = pl.row0() + t * kRowsPerTile + row_local;
             const bool valid = row_local < pl.tile_rows(t) && vrow < p.V;
             const uint32_t tcol =
                 tgroup + static_cast<uint32_t>((t - pl.group_first(g)) * p.slot_cols);

@@ -58,9 +58,9 @@ def test_toy_literal_generator_grinds_at_t3():
 
 
 @pytest.mark.parametrize("shape,grid", [
-    # (B, P, H, V, T, n_blocks), LM-head CTA cap: ragged vocab tails (V % 64,
+    # (B, P, H, V, T, n_blocks), LM-head CTA cap: ragged vocab tails (V % 8,
     # V % 128), a single K stage (H = 64), M = 1, several MMA chunks (M > 256),
-    # B P not a multiple of 16, CTAs with several 128-row tiles and a 64-row one.
+    # B P not a multiple of 16, CTAs with several 128-row tiles and a short one.
     ((1, 1, 64, 64, 4, 2), 0),
     ((3, 7, 128, 1000, 6, 2), 0),
     ((3, 7, 128, 1000, 6, 2), 3),
@@ -69,6 +69,8 @@ def test_toy_literal_generator_grinds_at_t3():
     ((2, 150, 64, 4160, 5, 1), 7),
     ((5, 64, 256, 8192, 12, 2), 9),
     ((1, 16, 256, 4096, 8, 4), 1),
+    ((2, 5, 128, 1003, 6, 2), 2),
+    ((1, 24, 64, 2085, 6, 1), 0),
 ])
 def test_ragged_shapes_trajectory(shape, grid):
     B, P, H, V, T, nb = shape

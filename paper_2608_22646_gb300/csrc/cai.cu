@@ -141,6 +141,7 @@ struct cai_ctx {
   int* row_of = nullptr;
   int* d_M = nullptr;
   unsigned* ticket = nullptr;
+  unsigned long long* pub = nullptr;  // last published step (CommitParams::pub)
   uint32_t* err = nullptr;
   __nv_bfloat16* hc = nullptr;
   float4* part = nullptr;
@@ -250,6 +251,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   cp.d_M = c->d_M;
   cp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
   cp.ticket = c->ticket;
+  cp.pub = c->pub;
   cp.hf = c->hf_dev;
   cp.err = c->err;
   cp.B = cfg.B;
@@ -510,6 +512,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->row_of, int, c->BP)
   CAI_ALLOC(c->d_M, int, 1)
   CAI_ALLOC(c->ticket, unsigned, 1)
+  CAI_ALLOC(c->pub, unsigned long long, 1)
   CAI_ALLOC(c->err, uint32_t, 1)
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
   CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * c->G)
@@ -615,6 +618,7 @@ int cai_reset(cai_ctx* c, void* stream_v) {
             cudaMemsetAsync(c->st.m_hist, 0, static_cast<size_t>(cfg.n_blocks) * cfg.T * 4, s) ==
                 cudaSuccess &&
             cudaMemsetAsync(c->ticket, 0, 4, s) == cudaSuccess &&
+            cudaMemsetAsync(c->pub, 0, 8, s) == cudaSuccess &&
             cudaMemsetAsync(c->err, 0, 4, s) == cudaSuccess &&
             cudaMemsetAsync(c->d_M, 0, 4, s) == cudaSuccess;
   if (!ok) return fail(c, CAI_ERR_CUDA);
@@ -748,6 +752,8 @@ int cai_state_upload(cai_ctx* c, const cai_host_state* src) {
     return CAI_ERR_ARG;
   int r = transfer(c, src, false);
   if (r != CAI_OK) return r;
+  // The uploaded state replaces what the last step published.
+  if (cudaMemset(c->pub, 0, 8) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
   c->blk = src->blk;
   c->t_next = src->t_next;
   c->block_done_seen = false;

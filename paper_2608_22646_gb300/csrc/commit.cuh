@@ -66,6 +66,7 @@ struct CommitParams {
   int* d_M;
   int* m_hist_slot;       // this step's M_t (written by the single-kernel step)
   unsigned* ticket;       // zero between launches
+  unsigned long long* pub;  // (step id + 1) << 32 | masked rows left, written by finish_step
   HostFlag* hf;           // device alias of the mapped host record
   uint32_t* err;
   int B, P, L, n_blocks, T, blk, t, step_id;
@@ -309,6 +310,11 @@ __device__ void finish_step(const CommitParams& p, int remaining = -1) {
     // itself through stream-ordered copies, so no system fence is needed.
     *reinterpret_cast<volatile unsigned long long*>(&p.hf->word) =
         host_flag_word(p.step_id, n == 0, err, p.blk);
+    // Device copy for the next step, which may already be running (see the
+    // LM-head kernel): it stops early when this step left nothing masked.
+    *reinterpret_cast<volatile unsigned long long*>(p.pub) =
+        (static_cast<unsigned long long>(static_cast<uint32_t>(p.step_id + 1)) << 32) |
+        static_cast<uint32_t>(n);
   }
 }
 

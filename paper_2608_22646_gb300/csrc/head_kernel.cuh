@@ -34,9 +34,14 @@
 // B P rows straight from the caller's hidden states (no gather; at N <= 256 a
 // step reads W once whatever N is), and the last CTA to finish (atomic
 // ticket, no waiting) merges the partials and applies the commit rule for
-// every sequence (commit.cuh).  A step is then one launch, and under
-// programmatic dependent launch the next step's prologue and first W stages
-// overlap this step's commit.
+// every sequence (commit.cuh).  A step is then one launch.  Nothing but the
+// commit depends on the previous step: W and the caller's hidden rows are
+// inputs, so under programmatic dependent launch the next step's CTAs start
+// streaming as soon as this step's CTAs leave their SMs, and wait for this
+// step (grid_dependency_wait) only to write their partials (which this
+// step's commit reads) and to commit.  If this step leaves nothing masked,
+// the next one learns it from the published step word (CommitParams::pub)
+// while streaming and stops at the next K block.
 //
 // Warp roles (192 threads, one CTA per SM):
 //   warp 0      producer (one lane): W stages (bulk copies), hidden stages (TMA)
@@ -116,13 +121,27 @@ struct CtaPlan {
 };
 
 // Rows this launch decodes.  Multi-kernel step: the masked rows the gather
-// kernel compacted.  Single-kernel step: all B P rows, unless the previous
-// step left nothing masked in a running sequence (and this is not a block's
-// step zero), in which case there is nothing to decode.  Read after
-// grid_dependency_wait().
-__device__ __forceinline__ int rows_to_decode(const int* d_M, int fused, int first, int M_fixed) {
-  if (!fused) return *d_M;
-  return (first || *d_M > 0) ? M_fixed : 0;
+// kernel compacted, read after grid_dependency_wait().  Single-kernel step:
+// all B P rows, known at launch (a step that turns out to have nothing to
+// decode stops early instead, see `skip`).
+__device__ __forceinline__ int rows_to_decode(const int* d_M, int fused, int M_fixed) {
+  return fused ? M_fixed : *d_M;
+}
+
+// Single-kernel step after step zero: whether the published step word `w`
+// says the previous step left nothing masked.  `decided` is set once the
+// word is the previous step's at all.  Step s publishes s + 1 (never 0,
+// which is the word after a reset or a state upload), so step s + 1 looks
+// for its own id.
+__device__ __forceinline__ unsigned long long load_pub(const unsigned long long* pub) {
+  return *reinterpret_cast<const volatile unsigned long long*>(pub);
+}
+__device__ __forceinline__ bool previous_left_nothing(unsigned long long w, int step_id,
+                                                      bool& decided) {
+  const uint32_t id = static_cast<uint32_t>(w >> 32);
+  if (id == 0u || id != static_cast<uint32_t>(step_id)) return false;
+  decided = true;
+  return static_cast<uint32_t>(w) == 0u;
 }
 
 __host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
@@ -199,6 +218,7 @@ struct HeadSmem {
   uint64_t* epib;    // 2: the four epilogue warps have written epi[buffer]
   uint32_t* tmem_slot;
   volatile int* abort;
+  volatile int* skip;  // the step stops early: nothing was left to decode
 };
 
 __host__ __device__ inline size_t head_smem_bytes(int n_stages, int n_bslots, int b_slot_bytes,
@@ -225,6 +245,7 @@ __device__ __forceinline__ HeadSmem carve(uint8_t* raw, const HeadParams& p) {
   s.epib = s.drain + 1;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.epib + 2);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+  s.skip = s.abort + 1;
   return s;
 }
 
@@ -271,6 +292,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     }
     mbar_init(sm.drain, 1);
     *sm.abort = 0;
+    *sm.skip = 0;
     fence_mbar_init();
   }
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
@@ -287,9 +309,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 
   // The weight does not depend on the previous kernels: the producer starts
   // streaming the first ring of W stages before waiting for them.  Everything
-  // that does (the masked-row count, the gathered rows, the partial buffer)
-  // is touched only after grid_dependency_wait().
+  // that does (the masked-row count, the gathered rows, the partial buffer,
+  // the commit state) is touched only after grid_dependency_wait().  A
+  // single-kernel step reads nothing the previous step writes before its
+  // partials, so only its epilogue and its commit wait.
   const int n_pre = min(p.n_stages, pl.n_tiles * KB);
+  const bool spec = p.fused && !p.first;  // may find out that nothing is masked
 
   if (warp == 0) {
     if (lane == 0) {
@@ -308,21 +333,34 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                         p.wpk + pl.stage_offset(g, kb, t, p.H), bytes, &sm.full_a[i], pol_w);
             }
       }
-      grid_dependency_wait();
-      const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
+      if (!p.fused) grid_dependency_wait();
+      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb;
       long long a_issued = 0, b_issued = 0;
-      bool ok = true;
-      for (int q = 0; q < n_chunks && ok; ++q) {
+      bool ok = true, decided = !spec, skipped = false;
+      // The word is loaded one K block ahead of its use, so its latency never
+      // holds up the stream of copies.
+      unsigned long long pub_w = spec ? load_pub(p.cp.pub) : 0ull;
+      for (int q = 0; q < n_chunks && ok && !skipped; ++q) {
         const int n0 = q * kChunkN;
         const int nq = (min(kChunkN, M - n0) + 15) & ~15;
-        for (int g = 0; g < pl.n_groups && ok; ++g) {
+        for (int g = 0; g < pl.n_groups && ok && !skipped; ++g) {
           for (int kb = 0; kb < KB && ok; ++kb) {
             if (!mbar_wait(&sm.empty_b[rb.slot], rb.phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
               ok = false;
               break;
             }
+            if (!decided && previous_left_nothing(pub_w, p.cp.step_id, decided)) {
+              // Stop at this K block: the hidden stage is completed empty and
+              // carries the stop mark to the MMA warp, which has consumed
+              // every W stage issued so far by the time it sees it.
+              *sm.skip = 1;
+              mbar_arrive(&sm.full_b[rb.slot]);
+              skipped = true;
+              break;
+            }
+            if (!decided) pub_w = load_pub(p.cp.pub);
             mbar_arrive_expect_tx(&sm.full_b[rb.slot], static_cast<uint32_t>(nq * 128));
             uint8_t* bdst = sm.b + static_cast<size_t>(rb.slot) * p.b_slot_bytes;
             for (int i = 0; i < nq / kBoxRowsB; ++i)
@@ -352,8 +390,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         }
       }
       if (a_issued < n_pre) {
-        // Nothing to decode (M = 0) or an abort before the prefetched stages
-        // were claimed: complete their phases so the W copies can be drained.
+        // Nothing to decode (M = 0, or a stop) or an abort before the prefetched
+        // stages were claimed: complete their phases so the copies can drain.
         for (long long i = a_issued; i < n_pre; ++i) mbar_arrive(&sm.full_a[i]);
         for (long long i = a_issued; i < n_pre; ++i) mbar_drain(&sm.full_a[i], 0, p.err);
       }
@@ -373,12 +411,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   } else if (warp == 1) {
     if (lane == 0) {
       // ---------------------------------------------------- MMA issuer --
-      grid_dependency_wait();
-      const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
+      if (!p.fused) grid_dependency_wait();
+      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb, racc;
-      bool ok = true;
-      for (int q = 0; q < n_chunks && ok; ++q) {
+      bool ok = true, skipped = false;
+      for (int q = 0; q < n_chunks && ok && !skipped; ++q) {
         const int n0 = q * kChunkN;
         const int nq = (min(kChunkN, M - n0) + 15) & ~15;
         const uint32_t idesc = idesc_bf16_f32(kRowsPerTile, static_cast<uint32_t>(nq));
@@ -393,6 +431,10 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
           for (int kb = 0; kb < KB && ok; ++kb) {
             if (!mbar_wait(&sm.full_b[rb.slot], rb.phase, sm.abort, p.err, kErrWaitFull)) {
               ok = false;
+              break;
+            }
+            if (spec && *sm.skip) {
+              skipped = true;
               break;
             }
             const uint32_t b_addr =
@@ -419,22 +461,24 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             mma_commit(&sm.empty_b[rb.slot]);
             rb.next(p.n_bslots);
           }
-          if (!ok) break;
+          if (!ok || skipped) break;
           mma_commit(&sm.accf[racc.slot]);
           racc.next(2);
         }
       }
-      if (!ok) {
-        // Abort path: wait for every MMA already issued before TMEM is freed.
+      if (!ok || skipped) {
+        // Abort or stop: wait for every MMA already issued before TMEM is freed.
         mma_commit(sm.drain);
         mbar_drain(sm.drain, 0, p.err);
       }
+      // Stop: release the epilogue, which waits for this group's accumulators.
+      if (skipped) mbar_arrive(&sm.accf[racc.slot]);
     }
     __syncwarp();
   } else {
     // --------------------------------------------------------- epilogue --
-    grid_dependency_wait();
-    const int M = rows_to_decode(p.d_M, p.fused, p.first, p.M_fixed);
+    if (!p.fused) grid_dependency_wait();
+    const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
     const int n_chunks = (M + kChunkN - 1) / kChunkN;
     if (!p.fused && threadIdx.x == 64 && cta == 0) *p.m_hist_slot = M;
     const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
@@ -471,6 +515,10 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             ok = false;
             break;
           }
+          if (spec && *sm.skip) {
+            ok = false;  // stop: nothing of this step is written
+            break;
+          }
           tc_fence_after();
           const uint32_t tgroup =
               tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
@@ -502,6 +550,10 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         for (int g = 0; g < pl.n_groups; ++g) {
           if (!mbar_wait(&sm.accf[racc.slot], racc.phase, sm.abort, p.err, kErrWaitAccFull)) {
             ok = false;
+            break;
+          }
+          if (spec && *sm.skip) {
+            ok = false;  // stop: nothing of this step is written
             break;
           }
           tc_fence_after();
@@ -552,6 +604,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
         ok = false;
         break;
       }
+      // The previous step's commit reads the same partial buffer.
+      if (p.fused) grid_dependency_wait();
       const int ncols = min(nq, M - n0);
       for (int col = ew * 32 + lane; col < ncols; col += 128) {
         const float4 a = epi[col];
@@ -575,7 +629,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   }
 
   if (p.fused) {
-    // Single-kernel step: the last CTA to finish commits the step.
+    // Single-kernel step: the last CTA to finish commits the step, after the
+    // previous step's commit (state, ticket) is complete.
+    grid_dependency_wait();
     __shared__ int s_last;
     if (threadIdx.x == 0) {
       __threadfence();

@@ -11,7 +11,7 @@ CSRC = os.path.join(PKG, "csrc")
 INCLUDE = os.path.join(ROOT, "include")
 LIB = os.path.join(PKG, "libcai.so")
 SOURCES = ["cai.cu"]
-DEPS = ["cai.cu", "ptx.cuh", "softmax.cuh", "commit.cuh", "head_kernel.cuh", "step_kernels.cuh",
+DEPS = ["cai.cu", "ptx.cuh", "softmax.cuh", "commit.cuh", "head_kernel.cuh", "step_kernels.cuh", "pair_kernel.cuh",
         "static_head.cuh"]
 
 

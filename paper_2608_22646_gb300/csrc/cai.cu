@@ -18,6 +18,7 @@
 #include <vector>
 
 #include "cai.h"
+#include "pair_kernel.cuh"
 #include "step_kernels.cuh"
 
 using namespace cai;
@@ -31,6 +32,11 @@ std::atomic<int> g_head_grid_limit{0};
 // environment turns it off (read once per context at cai_init).
 bool pdl_enabled() {
   const char* e = std::getenv("CAI_PDL");
+  return !(e && e[0] == '0');
+}
+
+bool pair_enabled() {
+  const char* e = std::getenv("CAI_PAIR");
   return !(e && e[0] == '0');
 }
 
@@ -149,6 +155,11 @@ struct cai_ctx {
   HostFlag* hf_host = nullptr;
   HostFlag* hf_dev = nullptr;
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
+  void* wt = nullptr;    // tile-major packed copy of W (pack_w_tiles_kernel), pair kernel
+  CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
+  bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
+  int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0;
+  size_t pair_smem = 0;
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
   const void* hid_mapped = nullptr;
@@ -244,6 +255,8 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   CommitParams cp{};
   cp.part = c->part;
   cp.n_part = c->G;
+  cp.n_part_pair = c->n_vt;
+  cp.pair_min_M = c->use_pair ? c->pair_min_M : INT_MAX;
   cp.identity_rows = c->fused ? 1 : 0;
   cp.st = c->st;
   cp.list = c->list;
@@ -323,6 +336,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
   hp.fused = c->fused ? 1 : 0;
   hp.M_fixed = c->BP;
+  hp.max_M = c->use_pair ? c->pair_min_M - 1 : INT_MAX;
   hp.first = first ? 1 : 0;
   hp.part = c->part;
   hp.err = c->err;
@@ -354,8 +368,27 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream,
                  c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
     return check_launch(c);
-  if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.launches++;
+  if (c->use_pair) {
+    // Only one of the two LM-head kernels decodes a step: the other reads
+    // this step's M and returns at once.
+    PairParams pp{};
+    pp.wt = static_cast<const uint8_t*>(c->wt);
+    pp.d_M = c->d_M;
+    pp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
+    pp.part = c->part;
+    pp.err = c->err;
+    pp.V = cfg.V;
+    pp.H = cfg.H;
+    pp.n_vt = c->n_vt;
+    pp.min_M = c->pair_min_M;
+    pp.n_stages = c->pair_stages;
+    if (launch_pdl(c->pdl, lm_head_pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
+                   c->tm_a, pp) != cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
+  }
+  if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.head_launches++;
 
   if (!c->fused) {
@@ -486,6 +519,46 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->n_bslots = bslots_for(stages);
   c->head_smem = head_smem_bytes(stages, c->n_bslots, c->b_slot_bytes, c->slot_cols);
 
+  // Pair kernel (multi-kernel steps only): steps with at least pair_min_M
+  // masked rows are tensor-bound and run on CTA pairs; a persistent grid of
+  // as many 2-CTA clusters as can be resident at once.  CAI_PAIR=0 disables
+  // it, CAI_PAIR_MIN_M sets the threshold.
+  c->use_pair = !c->fused && pair_enabled();
+  if (c->use_pair) {
+    const int mset = env_int("CAI_PAIR_MIN_M");
+    c->pair_min_M = mset > 0 ? mset : 128;
+    c->n_vt = (cfg->V + kPairTileVocab - 1) / kPairTileVocab;
+    cudaFuncAttributes pa{};
+    if (cudaFuncGetAttributes(&pa, lm_head_pair_kernel) != cudaSuccess) {
+      cudaGetLastError();
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    const size_t plimit = static_cast<size_t>(smem_optin) - pa.sharedSizeBytes;
+    int ps = 6;
+    while (ps > 2 && pair_smem_bytes(ps) > plimit) --ps;
+    c->pair_stages = ps;
+    c->pair_smem = pair_smem_bytes(ps);
+    int clusters = 0;
+    if (cudaFuncSetAttribute(lm_head_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                             static_cast<int>(c->pair_smem)) != cudaSuccess) {
+      cudaGetLastError();
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    cudaLaunchConfig_t qc = {};
+    qc.gridDim = dim3(static_cast<unsigned>(sms & ~1));
+    qc.blockDim = dim3(kPairThreads);
+    qc.dynamicSmemBytes = c->pair_smem;
+    if (cudaOccupancyMaxActiveClusters(&clusters, lm_head_pair_kernel, &qc) != cudaSuccess ||
+        clusters < 1) {
+      cudaGetLastError();
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    c->pair_grid = 2 * clusters;
+  }
+
   const size_t BL = static_cast<size_t>(cfg->B) * c->L;
   const size_t BN = static_cast<size_t>(cfg->B) * cfg->n_blocks;
   void* p;
@@ -515,7 +588,10 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->pub, unsigned long long, 1)
   CAI_ALLOC(c->err, uint32_t, 1)
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
-  CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * c->G)
+  CAI_ALLOC(c->part, float4,
+            static_cast<size_t>(c->rows_cap) * (c->use_pair && c->n_vt > c->G ? c->n_vt : c->G))
+  if (c->use_pair)
+    CAI_ALLOC(c->wt, uint8_t, static_cast<size_t>(2 * c->n_vt) * kPairHalf * 2 * cfg->H)
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
   CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   const void* w_src = W;
@@ -540,6 +616,10 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
         c->gmax, n_chunks);
+    if (c->use_pair)
+      pack_w_tiles_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+          static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wt), cfg->V, cfg->H,
+          static_cast<long long>(2 * c->n_vt) * kPairHalf * cfg->H / 8);
     const cudaError_t e1 = cudaGetLastError();
     const cudaError_t e2 = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
     if (w_tmp) cudaFree(w_tmp);
@@ -560,7 +640,8 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     return CAI_ERR_NOMEM;
   }
   std::memset(c->hf_host, 0, sizeof(HostFlag));
-  if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB)) {
+  if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB) ||
+      (c->use_pair && !make_map(&c->tm_a, c->hc, c->rows_cap, cfg->H, kPairHalf))) {
     release(c);
     delete c;
     return CAI_ERR_CUDA;
@@ -586,7 +667,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->stats.grid = c->G;
   c->stats.stages = c->n_stages;
   c->stats.n_max = c->n_max;
-  c->stats.kernels_per_step = c->fused ? 1 : 3;
+  c->stats.kernels_per_step = c->fused ? 1 : c->use_pair ? 4 : 3;
   r = cai_reset(c, stream);
   if (r != CAI_OK) {
     release(c);

@@ -59,6 +59,8 @@ struct StateArrays {
 struct CommitParams {
   const float4* part;     // [rows, n_part] softmax partials of this step
   int n_part;             // partial slots per row (one per LM-head CTA)
+  int n_part_pair;        // partial slots per row when the pair kernel decoded the step
+  int pair_min_M;         // steps with at least this many rows ran the pair kernel
   int identity_rows;      // 1: row of (b, p) is b P + p; 0: row_of[b P + p]
   StateArrays st;
   int* list;
@@ -105,7 +107,7 @@ struct CommitSmem {
   uint8_t bud[kMaxP];  // budget before this step
 };
 
-__device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs,
+__device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs, int n_part,
                                      int* left_after = nullptr) {
   __shared__ int s_eta, s_left, s_reason, s_unres, s_ell, s_running;
   int* s_tok = cs.tok;
@@ -150,11 +152,11 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
       }
 #pragma unroll
       for (int j = 0; j < kPosPerWarp; ++j) {
-        const float4* pr = p.part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * p.n_part;
+        const float4* pr = p.part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * n_part;
 #pragma unroll
         for (int u = 0; u < kPartPerLane; ++u) {
           const int k = lane + 32 * u;
-          q[j][u] = (row[j] >= 0 && k < p.n_part)
+          q[j][u] = (row[j] >= 0 && k < n_part)
                         ? __ldcg(pr + k)
                         : make_float4(kNegBig, 0.0f, __int_as_float(INT_MAX), 0.0f);
         }
@@ -168,8 +170,8 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
 #pragma unroll
         for (int u = 0; u < kPartPerLane; ++u)
           merge_tri(m, s, ix, q[j][u].x, q[j][u].y, __float_as_int(q[j][u].z));
-        for (int k = lane + 32 * kPartPerLane; k < p.n_part; k += 32) {
-          const float4 r = __ldcg(p.part + static_cast<size_t>(row[j]) * p.n_part + k);
+        for (int k = lane + 32 * kPartPerLane; k < n_part; k += 32) {
+          const float4 r = __ldcg(p.part + static_cast<size_t>(row[j]) * n_part + k);
           merge_tri(m, s, ix, r.x, r.y, __float_as_int(r.z));
         }
 #pragma unroll

@@ -71,6 +71,7 @@ struct HeadParams {
   int* m_hist_slot;    // where this step's M is recorded (multi-kernel step)
   int fused;           // 1: single-kernel step (see below), 0: gather / head / merge kernels
   int M_fixed;         // rows decoded by the single-kernel step (all B P positions)
+  int max_M;           // multi-kernel step: larger steps are left to lm_head_pair_kernel
   int first;           // the step is a block's step zero (every position masked)
   float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
   uint32_t* err;       // error word
@@ -121,11 +122,14 @@ struct CtaPlan {
 };
 
 // Rows this launch decodes.  Multi-kernel step: the masked rows the gather
-// kernel compacted, read after grid_dependency_wait().  Single-kernel step:
+// kernel compacted, read after grid_dependency_wait(), unless there are more
+// than max_M (lm_head_pair_kernel decodes those steps).  Single-kernel step:
 // all B P rows, known at launch (a step that turns out to have nothing to
 // decode stops early instead, see `skip`).
-__device__ __forceinline__ int rows_to_decode(const int* d_M, int fused, int M_fixed) {
-  return fused ? M_fixed : *d_M;
+__device__ __forceinline__ int rows_to_decode(const int* d_M, int fused, int M_fixed, int max_M) {
+  if (fused) return M_fixed;
+  const int m = *d_M;
+  return m > max_M ? 0 : m;
 }
 
 // Single-kernel step after step zero: whether the published step word `w`
@@ -334,7 +338,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             }
       }
       if (!p.fused) grid_dependency_wait();
-      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
+      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed, p.max_M);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb;
       long long a_issued = 0, b_issued = 0;
@@ -412,7 +416,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     if (lane == 0) {
       // ---------------------------------------------------- MMA issuer --
       if (!p.fused) grid_dependency_wait();
-      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
+      const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed, p.max_M);
       const int n_chunks = (M + kChunkN - 1) / kChunkN;
       Ring ra, rb, racc;
       bool ok = true, skipped = false;
@@ -478,9 +482,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   } else {
     // --------------------------------------------------------- epilogue --
     if (!p.fused) grid_dependency_wait();
-    const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed);
+    const int M = rows_to_decode(p.d_M, p.fused, p.M_fixed, p.max_M);
     const int n_chunks = (M + kChunkN - 1) / kChunkN;
-    if (!p.fused && threadIdx.x == 64 && cta == 0) *p.m_hist_slot = M;
+    if (!p.fused && threadIdx.x == 64 && cta == 0 && *p.d_M <= p.max_M) *p.m_hist_slot = M;
     const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
@@ -644,7 +648,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     for (int b = 0; b < p.cp.B; ++b) {
       int left = 0;
       // Every copy and MMA has completed: the W ring is free shared memory.
-      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), &left);
+      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), p.cp.n_part,
+                                       &left);
       remaining += left;
     }
     if (threadIdx.x == 0) *p.cp.m_hist_slot = decoded;

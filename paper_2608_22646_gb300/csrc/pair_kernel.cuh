@@ -1,0 +1,343 @@
+// LM head for steps with many masked rows (M > 128, several sequences), on
+// CTA pairs: the same quantities as lm_head_softmax_kernel (Box 1 of arXiv
+// 2608.22646: c_i = max_v p_theta(x_i = v) and argmax_v p_theta, logits never
+// leaving tensor memory), computed in the orientation a compute-bound
+// contraction wants.
+//
+// With hundreds to thousands of rows the contraction is tensor-bound (2 V H M
+// flops against 2 V H bytes of W), so it is run without swapping A and B:
+// the masked rows fill the MMA M dimension and the vocabulary the N dimension.
+// One tcgen05.mma of the pair (cta_group::2) computes a 256 x 256 tile:
+// each CTA holds 128 of the rows (its A half) and 128 of the vocabulary rows
+// (its B half) per K block, and keeps its 128 x 256 half of the accumulator
+// in tensor memory.  Per K block a CTA loads 32 KiB (16 KiB of hidden rows,
+// 16 KiB of W) for 2 * 128 * 256 * 64 flops, half the shared-memory traffic
+// per flop of a single-CTA 128 x 256 tile.
+//
+// A tensor-memory lane holds one row's logits, so the epilogue is a serial
+// online softmax per thread over the 256 columns of a tile, no shuffles.  It
+// writes one partial (max * log2 e, sum of 2^(z log2 e - max), argmax) per
+// row and vocabulary tile; the merge kernel combines a row's partials.
+//
+// Work: tiles (v, j) of 256 vocabulary rows x 256 masked rows, numbered
+// t = v * n_rt + j and dealt round-robin to the pairs of a persistent grid.
+// The pairs working at one time share few W tiles, each read from HBM once
+// and by the n_rt pairs of its row tiles from L2; the gathered hidden rows
+// (at most 2 x 65536 x 16384 bytes, in practice tens of MB) stay in L2.
+//
+// Roles per CTA (192 threads): warp 0 producer (hidden half by TMA, W half by
+// one bulk copy from a tile-major packed copy of W); warp 1 allocates tensor
+// memory and, in the even CTA, issues the MMAs, or, in the odd CTA, relays the
+// arrival of its stages to the even CTA; warps 2..5 epilogue.  Two
+// accumulator buffers let the epilogue of one tile overlap the next tile's MMAs.
+#pragma once
+
+#include <climits>
+#include "ptx.cuh"
+#include "softmax.cuh"
+
+namespace cai {
+
+constexpr int kPairThreads = 192;
+constexpr int kPairTileRows = 256;    // masked rows per pair tile (MMA M)
+constexpr int kPairTileVocab = 256;   // vocabulary rows per pair tile (MMA N)
+constexpr int kPairHalf = 128;        // rows of each per CTA
+constexpr int kPairBlockK = 64;       // K per stage (one 128-byte swizzled row)
+constexpr int kPairHalfBytes = kPairHalf * kPairBlockK * 2;  // 16 KiB
+constexpr int kPairStageBytes = 2 * kPairHalfBytes;          // A half + B half
+constexpr int kPairTmemCols = 2 * kPairTileVocab;            // two accumulators
+
+struct PairParams {
+  const uint8_t* wt;   // W packed tile-major (pack_w_tiles_kernel), 2 n_vt tiles of 128 rows
+  const int* d_M;      // masked rows of this step (device)
+  int* m_hist_slot;    // where this step's M is recorded, or null
+  float4* part;        // [rows, n_vt] partial per row and vocabulary tile
+  uint32_t* err;
+  int V, H;
+  int n_vt;            // ceil(V / 256)
+  int min_M;           // smaller steps are left to lm_head_softmax_kernel
+  int n_stages;
+};
+
+__host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
+  return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes +
+         static_cast<size_t>(3 * n_stages + 5) * 8 + 16;
+}
+
+// Pack W [V, H] (row-major bf16) tile-major for the pair kernel: 128-row
+// tile t, K block kb is the 16 KiB block at (t * (H / 64) + kb) * 16 KiB, in
+// the 128-byte-swizzled K-major layout (row r's 16-byte chunk c at
+// r * 128 + (c ^ (r & 7)) * 16).  Rows >= V are zero; n_tiles = 2 n_vt.
+__global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
+                                    int H, long long n_chunks) {
+  const int KB = H / kPairBlockK;
+  const long long tile_chunks = static_cast<long long>(KB) * (kPairHalfBytes / 16);
+  for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
+       d += static_cast<long long>(gridDim.x) * blockDim.x) {
+    const long long t = d / tile_chunks;
+    const int rem = static_cast<int>(d - t * tile_chunks);
+    const int kb = rem / (kPairHalfBytes / 16);
+    const int inblk = rem % (kPairHalfBytes / 16);  // 16-byte chunk in the block
+    const int r = inblk >> 3;
+    const int cl = (inblk & 7) ^ (r & 7);
+    const long long v = t * kPairHalf + r;
+    uint4 val = make_uint4(0u, 0u, 0u, 0u);
+    if (v < V) val = W[(v * H + static_cast<long long>(kb) * kPairBlockK) / 8 + cl];
+    out[d] = val;
+  }
+}
+
+struct PairSmem {
+  uint8_t* stage;      // n_stages x (A half, B half)
+  uint64_t* full;      // n_stages: this CTA's stage landed
+  uint64_t* empty;     // n_stages: the pair's MMAs are done with the stage
+  uint64_t* pfull;     // n_stages (even CTA): the odd CTA's stage landed
+  uint64_t* accf;      // 2: accumulator ready
+  uint64_t* acce;      // 2 (even CTA): accumulator drained by both epilogues
+  uint64_t* drain;     // 1 (even CTA): abort path, issued MMAs complete
+  uint32_t* tmem_slot;
+  volatile int* abort;
+};
+
+__device__ __forceinline__ PairSmem pair_carve(uint8_t* raw, int n_stages) {
+  PairSmem s;
+  uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) &
+                                             ~static_cast<uintptr_t>(1023));
+  s.stage = base;
+  s.full = reinterpret_cast<uint64_t*>(base + static_cast<size_t>(n_stages) * kPairStageBytes);
+  s.empty = s.full + n_stages;
+  s.pfull = s.empty + n_stages;
+  s.accf = s.pfull + n_stages;
+  s.acce = s.accf + 2;
+  s.drain = s.acce + 2;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
+  s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
+  return s;
+}
+
+struct PairRing {
+  int slot = 0;
+  uint32_t phase = 0;
+  __device__ void next(int n) {
+    if (++slot == n) {
+      slot = 0;
+      phase ^= 1u;
+    }
+  }
+};
+
+__device__ __forceinline__ void pair_drain(uint64_t* bar, uint32_t parity, uint32_t* err) {
+  const uint64_t t0 = global_timer_ns();
+  while (!mbar_try_wait(bar, parity)) {
+    if (global_timer_ns() - t0 > kWaitLimitNs) {
+      atomicOr(err, kErrDrain);
+      return;
+    }
+  }
+}
+
+__global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
+    lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const PairParams p) {
+  extern __shared__ uint8_t smem_raw[];
+  const int warp = threadIdx.x >> 5;
+  const int lane = threadIdx.x & 31;
+  const uint32_t rank = cluster_ctarank();  // 0: even CTA (issues the MMAs), 1: odd
+  const int pair = blockIdx.x >> 1;
+  const int n_pairs = gridDim.x >> 1;
+
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // d_M and the gathered rows of this step
+  const int M = *p.d_M;
+  if (M < p.min_M) return;  // both CTAs of every pair take the same branch
+  if (p.m_hist_slot && blockIdx.x == 0 && threadIdx.x == 0) *p.m_hist_slot = M;
+
+  PairSmem sm = pair_carve(smem_raw, p.n_stages);
+  const int KB = p.H / kPairBlockK;
+  const int n_rt = (M + kPairTileRows - 1) / kPairTileRows;
+  const int n_tiles = p.n_vt * n_rt;
+  const int my_tiles = pair < n_tiles ? (n_tiles - pair + n_pairs - 1) / n_pairs : 0;
+
+  if (threadIdx.x == 0) {
+    for (int s = 0; s < p.n_stages; ++s) {
+      mbar_init(&sm.full[s], 1);
+      mbar_init(&sm.empty[s], 1);
+      mbar_init(&sm.pfull[s], 1);
+    }
+    for (int a = 0; a < 2; ++a) {
+      mbar_init(&sm.accf[a], 1);
+      mbar_init(&sm.acce[a], 8);  // four epilogue warps in each CTA
+    }
+    mbar_init(sm.drain, 1);
+    *sm.abort = 0;
+    fence_mbar_init();
+  }
+  if (warp == 0 && lane == 0) prefetch_tmap(&tm_a);
+  if (warp == 1) {
+    tmem_alloc_pair(sm.tmem_slot, kPairTmemCols);
+    tmem_relinquish_pair();
+  }
+  tc_fence_before();
+  cluster_sync();  // barriers of both CTAs initialised, tensor memory allocated
+  tc_fence_after();
+  const uint32_t tmem_base = *sm.tmem_slot;
+
+  if (warp == 0) {
+    if (lane == 0) {
+      // ------------------------------------------------------ producer --
+      const uint64_t pol_a = policy_evict_last();
+      PairRing r;
+      long long issued = 0;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int t = pair + i * n_pairs;
+        const int v = t / n_rt, j = t - v * n_rt;
+        const int a_row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf;
+        const uint8_t* wsrc =
+            p.wt + (static_cast<size_t>(2 * v + static_cast<int>(rank)) * KB) * kPairHalfBytes;
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&sm.empty[r.slot], r.phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
+            ok = false;
+            break;
+          }
+          uint8_t* dst = sm.stage + static_cast<size_t>(r.slot) * kPairStageBytes;
+          mbar_arrive_expect_tx(&sm.full[r.slot], kPairStageBytes);
+          tma_load_2d(dst, &tm_a, &sm.full[r.slot], kb * kPairBlockK, a_row, pol_a);
+          bulk_load_nohint(dst + kPairHalfBytes, wsrc + static_cast<size_t>(kb) * kPairHalfBytes,
+                           kPairHalfBytes, &sm.full[r.slot]);
+          ++issued;
+          r.next(p.n_stages);
+        }
+      }
+      if (!ok) {
+        const long long f0 = issued > p.n_stages ? issued - p.n_stages : 0;
+        for (long long q = f0; q < issued; ++q)
+          pair_drain(&sm.full[q % p.n_stages], static_cast<uint32_t>((q / p.n_stages) & 1), p.err);
+      }
+    }
+    __syncwarp();
+  } else if (warp == 1) {
+    if (lane == 0 && rank == 0) {
+      // -------------------------------------------- MMA issuer (even CTA) --
+      const uint32_t idesc = idesc_bf16_f32(kPairTileRows, kPairTileVocab);
+      PairRing r;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        const int acc = i & 1;
+        if (!mbar_wait_cluster(&sm.acce[acc], ((i >> 1) & 1) ^ 1u, sm.abort, p.err,
+                               kErrWaitAccEmpty)) {
+          ok = false;
+          break;
+        }
+        tc_fence_after();
+        const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kPairTileVocab);
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&sm.full[r.slot], r.phase, sm.abort, p.err, kErrWaitFull) ||
+              !mbar_wait_cluster(&sm.pfull[r.slot], r.phase, sm.abort, p.err, kErrWaitFull)) {
+            ok = false;
+            break;
+          }
+          tc_fence_after();
+          const uint32_t a_addr = smem_addr(sm.stage + static_cast<size_t>(r.slot) * kPairStageBytes);
+          const uint32_t b_addr = a_addr + kPairHalfBytes;
+#pragma unroll
+          for (int kk = 0; kk < kPairBlockK / 16; ++kk)
+            mma_bf16_pair(d_tmem, sdesc_k_sw128(a_addr + kk * 32), sdesc_k_sw128(b_addr + kk * 32),
+                          idesc, (kb | kk) != 0 ? 1u : 0u);
+          mma_commit_pair(&sm.empty[r.slot], 0x3);
+          r.next(p.n_stages);
+        }
+        if (!ok) break;
+        mma_commit_pair(&sm.accf[acc], 0x3);
+      }
+      if (!ok) {
+        // Abort: wait for the MMAs already issued (they read both CTAs'
+        // shared memory) before anything is released.
+        mma_commit_pair(sm.drain, 0x1);
+        pair_drain(sm.drain, 0, p.err);
+      }
+    } else if (lane == 0) {
+      // ------------------------------------------------ relay (odd CTA) --
+      const uint32_t leader_pfull = mapa_shared(sm.pfull, 0);
+      PairRing r;
+      bool ok = true;
+      for (int i = 0; i < my_tiles && ok; ++i) {
+        for (int kb = 0; kb < KB; ++kb) {
+          if (!mbar_wait(&sm.full[r.slot], r.phase, sm.abort, p.err, kErrWaitFull)) {
+            ok = false;
+            break;
+          }
+          mbar_arrive_cluster(leader_pfull + static_cast<uint32_t>(r.slot * 8));
+          r.next(p.n_stages);
+        }
+      }
+    }
+    __syncwarp();
+  } else {
+    // --------------------------------------------------------- epilogue --
+    const int quarter = warp & 3;  // tensor-memory lanes 32 quarter .. 32 quarter + 31
+    const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t acce_remote = mapa_shared(sm.acce, 0);
+    for (int i = 0; i < my_tiles; ++i) {
+      const int t = pair + i * n_pairs;
+      const int v = t / n_rt, j = t - v * n_rt;
+      const int acc = i & 1;
+      if (!mbar_wait(&sm.accf[acc], (i >> 1) & 1, sm.abort, p.err, kErrWaitAccFull)) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + lane_base + static_cast<uint32_t>(acc * kPairTileVocab);
+      const int vbase = v * kPairTileVocab;
+      float m = kNegBig, s = 0.0f;
+      int ix = INT_MAX;
+#pragma unroll 1
+      for (int c = 0; c < kPairTileVocab / 32; ++c) {
+        uint32_t x[32];
+        tmem_ld_32cols(tbase + static_cast<uint32_t>(32 * c), x);
+        tmem_ld_wait();
+        const int v0 = vbase + 32 * c;
+        const int nvalid = min(32, p.V - v0);  // vocabulary rows past V are zero padding
+        float cm = kNegBig;
+        int ci = 0;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float z = __uint_as_float(x[k]) * kLog2e;
+          if (k < nvalid && z > cm) {
+            cm = z;
+            ci = k;
+          }
+        }
+        if (cm > m) {  // strictly: an equal maximum keeps the lower index
+          s *= fast_exp2(m - cm);
+          m = cm;
+          ix = v0 + ci;
+        }
+        float cs = 0.0f;
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          const float z = __uint_as_float(x[k]) * kLog2e;
+          cs += k < nvalid ? fast_exp2(z - m) : 0.0f;
+        }
+        s += cs;
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (rank == 0)
+          mbar_arrive(&sm.acce[acc]);
+        else
+          mbar_arrive_cluster(acce_remote + static_cast<uint32_t>(acc * 8));
+      }
+      const int row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf + quarter * 32 + lane;
+      if (row < M)
+        p.part[static_cast<size_t>(row) * p.n_vt + v] = make_float4(m, s, __int_as_float(ix), 0.0f);
+    }
+  }
+
+  tc_fence_before();
+  __syncthreads();
+  cluster_sync();  // no CTA leaves while the pair's MMAs or arrivals may touch it
+  if (warp == 1) {
+    tc_fence_after();
+    tmem_dealloc_pair(tmem_base, kPairTmemCols);
+  }
+}
+
+}  // namespace cai

@@ -83,7 +83,10 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
   __shared__ CommitSmem cs;
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // partials of this step, state of the previous one
-  merge_commit_sequence(p, blockIdx.x, cs);
+  // This step's M (d_M is rewritten only by the last CTA, after every CTA's
+  // merge) tells which LM-head kernel wrote the partials.
+  const int n_part = *p.d_M >= p.pair_min_M ? p.n_part_pair : p.n_part;
+  merge_commit_sequence(p, blockIdx.x, cs, n_part);
   if (gridDim.x > 1) {
     if (threadIdx.x == 0) {
       __threadfence();

@@ -88,7 +88,8 @@ EncodeTiledFn get_encoder() {
 
 // Row-major bf16 matrix [rows, cols] with a box of box_rows x 64 columns and
 // the 128-byte swizzle that the MMA descriptors expect.
-bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows) {
+bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint32_t box_rows,
+              CUtensorMapSwizzle swizzle = CU_TENSOR_MAP_SWIZZLE_128B) {
   EncodeTiledFn enc = get_encoder();
   if (!enc) return false;
   cuuint64_t dims[2] = {cols, rows};
@@ -96,7 +97,7 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
   cuuint32_t box[2] = {static_cast<cuuint32_t>(kBlockK), box_rows};
   cuuint32_t estr[2] = {1, 1};
   return enc(m, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(base), dims, strides, box,
-             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, CU_TENSOR_MAP_SWIZZLE_128B,
+             estr, CU_TENSOR_MAP_INTERLEAVE_NONE, swizzle,
              CU_TENSOR_MAP_L2_PROMOTION_L2_256B, CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
@@ -157,6 +158,7 @@ struct cai_ctx {
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
   void* wt = nullptr;    // tile-major packed copy of W (pack_w_tiles_kernel), pair kernel
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
+  CUtensorMap tm_w{};    // wt as [2 n_vt (H / 64) 128, 64], 16 KiB unswizzled boxes
   bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
   int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0;
   size_t pair_smem = 0;
@@ -373,7 +375,6 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     // Only one of the two LM-head kernels decodes a step: the other reads
     // this step's M and returns at once.
     PairParams pp{};
-    pp.wt = static_cast<const uint8_t*>(c->wt);
     pp.d_M = c->d_M;
     pp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
     pp.part = c->part;
@@ -384,7 +385,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     pp.min_M = c->pair_min_M;
     pp.n_stages = c->pair_stages;
     if (launch_pdl(c->pdl, lm_head_pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
-                   c->tm_a, pp) != cudaSuccess)
+                   c->tm_a, c->tm_w, pp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
   }
@@ -641,7 +642,11 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   }
   std::memset(c->hf_host, 0, sizeof(HostFlag));
   if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB) ||
-      (c->use_pair && !make_map(&c->tm_a, c->hc, c->rows_cap, cfg->H, kPairHalf))) {
+      (c->use_pair && !make_map(&c->tm_a, c->hc, c->rows_cap, cfg->H, kPairHalf)) ||
+      (c->use_pair &&
+       !make_map(&c->tm_w, c->wt, static_cast<uint64_t>(2 * c->n_vt) * (cfg->H / kPairBlockK) *
+                                      kPairHalf,
+                 kPairBlockK, kPairHalf, CU_TENSOR_MAP_SWIZZLE_NONE))) {
     release(c);
     delete c;
     return CAI_ERR_CUDA;

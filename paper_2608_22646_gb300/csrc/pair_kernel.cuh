@@ -25,11 +25,13 @@
 // and by the n_rt pairs of its row tiles from L2; the gathered hidden rows
 // (at most 2 x 65536 x 16384 bytes, in practice tens of MB) stay in L2.
 //
-// Roles per CTA (192 threads): warp 0 producer (hidden half by TMA, W half by
-// one bulk copy from a tile-major packed copy of W); warp 1 allocates tensor
-// memory and, in the even CTA, issues the MMAs, or, in the odd CTA, relays the
-// arrival of its stages to the even CTA; warps 2..5 epilogue.  Two
-// accumulator buffers let the epilogue of one tile overlap the next tile's MMAs.
+// Roles per CTA (192 threads): warp 0 producer (hidden half and W half, each
+// one TMA box; W from a tile-major packed copy in which every box is one
+// contiguous 16 KiB block); warp 1 allocates tensor memory and, in the even
+// CTA, issues the MMAs; warps 2..5 epilogue.  Both CTAs' copies of a stage
+// complete on the even CTA's barrier (cta_group::2 loads), which the even
+// CTA's producer arms with the bytes of both.  Two accumulator buffers let
+// the epilogue of one tile overlap the next tile's MMAs.
 #pragma once
 
 #include <climits>
@@ -48,7 +50,6 @@ constexpr int kPairStageBytes = 2 * kPairHalfBytes;          // A half + B half
 constexpr int kPairTmemCols = 2 * kPairTileVocab;            // two accumulators
 
 struct PairParams {
-  const uint8_t* wt;   // W packed tile-major (pack_w_tiles_kernel), 2 n_vt tiles of 128 rows
   const int* d_M;      // masked rows of this step (device)
   int* m_hist_slot;    // where this step's M is recorded, or null
   float4* part;        // [rows, n_vt] partial per row and vocabulary tile
@@ -61,13 +62,15 @@ struct PairParams {
 
 __host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
   return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes +
-         static_cast<size_t>(3 * n_stages + 5) * 8 + 16;
+         static_cast<size_t>(2 * n_stages + 5) * 8 + 16;
 }
 
 // Pack W [V, H] (row-major bf16) tile-major for the pair kernel: 128-row
 // tile t, K block kb is the 16 KiB block at (t * (H / 64) + kb) * 16 KiB, in
 // the 128-byte-swizzled K-major layout (row r's 16-byte chunk c at
-// r * 128 + (c ^ (r & 7)) * 16).  Rows >= V are zero; n_tiles = 2 n_vt.
+// r * 128 + (c ^ (r & 7)) * 16).  Rows >= V are zero; n_tiles = 2 n_vt.  The
+// kernel reads it through a tensor map of [2 n_vt (H / 64) 128, 64] bf16 with
+// 64 x 128 boxes and no swizzle: box (t (H / 64) + kb) is that block.
 __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
                                     int H, long long n_chunks) {
   const int KB = H / kPairBlockK;
@@ -89,9 +92,8 @@ __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restri
 
 struct PairSmem {
   uint8_t* stage;      // n_stages x (A half, B half)
-  uint64_t* full;      // n_stages: this CTA's stage landed
+  uint64_t* full;      // n_stages (even CTA): both CTAs' halves of the stage landed
   uint64_t* empty;     // n_stages: the pair's MMAs are done with the stage
-  uint64_t* pfull;     // n_stages (even CTA): the odd CTA's stage landed
   uint64_t* accf;      // 2: accumulator ready
   uint64_t* acce;      // 2 (even CTA): accumulator drained by both epilogues
   uint64_t* drain;     // 1 (even CTA): abort path, issued MMAs complete
@@ -106,8 +108,7 @@ __device__ __forceinline__ PairSmem pair_carve(uint8_t* raw, int n_stages) {
   s.stage = base;
   s.full = reinterpret_cast<uint64_t*>(base + static_cast<size_t>(n_stages) * kPairStageBytes);
   s.empty = s.full + n_stages;
-  s.pfull = s.empty + n_stages;
-  s.accf = s.pfull + n_stages;
+  s.accf = s.empty + n_stages;
   s.acce = s.accf + 2;
   s.drain = s.acce + 2;
   s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
@@ -137,7 +138,8 @@ __device__ __forceinline__ void pair_drain(uint64_t* bar, uint32_t parity, uint3
 }
 
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
-    lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_a, const PairParams p) {
+    lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_a,
+                        const __grid_constant__ CUtensorMap tm_w, const PairParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -161,7 +163,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     for (int s = 0; s < p.n_stages; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], 1);
-      mbar_init(&sm.pfull[s], 1);
     }
     for (int a = 0; a < 2; ++a) {
       mbar_init(&sm.accf[a], 1);
@@ -171,7 +172,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     *sm.abort = 0;
     fence_mbar_init();
   }
-  if (warp == 0 && lane == 0) prefetch_tmap(&tm_a);
+  if (warp == 0 && lane == 0) {
+    prefetch_tmap(&tm_a);
+    prefetch_tmap(&tm_w);
+  }
   if (warp == 1) {
     tmem_alloc_pair(sm.tmem_slot, kPairTmemCols);
     tmem_relinquish_pair();
@@ -185,6 +189,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     if (lane == 0) {
       // ------------------------------------------------------ producer --
       const uint64_t pol_a = policy_evict_last();
+      const uint32_t full0 = mapa_shared(sm.full, 0);  // the even CTA's barriers
       PairRing r;
       long long issued = 0;
       bool ok = true;
@@ -192,23 +197,24 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         const int t = pair + i * n_pairs;
         const int v = t / n_rt, j = t - v * n_rt;
         const int a_row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf;
-        const uint8_t* wsrc =
-            p.wt + (static_cast<size_t>(2 * v + static_cast<int>(rank)) * KB) * kPairHalfBytes;
+        const int w_box = (2 * v + static_cast<int>(rank)) * KB;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&sm.empty[r.slot], r.phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
             ok = false;
             break;
           }
           uint8_t* dst = sm.stage + static_cast<size_t>(r.slot) * kPairStageBytes;
-          mbar_arrive_expect_tx(&sm.full[r.slot], kPairStageBytes);
-          tma_load_2d(dst, &tm_a, &sm.full[r.slot], kb * kPairBlockK, a_row, pol_a);
-          bulk_load_nohint(dst + kPairHalfBytes, wsrc + static_cast<size_t>(kb) * kPairHalfBytes,
-                           kPairHalfBytes, &sm.full[r.slot]);
+          const uint32_t bar = full0 + static_cast<uint32_t>(r.slot * 8);
+          // The even CTA arms the stage for the bytes of both CTAs; a copy of
+          // the odd CTA that completes first leaves the phase open until then.
+          if (rank == 0) mbar_arrive_expect_tx(&sm.full[r.slot], 2 * kPairStageBytes);
+          tma_load_2d_pair(dst, &tm_a, bar, kb * kPairBlockK, a_row, pol_a);
+          tma_load_2d_pair_nohint(dst + kPairHalfBytes, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
           ++issued;
           r.next(p.n_stages);
         }
       }
-      if (!ok) {
+      if (!ok && rank == 0) {
         const long long f0 = issued > p.n_stages ? issued - p.n_stages : 0;
         for (long long q = f0; q < issued; ++q)
           pair_drain(&sm.full[q % p.n_stages], static_cast<uint32_t>((q / p.n_stages) & 1), p.err);
@@ -231,8 +237,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         tc_fence_after();
         const uint32_t d_tmem = tmem_base + static_cast<uint32_t>(acc * kPairTileVocab);
         for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&sm.full[r.slot], r.phase, sm.abort, p.err, kErrWaitFull) ||
-              !mbar_wait_cluster(&sm.pfull[r.slot], r.phase, sm.abort, p.err, kErrWaitFull)) {
+          if (!mbar_wait_cluster(&sm.full[r.slot], r.phase, sm.abort, p.err, kErrWaitFull)) {
             ok = false;
             break;
           }
@@ -254,21 +259,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         // shared memory) before anything is released.
         mma_commit_pair(sm.drain, 0x1);
         pair_drain(sm.drain, 0, p.err);
-      }
-    } else if (lane == 0) {
-      // ------------------------------------------------ relay (odd CTA) --
-      const uint32_t leader_pfull = mapa_shared(sm.pfull, 0);
-      PairRing r;
-      bool ok = true;
-      for (int i = 0; i < my_tiles && ok; ++i) {
-        for (int kb = 0; kb < KB; ++kb) {
-          if (!mbar_wait(&sm.full[r.slot], r.phase, sm.abort, p.err, kErrWaitFull)) {
-            ok = false;
-            break;
-          }
-          mbar_arrive_cluster(leader_pfull + static_cast<uint32_t>(r.slot * 8));
-          r.next(p.n_stages);
-        }
       }
     }
     __syncwarp();

@@ -181,6 +181,29 @@ __device__ __forceinline__ void tma_load_2d_nohint(void* dst, const CUtensorMap*
       : "memory");
 }
 
+// 2-D tiled TMA load by either CTA of a pair (cta_group::2) whose completion
+// is signalled on an mbarrier of the even CTA (`bar_cluster`, a
+// shared::cluster address from mapa_shared); the data lands in the issuing
+// CTA's shared memory.
+__device__ __forceinline__ void tma_load_2d_pair(void* dst, const CUtensorMap* map,
+                                                 uint32_t bar_cluster, int32_t x, int32_t y,
+                                                 uint64_t policy) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".cta_group::2.L2::cache_hint [%0], [%1, {%3, %4}], [%2], %5;" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y), "l"(policy)
+      : "memory");
+}
+__device__ __forceinline__ void tma_load_2d_pair_nohint(void* dst, const CUtensorMap* map,
+                                                        uint32_t bar_cluster, int32_t x,
+                                                        int32_t y) {
+  asm volatile(
+      "cp.async.bulk.tensor.2d.shared::cluster.global.tile.mbarrier::complete_tx::bytes"
+      ".cta_group::2 [%0], [%1, {%3, %4}], [%2];" ::"r"(smem_addr(dst)),
+      "l"(reinterpret_cast<uint64_t>(map)), "r"(bar_cluster), "r"(x), "r"(y)
+      : "memory");
+}
+
 // Contiguous bulk copy global -> shared without a cache hint.
 __device__ __forceinline__ void bulk_load_nohint(void* dst, const void* src, uint32_t bytes,
                                                  uint64_t* bar) {

@@ -25,10 +25,11 @@
  * before touching anything it produces (setting CAI_PDL=0 in the environment
  * before cai_init launches them plainly instead).  With B P > 256 a step is
  * gather, LM head, merge + commit; the LM head is then two kernels, of which
- * only one decodes a step: the swapped-operand kernel below 128 masked rows,
+ * only one decodes a step: the swapped-operand kernel below 32 masked rows,
  * the CTA-pair kernel (tcgen05 cta_group::2, the masked rows as MMA M) from
- * 128 rows on (CAI_PAIR=0 keeps every step on the first, CAI_PAIR_MIN_M=n
- * moves the threshold; both read at cai_init).  The batch runs
+ * 32 rows on, followed by a kernel that merges each row's per-tile partials
+ * (CAI_PAIR=0 keeps every step on the first, CAI_PAIR_MIN_M=n moves the
+ * threshold; both read at cai_init).  The batch runs
  * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
  * per sequence) and contribute no rows afterwards.  A context is not thread
  * safe; use one context per host thread.
@@ -161,8 +162,8 @@ typedef struct cai_stats {
   int32_t grid;             /* CTAs of the LM-head kernel                          */
   int32_t stages;           /* pipeline stages of the LM-head kernel               */
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
-  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 256); 4 with the CTA-pair
-                               LM head, 3 without it                               */
+  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 256); 5 with the CTA-pair
+                               LM head and its row merge, 3 without them           */
 } cai_stats;
 
 /* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")

@@ -152,6 +152,7 @@ struct cai_ctx {
   uint32_t* err = nullptr;
   __nv_bfloat16* hc = nullptr;
   float4* part = nullptr;
+  float4* rowres = nullptr;  // [rows_cap] merged triple per row (pair steps)
   void* hidden_stage = nullptr;
   HostFlag* hf_host = nullptr;
   HostFlag* hf_dev = nullptr;
@@ -160,7 +161,7 @@ struct cai_ctx {
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
   CUtensorMap tm_w{};    // wt as [2 n_vt (H / 64) 128, 64], 16 KiB unswizzled boxes
   bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
-  int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0;
+  int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0, reduce_grid = 0;
   size_t pair_smem = 0;
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
@@ -257,7 +258,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   CommitParams cp{};
   cp.part = c->part;
   cp.n_part = c->G;
-  cp.n_part_pair = c->n_vt;
+  cp.rowres = c->rowres;
   cp.pair_min_M = c->use_pair ? c->pair_min_M : INT_MAX;
   cp.identity_rows = c->fused ? 1 : 0;
   cp.st = c->st;
@@ -388,6 +389,16 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
                    c->tm_a, c->tm_w, pp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
+    ReduceParams rp{};
+    rp.part = c->part;
+    rp.rowres = c->rowres;
+    rp.d_M = c->d_M;
+    rp.n_part = c->n_vt;
+    rp.min_M = c->pair_min_M;
+    if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream, rp) !=
+        cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
   }
   if (c->profiling) cudaEventRecord(e1, stream);
   c->stats.head_launches++;
@@ -469,7 +480,20 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   // at least kMinCtaRows vocabulary rows per CTA), tile group size (tiles sharing one hidden
   // stage; two group buffers of gmax * slot_cols tensor-memory columns fit in
   // 512), ring depths within the opt-in shared memory.
+  // Pair kernel (multi-kernel steps only): steps with at least pair_min_M
+  // masked rows run on CTA pairs (CAI_PAIR=0 disables it, CAI_PAIR_MIN_M sets
+  // the threshold); the swapped-operand kernel then needs N < pair_min_M only,
+  // which keeps its tile groups large.
+  c->use_pair = !c->fused && pair_enabled();
+  if (c->use_pair) {
+    const int mset = env_int("CAI_PAIR_MIN_M");
+    c->pair_min_M = mset > 0 ? mset : 32;
+  }
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
+  if (c->use_pair) {
+    const int cap = round_up(c->pair_min_M > 1 ? c->pair_min_M - 1 : 1, 16);
+    if (c->n_max > cap) c->n_max = cap;
+  }
   c->slot_cols = round_up(c->n_max, 32);
   const int units = (cfg->V + kUnitRows - 1) / kUnitRows;
   // Single-kernel step: one SM is left to the CTA that commits the step, so
@@ -520,14 +544,9 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->n_bslots = bslots_for(stages);
   c->head_smem = head_smem_bytes(stages, c->n_bslots, c->b_slot_bytes, c->slot_cols);
 
-  // Pair kernel (multi-kernel steps only): steps with at least pair_min_M
-  // masked rows are tensor-bound and run on CTA pairs; a persistent grid of
-  // as many 2-CTA clusters as can be resident at once.  CAI_PAIR=0 disables
-  // it, CAI_PAIR_MIN_M sets the threshold.
-  c->use_pair = !c->fused && pair_enabled();
+  // Pair kernel launch shape: a persistent grid of as many 2-CTA clusters as
+  // can be resident at once.
   if (c->use_pair) {
-    const int mset = env_int("CAI_PAIR_MIN_M");
-    c->pair_min_M = mset > 0 ? mset : 128;
     c->n_vt = (cfg->V + kPairTileVocab - 1) / kPairTileVocab;
     cudaFuncAttributes pa{};
     if (cudaFuncGetAttributes(&pa, lm_head_pair_kernel) != cudaSuccess) {
@@ -558,6 +577,9 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
       return CAI_ERR_CUDA;
     }
     c->pair_grid = 2 * clusters;
+    const int warps_per_cta = kReduceThreads / 32;
+    const int want = (c->rows_cap + warps_per_cta - 1) / warps_per_cta;
+    c->reduce_grid = want < 4 * sms ? want : 4 * sms;
   }
 
   const size_t BL = static_cast<size_t>(cfg->B) * c->L;
@@ -591,8 +613,10 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
   CAI_ALLOC(c->part, float4,
             static_cast<size_t>(c->rows_cap) * (c->use_pair && c->n_vt > c->G ? c->n_vt : c->G))
-  if (c->use_pair)
+  if (c->use_pair) {
     CAI_ALLOC(c->wt, uint8_t, static_cast<size_t>(2 * c->n_vt) * kPairHalf * 2 * cfg->H)
+    CAI_ALLOC(c->rowres, float4, c->rows_cap)
+  }
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
   CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   const void* w_src = W;
@@ -672,7 +696,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->stats.grid = c->G;
   c->stats.stages = c->n_stages;
   c->stats.n_max = c->n_max;
-  c->stats.kernels_per_step = c->fused ? 1 : c->use_pair ? 4 : 3;
+  c->stats.kernels_per_step = c->fused ? 1 : c->use_pair ? 5 : 3;
   r = cai_reset(c, stream);
   if (r != CAI_OK) {
     release(c);

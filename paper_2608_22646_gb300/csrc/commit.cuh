@@ -59,7 +59,7 @@ struct StateArrays {
 struct CommitParams {
   const float4* part;     // [rows, n_part] softmax partials of this step
   int n_part;             // partial slots per row (one per LM-head CTA)
-  int n_part_pair;        // partial slots per row when the pair kernel decoded the step
+  const float4* rowres;   // [rows] merged triple per row when the pair kernel decoded the step
   int pair_min_M;         // steps with at least this many rows ran the pair kernel
   int identity_rows;      // 1: row of (b, p) is b P + p; 0: row_of[b P + p]
   StateArrays st;
@@ -107,8 +107,8 @@ struct CommitSmem {
   uint8_t bud[kMaxP];  // budget before this step
 };
 
-__device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs, int n_part,
-                                     int* left_after = nullptr) {
+__device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs,
+                                     const float4* part, int n_part, int* left_after = nullptr) {
   __shared__ int s_eta, s_left, s_reason, s_unres, s_ell, s_running;
   int* s_tok = cs.tok;
   int* s_cand = cs.cand;
@@ -152,7 +152,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
       }
 #pragma unroll
       for (int j = 0; j < kPosPerWarp; ++j) {
-        const float4* pr = p.part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * n_part;
+        const float4* pr = part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * n_part;
 #pragma unroll
         for (int u = 0; u < kPartPerLane; ++u) {
           const int k = lane + 32 * u;
@@ -171,7 +171,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
         for (int u = 0; u < kPartPerLane; ++u)
           merge_tri(m, s, ix, q[j][u].x, q[j][u].y, __float_as_int(q[j][u].z));
         for (int k = lane + 32 * kPartPerLane; k < n_part; k += 32) {
-          const float4 r = __ldcg(p.part + static_cast<size_t>(row[j]) * n_part + k);
+          const float4 r = __ldcg(part + static_cast<size_t>(row[j]) * n_part + k);
           merge_tri(m, s, ix, r.x, r.y, __float_as_int(r.z));
         }
 #pragma unroll

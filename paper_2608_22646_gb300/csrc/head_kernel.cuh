@@ -648,8 +648,8 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     for (int b = 0; b < p.cp.B; ++b) {
       int left = 0;
       // Every copy and MMA has completed: the W ring is free shared memory.
-      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), p.cp.n_part,
-                                       &left);
+      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), p.cp.part,
+                                       p.cp.n_part, &left);
       remaining += left;
     }
     if (threadIdx.x == 0) *p.cp.m_hist_slot = decoded;

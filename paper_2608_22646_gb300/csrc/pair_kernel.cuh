@@ -330,4 +330,53 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   }
 }
 
+// Second stage of a pair step: one warp per masked row merges the row's
+// n_vt tile partials (merge_tri: max, rescaled sum, lowest index among equal
+// maxima) into one triple, rowres[row], so that the commit reads one value per
+// row.  Returns at once when the step ran on the swapped-operand kernel.
+struct ReduceParams {
+  const float4* part;  // [rows, n_part]
+  float4* rowres;      // [rows]
+  const int* d_M;
+  int n_part;
+  int min_M;
+};
+
+constexpr int kReduceThreads = 256;
+
+__global__ void __launch_bounds__(kReduceThreads) reduce_partials_kernel(const ReduceParams p) {
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // the pair kernel's partials
+  const int M = *p.d_M;
+  if (M < p.min_M) return;
+  const int lane = threadIdx.x & 31;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < M; row += nw) {
+    const float4* pr = p.part + static_cast<size_t>(row) * p.n_part;
+    float m = kNegBig, s = 0.0f;
+    int ix = INT_MAX;
+    int k = lane;
+    for (; k + 96 < p.n_part; k += 128) {  // four loads in flight per lane
+      const float4 a = __ldcg(pr + k), b = __ldcg(pr + k + 32), c = __ldcg(pr + k + 64),
+                   d = __ldcg(pr + k + 96);
+      merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+      merge_tri(m, s, ix, b.x, b.y, __float_as_int(b.z));
+      merge_tri(m, s, ix, c.x, c.y, __float_as_int(c.z));
+      merge_tri(m, s, ix, d.x, d.y, __float_as_int(d.z));
+    }
+    for (; k < p.n_part; k += 32) {
+      const float4 a = __ldcg(pr + k);
+      merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+      const float so = __shfl_xor_sync(0xffffffffu, s, off);
+      const int io = __shfl_xor_sync(0xffffffffu, ix, off);
+      merge_tri(m, s, ix, mo, so, io);
+    }
+    if (lane == 0) p.rowres[row] = make_float4(m, s, __int_as_float(ix), 0.0f);
+  }
+}
+
 }  // namespace cai

@@ -84,9 +84,12 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // partials of this step, state of the previous one
   // This step's M (d_M is rewritten only by the last CTA, after every CTA's
-  // merge) tells which LM-head kernel wrote the partials.
-  const int n_part = *p.d_M >= p.pair_min_M ? p.n_part_pair : p.n_part;
-  merge_commit_sequence(p, blockIdx.x, cs, n_part);
+  // merge) tells which LM-head kernel decoded it: the pair kernel's tile
+  // partials were already merged into one triple per row.
+  if (*p.d_M >= p.pair_min_M)
+    merge_commit_sequence(p, blockIdx.x, cs, p.rowres, 1);
+  else
+    merge_commit_sequence(p, blockIdx.x, cs, p.part, p.n_part);
   if (gridDim.x > 1) {
     if (threadIdx.x == 0) {
       __threadfence();

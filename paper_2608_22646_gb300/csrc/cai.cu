@@ -340,6 +340,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.fused = c->fused ? 1 : 0;
   hp.M_fixed = c->BP;
   hp.max_M = c->use_pair ? c->pair_min_M - 1 : INT_MAX;
+  hp.prefetch = c->use_pair ? 0 : 1;
   hp.first = first ? 1 : 0;
   hp.part = c->part;
   hp.err = c->err;

@@ -72,6 +72,7 @@ struct HeadParams {
   int fused;           // 1: single-kernel step (see below), 0: gather / head / merge kernels
   int M_fixed;         // rows decoded by the single-kernel step (all B P positions)
   int max_M;           // multi-kernel step: larger steps are left to lm_head_pair_kernel
+  int prefetch;        // stream the first W stages before the dependency wait
   int first;           // the step is a block's step zero (every position masked)
   float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
   uint32_t* err;       // error word
@@ -317,7 +318,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   // the commit state) is touched only after grid_dependency_wait().  A
   // single-kernel step reads nothing the previous step writes before its
   // partials, so only its epilogue and its commit wait.
-  const int n_pre = min(p.n_stages, pl.n_tiles * KB);
+  // When most steps go to the pair kernel, copies started before M is known
+  // would mostly be wasted, so the launch asks for none.
+  const int n_pre = p.prefetch ? min(p.n_stages, pl.n_tiles * KB) : 0;
   const bool spec = p.fused && !p.first;  // may find out that nothing is masked
 
   if (warp == 0) {

@@ -121,17 +121,24 @@ class Clocks:
                 "samples": len(sm)}
 
 
-def _traffic_record(kernel_src: str):
-    """DRAM bytes per launch of the LM-head kernel from the committed ncu
-    summary, if it was taken on the current kernel source."""
+def _traffic_record(workload: str):
+    """DRAM bytes per launch of the workload's dominant LM-head kernel from the
+    committed ncu summaries, if they were taken on the current kernel source."""
     p = os.path.join(PROFILES, "lm_head_traffic.json")
     if not os.path.exists(p):
         return None
     with open(p) as f:
-        rec = json.load(f)
-    with open(kernel_src, "rb") as f:
-        h = hashlib.sha256(f.read()).hexdigest()[:16]
-    return rec if rec.get("kernel_sha") == h else None
+        recs = json.load(f).get("records", [])
+    for rec in recs:
+        if rec.get("workload") != workload:
+            continue
+        src = os.path.join(ROOT, "paper_2608_22646_gb300", "csrc", rec["source"])
+        if not os.path.exists(src):
+            return None
+        with open(src, "rb") as f:
+            h = hashlib.sha256(f.read()).hexdigest()[:16]
+        return rec if rec.get("source_sha") == h else None
+    return None
 
 
 def run_trajectory(cai, ctx, hidden, wl, lag_poll=True, stream=None):
@@ -304,28 +311,36 @@ def main():
     t_tc = sum(f / (tf * 1e12) for f in flops_t)
     t_roof = sum(max(b / (hbm * 1e9), f / (tf * 1e12)) for b, f in zip(bytes_t, flops_t))
     head_s = max(head_ms, 1e-9) / 1e3 / args.steps       # LM-head time per generation
-    tr = _traffic_record(os.path.join(ROOT, "paper_2608_22646_gb300", "csrc", "head_kernel.cuh"))
+    tr = _traffic_record(wl.name)
     per_launch = max(1, head_launches // max(1, args.steps))
-    common = {"kernel": "lm_head_softmax_kernel", "head_launches": head_launches,
+    kps = int(stats1["kernels_per_step"])
+    kernel = ("lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
+              if kps == 1 else
+              "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows), "
+              "with reduce_partials_kernel" if kps == 5 else "lm_head_softmax_kernel")
+    common = {"kernel": kernel, "head_launches": head_launches,
               "head_ms_total": round(head_ms, 3),
               "roofline_time_frac": round(t_roof / head_s, 4),
-              "timing": "CUDA events around every LM-head launch, second pass of the same "
-                        "K generations"}
+              "timing": "CUDA events around every step's LM-head launch(es) (multi-kernel "
+                        "steps: both LM-head kernels and the row merge, not gather or commit), "
+                        "second pass of the same K generations"}
+    traffic = tr["dram_bytes_per_launch"] if tr else None
+    traffic_basis = ("ncu dram read+write of one launch with M = %d (%s); algorithmic bytes of "
+                     "that launch %d" % (tr["captured_M"], tr["summary"],
+                                         tr["algorithmic_bytes_of_profiled_launch"])
+                     if tr else None)
     if t_hbm >= t_tc:
         achieved = sum(bytes_t) / head_s / 1e9
         roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
                 "frac": round(achieved / hbm, 4),
-                "traffic": (tr["dram_bytes_per_launch"] if tr and tr.get("workload") == wl.name
-                            else None),
-                "traffic_basis": ("ncu dram read+write of one full-mask launch; algorithmic bytes "
-                                  "of that launch %d" % tr["algorithmic_bytes_of_profiled_launch"])
-                                 if tr and tr.get("workload") == wl.name else None,
+                "traffic": traffic, "traffic_basis": traffic_basis,
                 "algorithmic_bytes_per_launch": round(sum(bytes_t) / per_launch),
                 "peak_source": f"{peak_kind} hbm_gbs", **common}
     else:
         achieved = sum(flops_t) / head_s / 1e12
         roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": tf,
-                "unit": "TFLOP/s", "frac": round(achieved / tf, 4), "traffic": None,
+                "unit": "TFLOP/s", "frac": round(achieved / tf, 4),
+                "traffic": traffic, "traffic_basis": traffic_basis,
                 "algorithmic_flops_per_launch": round(sum(flops_t) / per_launch),
                 "peak_source": f"{peak_kind} bf16 sustained", **common}
 

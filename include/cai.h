@@ -66,6 +66,8 @@ extern "C" {
 #define CAI_FLUSH_ON_EXIT 4u    /* commit still-masked tokens to their argmax when a block exits */
 #define CAI_QUARTER_POS 8u      /* position/budget tiers at P/4, P/2, 3P/4 instead of 16/32/48 */
 #define CAI_QUARTER_BLOCKS 16u  /* theta_e^(b) indexed by the quarter of the output block b is in */
+#define CAI_NO_BLOCK_SCHEDULE 32u /* Box 3 alone: every block ends at theta_e1 (ablation "APD") */
+#define CAI_FIXED_THRESHOLD 64u /* fixed-threshold rule (Fast-dLLM): theta^(b)(t) = theta_s      */
 
 #define CAI_PRESET_LLADA 0      /* gating ON  (Section 5: LLaDA-8B-Instruct) */
 #define CAI_PRESET_DREAM 1      /* gating OFF (Section 5: Dream-7B-Instruct) */

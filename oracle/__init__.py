@@ -30,6 +30,8 @@ POS_FACTOR = 2
 FLUSH_ON_EXIT = 4
 QUARTER_POS = 8
 QUARTER_BLOCKS = 16
+NO_BLOCK_SCHEDULE = 32   # Box 3 alone: theta_e1 in every block ("APD" ablation row)
+FIXED_THRESHOLD = 64     # fixed-threshold rule (Fast-dLLM): theta = theta_s always
 
 MASK = -1
 RUNNING, EXIT_DONE, EXIT_GRIND, EXIT_TMAX = 0, 1, 2, 3

@@ -47,6 +47,12 @@
  *     that reaches t = T - 1 without either exit is "T exhausted".
  *   - the batch runs blocks and steps in lockstep; each sequence keeps its
  *     own low-yield counter and exit state.
+ *
+ * Ablation variants (Section 5.3, Table "HumanEval ablation"):
+ *   - CAI_O_NO_BLOCK_SCHEDULE: Box 3 alone ("APD"): every block ends at
+ *     theta_e1 = 0.70 instead of Box 4's theta_e^(b).
+ *   - CAI_O_FIXED_THRESHOLD: the fixed-threshold rule of Fast-dLLM that the
+ *     paper compares with: theta^(b)(t) = theta_s for every step and block.
  */
 #include <math.h>
 #include <pthread.h>
@@ -59,6 +65,8 @@
 #define CAI_O_FLUSH_ON_EXIT 4u
 #define CAI_O_QUARTER_POS 8u
 #define CAI_O_QUARTER_BLOCKS 16u
+#define CAI_O_NO_BLOCK_SCHEDULE 32u
+#define CAI_O_FIXED_THRESHOLD 64u
 
 #define CAI_O_MASK (-1)
 
@@ -208,6 +216,7 @@ int32_t cai_o_softmax_row(const uint16_t* W, int32_t V, int32_t H, const uint16_
 double cai_o_theta_e(const cai_o_cfg* c, int32_t b) {
   int32_t be = b;
   if (c->flags & CAI_O_QUARTER_BLOCKS) be = 1 + (4 * (b - 1)) / c->n_blocks;
+  if (c->flags & CAI_O_NO_BLOCK_SCHEDULE) be = 1;
   double th = c->theta_e1 - c->theta_e_step * (double)(be - 1);
   if (th < c->theta_e_min) th = c->theta_e_min;
   return th;
@@ -216,6 +225,7 @@ double cai_o_theta_e(const cai_o_cfg* c, int32_t b) {
 /* Boxes 3 and 4: theta^(b)(t) = theta_s while t < wT, else
  * theta_e^(b) + (theta_s - theta_e^(b))/2 (1 + cos(pi (t - wT) / (T - wT))). */
 double cai_o_theta_block(const cai_o_cfg* c, int32_t b, int32_t t) {
+  if (c->flags & CAI_O_FIXED_THRESHOLD) return c->theta_s;
   if (100 * t < c->warmup_pct * c->T) return c->theta_s;
   const double pi = 3.14159265358979323846;
   double wT = (double)c->warmup_pct * (double)c->T / 100.0;

@@ -35,6 +35,8 @@ CAI_POS_FACTOR = 2
 CAI_FLUSH_ON_EXIT = 4
 CAI_QUARTER_POS = 8
 CAI_QUARTER_BLOCKS = 16
+CAI_NO_BLOCK_SCHEDULE = 32
+CAI_FIXED_THRESHOLD = 64
 
 CAI_PRESET_LLADA = 0
 CAI_PRESET_DREAM = 1

@@ -205,7 +205,7 @@ int validate(const cai_config* c) {
       c->n_blocks > 32767 || static_cast<int64_t>(c->n_blocks) * c->P > (1 << 24))
     return CAI_ERR_SHAPE;
   if (c->warmup_pct < 0 || c->warmup_pct > 100 || c->K < 1 || (c->eta_mode != 0 && c->eta_mode != 1) ||
-      !(c->clip_lo <= c->clip_hi) || (c->flags & ~31u) != 0)
+      !(c->clip_lo <= c->clip_hi) || (c->flags & ~127u) != 0)
     return CAI_ERR_ARG;
   return CAI_OK;
 }
@@ -230,11 +230,13 @@ void release(cai_ctx* c) {
 double theta_e_of(const cai_config& c, int b1) {
   int be = b1;
   if (c.flags & CAI_QUARTER_BLOCKS) be = 1 + (4 * (b1 - 1)) / c.n_blocks;
+  if (c.flags & CAI_NO_BLOCK_SCHEDULE) be = 1;
   double th = c.theta_e1 - c.theta_e_step * static_cast<double>(be - 1);
   return th < c.theta_e_min ? c.theta_e_min : th;
 }
 
 double theta_block_of(const cai_config& c, int b1, int t) {
+  if (c.flags & CAI_FIXED_THRESHOLD) return c.theta_s;
   if (100 * t < c.warmup_pct * c.T) return c.theta_s;
   const double wT = static_cast<double>(c.warmup_pct) * c.T / 100.0;
   const double u = (t - wT) / (c.T - wT);

@@ -213,6 +213,53 @@ def test_theta_block_shape(T, b):
     assert th[T - 1] - te <= alpha * (math.pi * (1 - uL)) ** 2 / 2 + 1e-12
 
 
+def test_ablation_variants_thresholds():
+    # Box 3 alone ("APD" row of the ablation table): every block follows the
+    # block-1 schedule of the golden table (theta_e = 0.70), not Box 4's.
+    apd = oracle.Config(T=32, n_blocks=8, flags=oracle.NO_BLOCK_SCHEDULE)
+    for T, b, t, th in _rows("theta_schedule.txt"):
+        if int(b) != 1:
+            continue
+        cfg = oracle.Config(T=int(T), n_blocks=8, flags=oracle.NO_BLOCK_SCHEDULE)
+        for blk in (1, 2, 4, 8):
+            assert abs(oracle.theta_block(cfg, blk, int(t)) - float(th)) < 6e-7, (T, blk, t)
+    assert all(oracle.theta_e(apd, b) == pytest.approx(0.70, abs=1e-15) for b in range(1, 9))
+    # the fixed-threshold rule the paper compares with (Fast-dLLM): theta_s at
+    # every step of every block, position factors still applied when enabled
+    for ts in (0.9, 0.7):
+        fx = oracle.Config(T=32, P=64, n_blocks=8, theta_s=ts, flags=oracle.FIXED_THRESHOLD)
+        assert {oracle.theta_block(fx, b, t) for b in range(1, 9) for t in range(32)} == {ts}
+        assert oracle.theta_token(fx, 5, 31, 63) == ts
+        fxp = oracle.Config(T=32, P=64, n_blocks=8, theta_s=ts,
+                            flags=oracle.FIXED_THRESHOLD | oracle.POS_FACTOR)
+        assert oracle.theta_token(fxp, 3, 20, 0) == pytest.approx(ts * 0.8, abs=1e-15)
+        assert oracle.theta_token(fxp, 3, 20, 60) == pytest.approx(min(ts * 1.1, 0.98), abs=1e-15)
+
+
+def test_fixed_threshold_trajectory_commits_exactly_above_threshold():
+    # With the fixed rule, gating off and no position factor, a token commits
+    # at step t iff its confidence is >= theta_s: check every step of a toy
+    # trajectory against the step's own confidences.
+    wl = synth.WORKLOADS["toy"]
+    cfg = oracle.Config(B=1, P=wl.P, T=wl.T, n_blocks=wl.n_blocks, theta_s=0.7,
+                        flags=oracle.FIXED_THRESHOLD)
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device="cpu")
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    Wb = oracle.bf16_bits(W)
+    st = oracle.State(cfg)
+    for blk in range(wl.n_blocks):
+        for t in range(wl.T):
+            before = st.tok.copy()
+            out = oracle.step(st, Wb, oracle.bf16_bits(hs(blk, t)), blk, t, 2)
+            sl = slice(blk * wl.P, (blk + 1) * wl.P)
+            was = before[0, sl] == oracle.MASK
+            now = st.tok[0, sl] != oracle.MASK
+            conf = st.conf[0, sl]
+            assert np.array_equal(now & was, was & (conf >= 0.7)), (blk, t)
+            if st.exit_reason[0, blk] != oracle.RUNNING:
+                break
+
+
 def test_position_factor_printed():
     cfg = oracle.Config(P=64)
     for p, r in _rows("position_factors.txt"):

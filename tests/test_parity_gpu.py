@@ -95,6 +95,10 @@ def test_ragged_shapes_trajectory(shape, grid):
     (cai.CAI_PRESET_DREAM, None),  # gating OFF: budgets and grinding exit disabled
     (cai.CAI_PRESET_LLADA, cai.CAI_GATING | cai.CAI_POS_FACTOR | cai.CAI_FLUSH_ON_EXIT),
     (cai.CAI_PRESET_LLADA, cai.CAI_GATING | cai.CAI_QUARTER_BLOCKS),
+    # ablation rows of the paper's component table: "+APD" (Box 3 alone) and
+    # "+APD+Block" (Boxes 3-4), both without budgets or position factors
+    (cai.CAI_PRESET_LLADA, cai.CAI_NO_BLOCK_SCHEDULE),
+    (cai.CAI_PRESET_LLADA, 0),
 ])
 def test_controller_variants(preset, flags):
     wl = _wl("toy", B=4, a0="bimodal", gen_len=128)
@@ -104,6 +108,23 @@ def test_controller_variants(preset, flags):
         parity.run_checked_trajectory(ctx, W, hs)
     finally:
         cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("theta", [0.9, 0.7])
+def test_fixed_threshold_rule(theta):
+    # The fixed-threshold rule the paper compares with (Fast-dLLM), on a batch
+    # of four and on a multi-kernel context (B P = 320).
+    for B, P, gen in ((4, 16, 64), (5, 64, 128)):
+        wl = _wl("toy", B=B, P=P, a0="bimodal", gen_len=gen)
+        W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+        cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+        cfg.flags = cai.CAI_FIXED_THRESHOLD
+        cfg.theta_s = theta
+        ctx = cai.cai_init(cfg, W)
+        try:
+            parity.run_checked_trajectory(ctx, W, synth.HiddenStates(wl, W, "calibrated", seed=5))
+        finally:
+            cai.cai_free(ctx)
 
 
 def test_fraction_eta_mode():

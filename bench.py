@@ -41,6 +41,7 @@ if ROOT not in sys.path:
 
 METRIC = "masked positions decoded/s (fused head+commit) at 1 GB300; % of HBM/tensor roofline"
 UNIT = "positions/s"
+FINAL_NORM_EPS = 1e-5
 PROFILES = os.path.join(ROOT, "profiles")
 
 
@@ -153,9 +154,10 @@ def run_trajectory(cai, ctx, hidden, wl, lag_poll=True, stream=None):
             cai.cai_denoise_step(ctx, hidden[blk][t], stream)
 
 
-def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0):
+def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0, norm=None):
     """The oracle as it stands on the host cores: full steps of the same
-    trajectory (all masked rows of each step), for about budget_s seconds."""
+    trajectory (all masked rows of each step), for about budget_s seconds.
+    ``norm`` = (weight, eps) when the final RMSNorm is part of the head."""
     import oracle
     cfg = oracle.Config(B=wl.B, P=wl.P, T=wl.T, n_blocks=wl.n_blocks)
     st = oracle.State(cfg)
@@ -167,7 +169,7 @@ def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0):
     for blk in range(wl.n_blocks):
         for t in range(wl.T):
             h = oracle.bf16_bits(hs_fn(blk, t))
-            out = oracle.step(st, Wb, h, blk, t, threads)
+            out = oracle.step(st, Wb, h, blk, t, threads, *(norm or ()))
             rows += out["M"]
             steps += 1
             if np.all(st.exit_reason[:, blk] != 0) or time.perf_counter() - t0 > budget_s:
@@ -205,6 +207,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-profile", action="store_true",
                     help="time the region without per-kernel events (no roofline figure)")
+    ap.add_argument("--final-norm", action="store_true",
+                    help="the model's final RMSNorm inside the head (cai_init_rmsnorm): inputs "
+                         "are the rows before that norm")
     args = ap.parse_args()
 
     import torch
@@ -241,11 +246,15 @@ def main():
 
     W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device=dev)
     hs = synth.HiddenStates(wl, W, args.generator, seed=wl.seed_h + 1000 * rank)
+    norm = None
+    if args.final_norm:
+        norm = (synth.final_norm_weight(wl.H, device=dev), FINAL_NORM_EPS)
+        hs = synth.PreNormHidden(hs)
     hidden = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
     torch.cuda.synchronize()
 
     cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
-    ctx = cai.cai_init(cfg, W)
+    ctx = cai.cai_init_rmsnorm(cfg, W, *norm) if norm else cai.cai_init(cfg, W)
 
     for _ in range(args.warmup):
         cai.cai_reset(ctx)
@@ -350,6 +359,7 @@ def main():
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded LLaDA/Dream-shaped weight and hidden states; no model weights)",
         "config": {**_workload_desc(wl, args.generator), "parallelism": f"replicas x{world}",
+                   "final_norm_in_head": bool(args.final_norm),
                    "positions_per_step": positions,
                    "denoising_steps_per_generation": nonzero_launch,
                    "step_calls_per_generation": int(steps_issued)},
@@ -361,7 +371,7 @@ def main():
     if not args.no_e2e:
         line["e2e"] = e2e_run(cai, ctx, hs, wl, args, dist, dev)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, W, lambda b, t: hidden[b][t])
+        line["cpu_baseline"] = cpu_baseline(wl, W, lambda b, t: hidden[b][t], norm=norm)
     cai.cai_free(ctx)
     if rank == 0:
         print(json.dumps(line), flush=True)
@@ -411,6 +421,10 @@ def run_reference(args, wl):
     oracle.build()
     W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device="cpu")
     hs = synth.HiddenStates(wl, W, args.generator)
+    norm = ()
+    if args.final_norm:
+        norm = (synth.final_norm_weight(wl.H), FINAL_NORM_EPS)
+        hs = synth.PreNormHidden(hs)
     cfg = oracle.Config(B=wl.B, P=wl.P, T=wl.T, n_blocks=wl.n_blocks)
     st = oracle.State(cfg)
     Wb = oracle.bf16_bits(W)
@@ -434,7 +448,7 @@ def run_reference(args, wl):
                 continue
             h = oracle.bf16_bits(hs(b, t))
             t0 = time.perf_counter()
-            out = oracle.step(st, Wb, h, b, t, threads)
+            out = oracle.step(st, Wb, h, b, t, threads, *norm)
             return out["M"], time.perf_counter() - t0
 
     for _ in range(args.warmup):
@@ -449,7 +463,8 @@ def run_reference(args, wl):
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
             "ms_per_step": round(dt / k * 1e3, 3), "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
-            "config": _workload_desc(wl, args.generator),
+            "config": {**_workload_desc(wl, args.generator),
+                       "final_norm_in_head": bool(args.final_norm)},
             "cpu_baseline": {"value": round(v, 3), "unit": UNIT, "cores": threads,
                              "kind": "oracle",
                              "sample": f"{k} denoising steps of the trajectory, {rows} masked rows"},

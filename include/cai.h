@@ -186,6 +186,25 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
 int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out);
 
 /*
+ * cai_init with the model's final RMSNorm inside the decoding head.  The paper
+ * has no counterpart: Box 1's p_theta is computed from the normalised last
+ * hidden state, and this entry point lets the caller pass the last layer's
+ * output before that norm, saving the pass over the hidden states that a
+ * separate norm kernel would make.  Each decoded row h then becomes
+ *   x = g * h / sqrt(mean_k h_k^2 + eps)
+ * before z = W x.  norm_weight g is [H] bf16 (host or device; read during this
+ * call only); eps >= 0.  The weight is folded into the library's packed copies
+ * of W (W[v,k] g[k], rounded to bf16 once); 1 / sqrt(mean h^2 + eps) is
+ * computed per row in fp32 from the bf16 row and scales the row's logits in
+ * fp32 before the softmax.  Single-kernel steps add one small kernel per step
+ * for the row scales; multi-kernel steps compute them in the gather.
+ * Errors: as cai_init, and CAI_ERR_ARG for a NULL or misaligned norm_weight or
+ * a negative or non-finite eps.
+ */
+int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weight, double eps,
+                     void* stream, cai_ctx** out);
+
+/*
  * Local step t = 0 of the current block (Algorithm 1, step-zero init): every
  * position of every sequence is masked, so M = B P rows are decoded.  Stores
  * s_i and B_i, then applies the commit rule with theta^(b)(0).

@@ -81,6 +81,9 @@ def lib():
         _lib.cai_o_head_rows.restype = i32
         _lib.cai_o_head_rows.argtypes = [u16p, i32, i32, u16p, i32, i32,
                                          u16p, u16p, u16p, u16p, u16p]
+        _lib.cai_o_head_rows_norm.restype = i32
+        _lib.cai_o_head_rows_norm.argtypes = [u16p, i32, i32, u16p, i32, u16p, d, i32,
+                                              u16p, u16p, u16p, u16p, u16p]
         _lib.cai_o_softmax_row.restype = i32
         _lib.cai_o_softmax_row.argtypes = [u16p, i32, i32, u16p, u16p, u16p]
         for name in ("cai_o_theta_e",):
@@ -145,8 +148,10 @@ def bf16_bits(x) -> np.ndarray:
     return np.ascontiguousarray(x.detach().cpu().contiguous().view(torch.int16).numpy().view(np.uint16))
 
 
-def head_rows(W, rows, n_threads: int | None = None) -> dict:
+def head_rows(W, rows, n_threads: int | None = None, norm_weight=None, eps: float = 0.0) -> dict:
     """Box 1 for every row of ``rows`` [M, H] against ``W`` [V, H] (bf16).
+    With ``norm_weight`` g [H] (bf16), each row h is first put through the
+    model's final RMSNorm, g * h / sqrt(mean(h^2) + eps), in fp64.
 
     Returns conf (c = max_v p), idx (argmax, lowest index on ties), zmax,
     lse (log-sum-exp) and gap (top-1 minus top-2 logit), all fp64/int32."""
@@ -158,9 +163,14 @@ def head_rows(W, rows, n_threads: int | None = None) -> dict:
     out["idx"] = np.zeros(M, np.int32)
     if n_threads is None:
         n_threads = os.cpu_count() or 1
-    rc = lib().cai_o_head_rows(_ptr(Wb), V, H, _ptr(Rb), M, n_threads, _ptr(out["conf"]),
-                               _ptr(out["idx"]), _ptr(out["zmax"]), _ptr(out["lse"]),
-                               _ptr(out["gap"]))
+    gb = None
+    if norm_weight is not None:
+        gb = bf16_bits(norm_weight).reshape(-1)
+        assert gb.shape[0] == H
+    rc = lib().cai_o_head_rows_norm(_ptr(Wb), V, H, _ptr(Rb), M,
+                                    None if gb is None else _ptr(gb), float(eps), n_threads,
+                                    _ptr(out["conf"]), _ptr(out["idx"]), _ptr(out["zmax"]),
+                                    _ptr(out["lse"]), _ptr(out["gap"]))
     if rc != 0:
         raise RuntimeError(f"oracle head failed: {rc}")
     return out
@@ -271,10 +281,12 @@ def controller_step(st: State, blk: int, t: int, conf_bp: np.ndarray, idx_bp: np
     lib().cai_o_controller_step(ctypes.byref(c), ctypes.byref(cs), blk, t, _ptr(conf_bp), _ptr(idx_bp))
 
 
-def step(st: State, W, hidden_bph, blk: int, t: int, n_threads: int | None = None) -> dict:
-    """One denoising step: the head on every masked row of a running sequence
-    (rows taken in (b, p) order), then the controller.  Returns the head
-    outputs scattered to [B, P] (NaN / -1 where not computed) and M_t."""
+def step(st: State, W, hidden_bph, blk: int, t: int, n_threads: int | None = None,
+         norm_weight=None, eps: float = 0.0) -> dict:
+    """One denoising step: the head (after the final RMSNorm when
+    ``norm_weight`` is given) on every masked row of a running sequence (rows
+    taken in (b, p) order), then the controller.  Returns the head outputs
+    scattered to [B, P] (NaN / -1 where not computed) and M_t."""
     cfg = st.cfg
     hb = bf16_bits(hidden_bph).reshape(cfg.B, cfg.P, -1)
     mk = st.masked(blk)
@@ -284,7 +296,7 @@ def step(st: State, W, hidden_bph, blk: int, t: int, n_threads: int | None = Non
     idx = np.full((cfg.B, cfg.P), -1, np.int32)
     gap = np.full((cfg.B, cfg.P), np.nan)
     if M:
-        h = head_rows(W, np.ascontiguousarray(rows), n_threads)
+        h = head_rows(W, np.ascontiguousarray(rows), n_threads, norm_weight, eps)
         conf[mk], idx[mk], gap[mk] = h["conf"], h["idx"], h["gap"]
     controller_step(st, blk, t, np.nan_to_num(conf), idx)
     return {"conf": conf, "idx": idx, "gap": gap, "M": M, "masked": mk}

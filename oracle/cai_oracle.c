@@ -101,16 +101,25 @@ double cai_o_bf16_to_double(uint16_t bits) {
 /* ------------------------------------------------------ decoding head -- */
 
 /* Box 1 for one row h of length H against every row of W [V, H]:
- *   z_v = sum_k W[v,k] h[k]
+ *   z_v = sum_k W[v,k] x[k], with x = h, or, when the model's final RMSNorm is
+ *   part of the head (g != NULL), x[k] = g[k] h[k] / r, r = sqrt(sum_k h[k]^2 / H + eps)
  *   m   = max_v z_v, idx = lowest v with z_v = m
  *   S   = sum_v exp(z_v - m),  c = max_v p_v = exp(m - LSE) = 1 / S
  * gap = m - (largest z_v over v != idx), +inf when V = 1. */
-static void head_one_row(const uint16_t* W, int32_t V, int32_t H, const uint16_t* h, double* z,
-                         double* conf, int32_t* argmax, double* zmax, double* lse, double* gap) {
+static void head_one_row(const uint16_t* W, int32_t V, int32_t H, const uint16_t* h,
+                         const uint16_t* g, double eps, double* x, double* z, double* conf,
+                         int32_t* argmax, double* zmax, double* lse, double* gap) {
+  for (int32_t k = 0; k < H; ++k) x[k] = cai_o_bf16_to_double(h[k]);
+  if (g) {
+    double ss = 0.0;
+    for (int32_t k = 0; k < H; ++k) ss += x[k] * x[k];
+    const double r = sqrt(ss / (double)H + eps);
+    for (int32_t k = 0; k < H; ++k) x[k] = cai_o_bf16_to_double(g[k]) * x[k] / r;
+  }
   for (int32_t v = 0; v < V; ++v) {
     const uint16_t* w = W + (size_t)v * (size_t)H;
     double acc = 0.0;
-    for (int32_t k = 0; k < H; ++k) acc += cai_o_bf16_to_double(w[k]) * cai_o_bf16_to_double(h[k]);
+    for (int32_t k = 0; k < H; ++k) acc += cai_o_bf16_to_double(w[k]) * x[k];
     z[v] = acc;
   }
   double m = z[0];
@@ -138,6 +147,8 @@ typedef struct {
   const uint16_t* W;
   int32_t V, H;
   const uint16_t* rows;
+  const uint16_t* g;
+  double eps;
   int32_t M, first, stride;
   double *conf, *zmax, *lse, *gap;
   int32_t* argmax;
@@ -147,23 +158,29 @@ typedef struct {
 static void* head_worker(void* arg) {
   head_job* j = (head_job*)arg;
   double* z = (double*)malloc(sizeof(double) * (size_t)j->V);
-  if (!z) {
+  double* x = (double*)malloc(sizeof(double) * (size_t)j->H);
+  if (!z || !x) {
+    free(z);
+    free(x);
     j->failed = 1;
     return NULL;
   }
   for (int32_t i = j->first; i < j->M; i += j->stride) {
-    head_one_row(j->W, j->V, j->H, j->rows + (size_t)i * (size_t)j->H, z, &j->conf[i], &j->argmax[i],
-                 &j->zmax[i], &j->lse[i], &j->gap[i]);
+    head_one_row(j->W, j->V, j->H, j->rows + (size_t)i * (size_t)j->H, j->g, j->eps, x, z,
+                 &j->conf[i], &j->argmax[i], &j->zmax[i], &j->lse[i], &j->gap[i]);
   }
   free(z);
+  free(x);
   return NULL;
 }
 
-/* Decoding head over M rows [M, H].  Rows are spread over n_threads threads;
- * each row is computed start to end by one thread.  Returns 0 on success. */
-int32_t cai_o_head_rows(const uint16_t* W, int32_t V, int32_t H, const uint16_t* rows, int32_t M,
-                        int32_t n_threads, double* conf, int32_t* argmax, double* zmax, double* lse,
-                        double* gap) {
+/* Decoding head over M rows [M, H], with the model's final RMSNorm (weight g
+ * [H], epsilon eps) applied to each row first when g is not NULL.  Rows are
+ * spread over n_threads threads; each row is computed start to end by one
+ * thread.  Returns 0 on success. */
+int32_t cai_o_head_rows_norm(const uint16_t* W, int32_t V, int32_t H, const uint16_t* rows,
+                             int32_t M, const uint16_t* g, double eps, int32_t n_threads,
+                             double* conf, int32_t* argmax, double* zmax, double* lse, double* gap) {
   if (V <= 0 || H <= 0 || M < 0) return -1;
   if (M == 0) return 0;
   if (n_threads < 1) n_threads = 1;
@@ -177,7 +194,7 @@ int32_t cai_o_head_rows(const uint16_t* W, int32_t V, int32_t H, const uint16_t*
   }
   int32_t rc = 0;
   for (int32_t t = 0; t < n_threads; ++t) {
-    head_job j = {W, V, H, rows, M, t, n_threads, conf, zmax, lse, gap, argmax, 0};
+    head_job j = {W, V, H, rows, g, eps, M, t, n_threads, conf, zmax, lse, gap, argmax, 0};
     jobs[t] = j;
   }
   int32_t started = 0;
@@ -198,11 +215,21 @@ int32_t cai_o_head_rows(const uint16_t* W, int32_t V, int32_t H, const uint16_t*
 
 /* Full probability vector of one row (for the sum-to-one and brute-force
  * pins): p_v = exp(z_v - m) / S. */
+/* Box 1 without the final RMSNorm. */
+int32_t cai_o_head_rows(const uint16_t* W, int32_t V, int32_t H, const uint16_t* rows, int32_t M,
+                        int32_t n_threads, double* conf, int32_t* argmax, double* zmax, double* lse,
+                        double* gap) {
+  return cai_o_head_rows_norm(W, V, H, rows, M, NULL, 0.0, n_threads, conf, argmax, zmax, lse, gap);
+}
+
 int32_t cai_o_softmax_row(const uint16_t* W, int32_t V, int32_t H, const uint16_t* h, double* z_out,
                           double* p_out) {
   double conf, zmax, lse, gap;
   int32_t idx;
-  head_one_row(W, V, H, h, z_out, &conf, &idx, &zmax, &lse, &gap);
+  double* x = (double*)malloc(sizeof(double) * (size_t)H);
+  if (!x) return -1;
+  head_one_row(W, V, H, h, NULL, 0.0, x, z_out, &conf, &idx, &zmax, &lse, &gap);
+  free(x);
   double S = 0.0;
   for (int32_t v = 0; v < V; ++v) S += exp(z_out[v] - zmax);
   for (int32_t v = 0; v < V; ++v) p_out[v] = exp(z_out[v] - zmax) / S;

@@ -45,7 +45,8 @@ CAI_MASK_TOKEN = -1
 CAI_RUNNING, CAI_EXIT_DONE, CAI_EXIT_GRIND, CAI_EXIT_TMAX = 0, 1, 2, 3
 
 # Every symbol include/cai.h declares.
-EXPORTS = ("cai_config_default", "cai_init", "cai_first_step", "cai_denoise_step",
+EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step",
+           "cai_denoise_step",
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
@@ -99,6 +100,8 @@ def _load():
     sig = {
         "cai_config_default": (ctypes.c_int, [ctypes.POINTER(cai_config), i32, i32, i32, i32, i32, i32, i32]),
         "cai_init": (ctypes.c_int, [ctypes.POINTER(cai_config), vp, vp, ctypes.POINTER(vp)]),
+        "cai_init_rmsnorm": (ctypes.c_int, [ctypes.POINTER(cai_config), vp, vp, ctypes.c_double, vp,
+                                            ctypes.POINTER(vp)]),
         "cai_first_step": (ctypes.c_int, [vp, vp, vp]),
         "cai_denoise_step": (ctypes.c_int, [vp, vp, vp]),
         "cai_block_advance": (ctypes.c_int, [vp, vp]),
@@ -173,10 +176,12 @@ def cai_config_default(preset: int, B: int, P: int, H: int, V: int, T: int, n_bl
 class Ctx:
     """Owning handle of a ``cai_ctx*``; also keeps the sizes for the copies."""
 
-    def __init__(self, handle: int, cfg: cai_config, W):
+    def __init__(self, handle: int, cfg: cai_config, W, norm_weight=None, norm_eps: float = 0.0):
         self.handle = handle
         self.cfg = cfg
         self._W = W  # the weight must outlive the context
+        self.norm_weight = norm_weight
+        self.norm_eps = norm_eps
 
     @property
     def L(self) -> int:
@@ -187,6 +192,15 @@ def cai_init(cfg: cai_config, W, stream=None) -> Ctx:
     h = ctypes.c_void_p()
     _check(lib().cai_init(ctypes.byref(cfg), _ptr(W), _stream(stream), ctypes.byref(h)), "cai_init")
     return Ctx(h.value, cfg, W)
+
+
+def cai_init_rmsnorm(cfg: cai_config, W, norm_weight, eps: float, stream=None) -> Ctx:
+    """cai_init with the model's final RMSNorm (weight ``norm_weight`` [H] bf16,
+    epsilon ``eps``) applied to every decoded row inside the head."""
+    h = ctypes.c_void_p()
+    _check(lib().cai_init_rmsnorm(ctypes.byref(cfg), _ptr(W), _ptr(norm_weight), float(eps),
+                                  _stream(stream), ctypes.byref(h)), "cai_init_rmsnorm")
+    return Ctx(h.value, cfg, W, norm_weight, float(eps))
 
 
 def cai_first_step(ctx: Ctx, hidden, stream=None) -> None:

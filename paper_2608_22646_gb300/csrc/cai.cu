@@ -161,6 +161,11 @@ struct cai_ctx {
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
   CUtensorMap tm_w{};    // wt as [2 n_vt (H / 64) 128, 64], 16 KiB unswizzled boxes
   bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
+  bool norm = false;     // the model's final RMSNorm is part of the head (cai_init_rmsnorm)
+  float norm_eps = 0.0f;
+  float* inv_r = nullptr;  // [rows_cap] 1 / sqrt(mean h^2 + eps) of this step's rows
+  void (*head_kernel)(CUtensorMap, HeadParams) = nullptr;
+  void (*pair_kernel)(CUtensorMap, CUtensorMap, PairParams) = nullptr;
   int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0, reduce_grid = 0;
   size_t pair_smem = 0;
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
@@ -324,15 +329,32 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     gp.BP = c->BP;
     gp.H = cfg.H;
     gp.first = first ? 1 : 0;
+    gp.inv_r = c->norm ? c->inv_r : nullptr;
+    gp.eps = c->norm_eps;
     const int g_grid = c->rows_cap / kGatherRowsPerCta;
     if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) !=
         cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
-  } else if (hid != c->hid_mapped) {
-    // The single-kernel step reads the caller's [B P, H] rows through TMA.
-    if (!make_map(&c->tm_hid, hid, c->BP, cfg.H, kBoxRowsB)) return CAI_ERR_ARG;
-    c->hid_mapped = hid;
+  } else {
+    if (hid != c->hid_mapped) {
+      // The single-kernel step reads the caller's [B P, H] rows through TMA.
+      if (!make_map(&c->tm_hid, hid, c->BP, cfg.H, kBoxRowsB)) return CAI_ERR_ARG;
+      c->hid_mapped = hid;
+    }
+    if (c->norm) {
+      RmsParams rp{};
+      rp.hidden = static_cast<const __nv_bfloat16*>(hid);
+      rp.inv_r = c->inv_r;
+      rp.rows = c->BP;
+      rp.H = cfg.H;
+      rp.eps = c->norm_eps;
+      const int warps = kGatherThreads / 32;
+      if (launch_pdl(c->pdl, row_rms_kernel, (c->BP + warps - 1) / warps, kGatherThreads, 0,
+                     stream, rp) != cudaSuccess)
+        return check_launch(c);
+      c->stats.launches++;
+    }
   }
 
   HeadParams hp{};
@@ -355,6 +377,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.slot_cols = c->slot_cols;
   hp.gmax = c->gmax;
   hp.tmem_cols = c->tmem_cols;
+  hp.inv_r = c->inv_r;
   const CommitParams cp = commit_params(c, t, step_id);
   if (c->fused) hp.cp = cp;
   cudaEvent_t e0 = nullptr, e1 = nullptr;
@@ -371,7 +394,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     c->ev_used += 2;
     cudaEventRecord(e0, stream);
   }
-  if (launch_pdl(c->pdl, lm_head_softmax_kernel, c->G, kHeadThreads, c->head_smem, stream,
+  if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream,
                  c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
     return check_launch(c);
   c->stats.launches++;
@@ -388,7 +411,8 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     pp.n_vt = c->n_vt;
     pp.min_M = c->pair_min_M;
     pp.n_stages = c->pair_stages;
-    if (launch_pdl(c->pdl, lm_head_pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
+    pp.inv_r = c->inv_r;
+    if (launch_pdl(c->pdl, c->pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
                    c->tm_a, c->tm_w, pp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
@@ -451,7 +475,11 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
   return CAI_OK;
 }
 
-int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) {
+namespace {
+
+// cai_init and cai_init_rmsnorm; g (bf16 [H], host or device) is null for cai_init.
+int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, void* stream,
+              cai_ctx** out) {
   if (!cfg || !W || !out) return CAI_ERR_ARG;
   *out = nullptr;
   int r = validate(cfg);
@@ -478,6 +506,10 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   c->rows_cap = round_up(c->BP, 16);
   c->pdl = pdl_enabled();
   c->fused = c->BP <= kChunkN;
+  c->norm = g != nullptr;
+  c->norm_eps = static_cast<float>(eps);
+  c->head_kernel = c->norm ? lm_head_softmax_kernel<true> : lm_head_softmax_kernel<false>;
+  c->pair_kernel = c->norm ? lm_head_pair_kernel<true> : lm_head_pair_kernel<false>;
 
   // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
   // at least kMinCtaRows vocabulary rows per CTA), tile group size (tiles sharing one hidden
@@ -532,7 +564,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   };
   // Dynamic shared memory may use what the kernel's static shared memory leaves.
   cudaFuncAttributes head_attr{};
-  if (cudaFuncGetAttributes(&head_attr, lm_head_softmax_kernel) != cudaSuccess) {
+  if (cudaFuncGetAttributes(&head_attr, c->head_kernel) != cudaSuccess) {
     cudaGetLastError();
     delete c;
     return CAI_ERR_CUDA;
@@ -552,7 +584,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   if (c->use_pair) {
     c->n_vt = (cfg->V + kPairTileVocab - 1) / kPairTileVocab;
     cudaFuncAttributes pa{};
-    if (cudaFuncGetAttributes(&pa, lm_head_pair_kernel) != cudaSuccess) {
+    if (cudaFuncGetAttributes(&pa, c->pair_kernel) != cudaSuccess) {
       cudaGetLastError();
       delete c;
       return CAI_ERR_CUDA;
@@ -563,7 +595,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     c->pair_stages = ps;
     c->pair_smem = pair_smem_bytes(ps);
     int clusters = 0;
-    if (cudaFuncSetAttribute(lm_head_pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+    if (cudaFuncSetAttribute(c->pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(c->pair_smem)) != cudaSuccess) {
       cudaGetLastError();
       delete c;
@@ -573,7 +605,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     qc.gridDim = dim3(static_cast<unsigned>(sms & ~1));
     qc.blockDim = dim3(kPairThreads);
     qc.dynamicSmemBytes = c->pair_smem;
-    if (cudaOccupancyMaxActiveClusters(&clusters, lm_head_pair_kernel, &qc) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&clusters, c->pair_kernel, &qc) != cudaSuccess ||
         clusters < 1) {
       cudaGetLastError();
       delete c;
@@ -622,10 +654,37 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   }
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
   CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
+  if (c->norm) {
+    CAI_ALLOC(c->inv_r, float, c->rows_cap)
+    if (cudaMemset(c->inv_r, 0, sizeof(float) * c->rows_cap) != cudaSuccess) {
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+  }
+  // The norm weight, on the device for the pack kernels (staged if host).
+  const __nv_bfloat16* g_dev = static_cast<const __nv_bfloat16*>(g);
+  void* g_tmp = nullptr;
+  if (g && !is_device_ptr(g)) {
+    if ((r = dev_alloc(&g_tmp, static_cast<size_t>(cfg->H) * 2)) != CAI_OK) {
+      release(c);
+      delete c;
+      return r;
+    }
+    if (cudaMemcpy(g_tmp, g, static_cast<size_t>(cfg->H) * 2, cudaMemcpyHostToDevice) !=
+        cudaSuccess) {
+      cudaFree(g_tmp);
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    g_dev = static_cast<const __nv_bfloat16*>(g_tmp);
+  }
   const void* w_src = W;
   void* w_tmp = nullptr;
   if (!is_device_ptr(W)) {
     if ((r = dev_alloc(&w_tmp, static_cast<size_t>(cfg->V) * cfg->H * 2)) != CAI_OK) {
+      if (g_tmp) cudaFree(g_tmp);
       release(c);
       delete c;
       return r;
@@ -633,6 +692,7 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     if (cudaMemcpy(w_tmp, W, static_cast<size_t>(cfg->V) * cfg->H * 2, cudaMemcpyHostToDevice) !=
         cudaSuccess) {
       cudaFree(w_tmp);
+      if (g_tmp) cudaFree(g_tmp);
       release(c);
       delete c;
       return CAI_ERR_CUDA;
@@ -643,14 +703,15 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
     const long long n_chunks = static_cast<long long>(units) * kUnitRows * cfg->H / 8;
     pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
         static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
-        c->gmax, n_chunks);
+        c->gmax, n_chunks, g_dev);
     if (c->use_pair)
       pack_w_tiles_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
           static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wt), cfg->V, cfg->H,
-          static_cast<long long>(2 * c->n_vt) * kPairHalf * cfg->H / 8);
+          static_cast<long long>(2 * c->n_vt) * kPairHalf * cfg->H / 8, g_dev);
     const cudaError_t e1 = cudaGetLastError();
     const cudaError_t e2 = cudaStreamSynchronize(static_cast<cudaStream_t>(stream));
     if (w_tmp) cudaFree(w_tmp);
+    if (g_tmp) cudaFree(g_tmp);
     if (e1 != cudaSuccess || e2 != cudaSuccess) {
       release(c);
       delete c;
@@ -682,9 +743,9 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   // small gather and merge CTAs can be resident on an SM beside an LM-head
   // CTA; under programmatic dependent launch they then start, and wait, while
   // the neighbouring kernel still runs.
-  if (cudaFuncSetAttribute(lm_head_softmax_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
+  if (cudaFuncSetAttribute(c->head_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                            static_cast<int>(c->head_smem)) != cudaSuccess ||
-      cudaFuncSetAttribute(lm_head_softmax_kernel,
+      cudaFuncSetAttribute(c->head_kernel,
                            cudaFuncAttributePreferredSharedMemoryCarveout,
                            cudaSharedmemCarveoutMaxShared) != cudaSuccess ||
       cudaFuncSetAttribute(gather_rows_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -708,6 +769,20 @@ int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) 
   }
   *out = c;
   return CAI_OK;
+}
+
+}  // namespace
+
+int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) {
+  return init_impl(cfg, W, nullptr, 0.0, stream, out);
+}
+
+int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weight, double eps,
+                     void* stream, cai_ctx** out) {
+  if (!norm_weight || reinterpret_cast<uintptr_t>(norm_weight) % 2 != 0 || !(eps >= 0.0) ||
+      !std::isfinite(eps))
+    return CAI_ERR_ARG;
+  return init_impl(cfg, W, norm_weight, eps, stream, out);
 }
 
 int cai_reset(cai_ctx* c, void* stream_v) {

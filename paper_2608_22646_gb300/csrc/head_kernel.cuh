@@ -50,6 +50,7 @@
 #pragma once
 
 #include <climits>
+#include <cuda_bf16.h>
 #include "commit.cuh"
 #include "ptx.cuh"
 #include "softmax.cuh"
@@ -84,6 +85,7 @@ struct HeadParams {
   int slot_cols;       // tensor-memory columns per tile accumulator (round32(n_max))
   int gmax;            // largest tile group
   int tmem_cols;       // allocated tensor-memory columns (>= 2 gmax slot_cols)
+  const float* inv_r;  // final-norm row scales 1 / sqrt(mean h^2 + eps) [rows] (kNorm only)
   CommitParams cp;     // commit rule, run by the last CTA of a single-kernel step
 };
 
@@ -160,6 +162,15 @@ __host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
   return p;
 }
 
+// Eight bf16 values times eight bf16 weights, rounded to bf16 (final-norm
+// weight folded into W: W[v,k] g[k]).
+__device__ __forceinline__ uint4 scale_chunk(uint4 w, const __nv_bfloat16* g) {
+  __nv_bfloat16* e = reinterpret_cast<__nv_bfloat16*>(&w);
+#pragma unroll
+  for (int i = 0; i < 8; ++i) e[i] = __float2bfloat16_rn(__bfloat162float(e[i]) * __bfloat162float(g[i]));
+  return w;
+}
+
 // Pack W [V, H] (row-major bf16) for a grid of G CTAs over `units` units of
 // kUnitRows rows and groups of up to gmax tiles.  Inside a stage block, row r's
 // 16-byte chunk c (k = 8c..8c+7 of the block's 64) sits at
@@ -167,7 +178,8 @@ __host__ __device__ inline CtaPlan cta_plan(int c, int units, int G, int gmax) {
 // atoms.  Rows >= V are zero.  One thread per destination 16-byte chunk;
 // n_chunks = units * kUnitRows * H / 8.
 __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
-                                   int H, int units, int G, int gmax, long long n_chunks) {
+                                   int H, int units, int G, int gmax, long long n_chunks,
+                                   const __nv_bfloat16* __restrict__ gw) {
   const long long unit_bytes = 2ll * kUnitRows * H;
   for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
        d += static_cast<long long>(gridDim.x) * blockDim.x) {
@@ -192,6 +204,7 @@ __global__ void pack_weight_kernel(const uint4* __restrict__ W, uint4* __restric
     const long long v = static_cast<long long>(pl.row0()) + t * kRowsPerTile + r;
     uint4 val = make_uint4(0u, 0u, 0u, 0u);
     if (v < V) val = W[(v * H + static_cast<long long>(kb) * kBlockK) / 8 + cl];
+    if (gw) val = scale_chunk(val, gw + kb * kBlockK + cl * 8);
     out[d] = val;
   }
 }
@@ -268,6 +281,10 @@ struct Ring {
 
 // ---------------------------------------------------------------- kernel --
 
+// kNorm: the model's final RMSNorm is part of the head.  Its weight is
+// already folded into W; row n's logits are scaled by inv_r[n] (written by
+// the previous kernel in the stream: row_rms_kernel or the gather).
+template <bool kNorm>
 __global__ void __launch_bounds__(kHeadThreads, 1)
     lm_head_softmax_kernel(const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
   extern __shared__ uint8_t smem_raw[];
@@ -527,6 +544,16 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             break;
           }
           tc_fence_after();
+          float sc[32];
+#pragma unroll
+          for (int c = 0; c < 32; ++c) sc[c] = kLog2e;
+          if constexpr (kNorm) {
+            // The row scales come from the previous kernel in the stream.
+            if (p.fused) grid_dependency_wait();
+#pragma unroll
+            for (int c = 0; c < 32; ++c)
+              if (n0 + c < M) sc[c] = kLog2e * __ldg(p.inv_r + n0 + c);
+          }
           const uint32_t tgroup =
               tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
           for (int t = pl.group_first(g); t < pl.group_first(g) + pl.group_count(g); ++t) {
@@ -540,7 +567,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
             if (valid) {
 #pragma unroll
               for (int c = 0; c < 32; ++c)
-                online_update(lm[c], ls[c], li[c], __uint_as_float(v[c]) * kLog2e, vrow);
+                online_update(lm[c], ls[c], li[c], __uint_as_float(v[c]) * sc[c], vrow);
             }
           }
           tc_fence_before();
@@ -580,7 +607,13 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 tmem_ld_wait();
                 float m, s;
                 int i;
-                transpose_reduce32(v, valid, vrow, lane, m, s, i);
+                if constexpr (kNorm) {
+                  if (p.fused && g == 0 && t == pl.group_first(g) && c == 0)
+                    grid_dependency_wait();  // row scales from the previous kernel
+                  transpose_reduce32(v, valid, vrow, lane, m, s, i, p.inv_r + n0 + 32 * c);
+                } else {
+                  transpose_reduce32(v, valid, vrow, lane, m, s, i);
+                }
                 merge_tri(rm[c], rs[c], ri[c], m, s, i);
               }
             }

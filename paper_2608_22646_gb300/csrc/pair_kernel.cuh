@@ -35,6 +35,7 @@
 #pragma once
 
 #include <climits>
+#include "head_kernel.cuh"
 #include "ptx.cuh"
 #include "softmax.cuh"
 
@@ -58,6 +59,7 @@ struct PairParams {
   int n_vt;            // ceil(V / 256)
   int min_M;           // smaller steps are left to lm_head_softmax_kernel
   int n_stages;
+  const float* inv_r;  // final-norm row scales [rows] (kNorm only)
 };
 
 __host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
@@ -72,7 +74,7 @@ __host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
 // kernel reads it through a tensor map of [2 n_vt (H / 64) 128, 64] bf16 with
 // 64 x 128 boxes and no swizzle: box (t (H / 64) + kb) is that block.
 __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restrict__ out, int V,
-                                    int H, long long n_chunks) {
+                                    int H, long long n_chunks, const __nv_bfloat16* __restrict__ gw) {
   const int KB = H / kPairBlockK;
   const long long tile_chunks = static_cast<long long>(KB) * (kPairHalfBytes / 16);
   for (long long d = blockIdx.x * static_cast<long long>(blockDim.x) + threadIdx.x; d < n_chunks;
@@ -86,6 +88,7 @@ __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restri
     const long long v = t * kPairHalf + r;
     uint4 val = make_uint4(0u, 0u, 0u, 0u);
     if (v < V) val = W[(v * H + static_cast<long long>(kb) * kPairBlockK) / 8 + cl];
+    if (gw) val = scale_chunk(val, gw + kb * kPairBlockK + cl * 8);
     out[d] = val;
   }
 }
@@ -137,6 +140,9 @@ __device__ __forceinline__ void pair_drain(uint64_t* bar, uint32_t parity, uint3
   }
 }
 
+// kNorm: as in lm_head_softmax_kernel, row n's logits are scaled by inv_r[n]
+// (written by the gather).
+template <bool kNorm>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_a,
                         const __grid_constant__ CUtensorMap tm_w, const PairParams p) {
@@ -274,6 +280,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       if (!mbar_wait(&sm.accf[acc], (i >> 1) & 1, sm.abort, p.err, kErrWaitAccFull)) break;
       tc_fence_after();
       const uint32_t tbase = tmem_base + lane_base + static_cast<uint32_t>(acc * kPairTileVocab);
+      const int row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf + quarter * 32 + lane;
+      float rs = kLog2e;
+      if constexpr (kNorm) {
+        if (row < M) rs = kLog2e * __ldg(p.inv_r + row);
+      }
       const int vbase = v * kPairTileVocab;
       float m = kNegBig, s = 0.0f;
       int ix = INT_MAX;
@@ -288,7 +299,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         int ci = 0;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          const float z = __uint_as_float(x[k]) * kLog2e;
+          const float z = __uint_as_float(x[k]) * rs;
           if (k < nvalid && z > cm) {
             cm = z;
             ci = k;
@@ -302,7 +313,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         float cs = 0.0f;
 #pragma unroll
         for (int k = 0; k < 32; ++k) {
-          const float z = __uint_as_float(x[k]) * kLog2e;
+          const float z = __uint_as_float(x[k]) * rs;
           cs += k < nvalid ? fast_exp2(z - m) : 0.0f;
         }
         s += cs;
@@ -315,7 +326,6 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         else
           mbar_arrive_cluster(acce_remote + static_cast<uint32_t>(acc * 8));
       }
-      const int row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf + quarter * 32 + lane;
       if (row < M)
         p.part[static_cast<size_t>(row) * p.n_vt + v] = make_float4(m, s, __int_as_float(ix), 0.0f);
     }

@@ -61,14 +61,18 @@ __device__ __forceinline__ void transpose_merge32(float (&m)[32], float (&s)[32]
 }
 
 // 32 rows (one per lane) x 32 columns of logits -> lane l holds the
-// (max, sum, argmax) of column l over the 32 rows.
+// (max, sum, argmax) of column l over the 32 rows.  Column c's logits are
+// scaled by log2 e, times col_scale[c] when given (a per-row normalisation
+// of the decoded hidden states, see lm_head_softmax_kernel).
 __device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
-                                                   int lane, float& om, float& os, int& oi) {
+                                                   int lane, float& om, float& os, int& oi,
+                                                   const float* col_scale = nullptr) {
   float m[32], s[32];
   int ix[32];
 #pragma unroll
   for (int c = 0; c < 32; ++c) {
-    m[c] = valid ? __uint_as_float(v[c]) * kLog2e : kNegBig;
+    const float sc = col_scale ? kLog2e * __ldg(col_scale + c) : kLog2e;
+    m[c] = valid ? __uint_as_float(v[c]) * sc : kNegBig;
     s[c] = valid ? 1.0f : 0.0f;
     ix[c] = valid ? vrow : INT_MAX;
   }

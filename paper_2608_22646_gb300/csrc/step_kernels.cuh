@@ -26,7 +26,21 @@ struct GatherParams {
   int* d_M;                     // masked rows of this step
   int B, BP, H;
   int first;                    // step zero: every position of every sequence
+  float* inv_r;                 // final norm: 1 / sqrt(mean h^2 + eps) per row, or null
+  float eps;
 };
+
+// Sum of squares of eight bf16 values, in fp32.
+__device__ __forceinline__ float sumsq8(uint4 x) {
+  const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&x);
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float f = __bfloat162float(e[i]);
+    s = fmaf(f, f, s);
+  }
+  return s;
+}
 
 __global__ void __launch_bounds__(kGatherThreads)
     gather_rows_kernel(const GatherParams p) {
@@ -42,17 +56,61 @@ __global__ void __launch_bounds__(kGatherThreads)
   }
   const int rows_pad = (M + 15) & ~15;
   const int r = blockIdx.x * kGatherRowsPerCta + threadIdx.x / 64;
-  if (r >= rows_pad) return;
   const int t = threadIdx.x & 63;
   const int nvec = p.H / 8;  // 16-byte vectors per row
-  uint4* dst = reinterpret_cast<uint4*>(p.hc + static_cast<size_t>(r) * p.H);
-  if (r < M) {
-    const int src_row = p.first ? r : p.list[r];
-    const uint4* src = reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(src_row) * p.H);
-    for (int v = t; v < nvec; v += 64) dst[v] = __ldg(src + v);
-  } else {
-    for (int v = t; v < nvec; v += 64) dst[v] = make_uint4(0u, 0u, 0u, 0u);
+  float ss = 0.0f;
+  if (r < rows_pad) {
+    uint4* dst = reinterpret_cast<uint4*>(p.hc + static_cast<size_t>(r) * p.H);
+    if (r < M) {
+      const int src_row = p.first ? r : p.list[r];
+      const uint4* src =
+          reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(src_row) * p.H);
+      for (int v = t; v < nvec; v += 64) {
+        const uint4 x = __ldg(src + v);
+        dst[v] = x;
+        if (p.inv_r) ss += sumsq8(x);
+      }
+    } else {
+      for (int v = t; v < nvec; v += 64) dst[v] = make_uint4(0u, 0u, 0u, 0u);
+    }
   }
+  if (!p.inv_r) return;
+  // A row's 64 threads are two whole warps: reduce in each, then across the two.
+  __shared__ float s_half[kGatherThreads / 32];
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  if ((threadIdx.x & 31) == 0) s_half[threadIdx.x >> 5] = ss;
+  __syncthreads();
+  if (t == 0 && r < rows_pad) {
+    const float tot = s_half[threadIdx.x >> 5] + s_half[(threadIdx.x >> 5) + 1];
+    p.inv_r[r] = r < M ? rsqrtf(tot / static_cast<float>(p.H) + p.eps) : 1.0f;
+  }
+}
+
+// ------------------------------------------------ final-norm row scales --
+
+struct RmsParams {
+  const __nv_bfloat16* hidden;  // [rows, H] the caller's rows (single-kernel step)
+  float* inv_r;                 // [rows] 1 / sqrt(mean h^2 + eps)
+  int rows, H;
+  float eps;
+};
+
+// One warp per row.  Reads only the caller's rows; writes inv_r, which the
+// previous LM-head launch may still read, so it waits for that kernel first.
+__global__ void __launch_bounds__(kGatherThreads) row_rms_kernel(const RmsParams p) {
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
+  const int lane = threadIdx.x & 31;
+  float ss = 0.0f;
+  if (row < p.rows) {
+    const uint4* src = reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(row) * p.H);
+    for (int v = lane; v < p.H / 8; v += 32) ss += sumsq8(__ldg(src + v));
+  }
+#pragma unroll
+  for (int off = 16; off >= 1; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+  grid_dependency_wait();
+  if (row < p.rows && lane == 0) p.inv_r[row] = rsqrtf(ss / static_cast<float>(p.H) + p.eps);
 }
 
 // ------------------------------------------------------ list rebuild -----

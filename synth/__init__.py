@@ -151,3 +151,29 @@ class HiddenStates:
             out.copy_(h)
             return out
         return h
+
+
+# ---------------------------------------------------------------- final norm --
+
+def final_norm_weight(H: int, seed: int = 5, device="cpu") -> torch.Tensor:
+    """Stand-in for the weight of a model's final RMSNorm: 1 + 0.15 N(0, 1), bf16."""
+    g = _gen(seed * 7 + 3, device)
+    return (1.0 + 0.15 * torch.randn(H, generator=g, device=device,
+                                     dtype=torch.float32)).to(torch.bfloat16)
+
+
+class PreNormHidden:
+    """The rows of a ``HiddenStates`` generator times a fixed positive scale per
+    position (0.3 to 3.0): a stand-in for the last layer's output before the
+    model's final RMSNorm, which removes the scale again."""
+
+    def __init__(self, hs: HiddenStates, seed: int = 21):
+        wl = hs.wl
+        g = _gen(seed * 13 + 5, hs.device)
+        self.hs = hs
+        self.wl = wl
+        self.scale = 0.3 + 2.7 * torch.rand((wl.B, wl.P, 1), generator=g, device=hs.device,
+                                            dtype=torch.float32)
+
+    def __call__(self, blk: int, s: int) -> torch.Tensor:
+        return (self.hs(blk, s).to(torch.float32) * self.scale).to(torch.bfloat16)

@@ -68,8 +68,9 @@ class StepReport:
 
 
 def check_step(ocfg: oracle.Config, W, hidden_bph, pre: dict, post: dict, blk: int, t: int,
-               rep: StepReport | None = None) -> StepReport:
-    """Teacher-forced check of one GPU step (pre -> post) against the oracle."""
+               rep: StepReport | None = None, norm_weight=None, eps: float = 0.0) -> StepReport:
+    """Teacher-forced check of one GPU step (pre -> post) against the oracle
+    (with the final RMSNorm in the head when ``norm_weight`` is given)."""
     rep = rep or StepReport()
     st = to_oracle_state(ocfg, pre)
     B, P = ocfg.B, ocfg.P
@@ -82,7 +83,7 @@ def check_step(ocfg: oracle.Config, W, hidden_bph, pre: dict, post: dict, blk: i
     idx_o = np.full((B, P), -1, np.int32)
     gap_o = np.full((B, P), np.inf)
     if M:
-        h = oracle.head_rows(W, np.ascontiguousarray(hb[mk]))
+        h = oracle.head_rows(W, np.ascontiguousarray(hb[mk]), norm_weight=norm_weight, eps=eps)
         conf_o[mk], idx_o[mk], gap_o[mk] = h["conf"], h["idx"], h["gap"]
     g_conf = post["conf"][:, sl].astype(np.float64)
     g_cand = post["cand"][:, sl]
@@ -143,7 +144,7 @@ def run_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_blocks: int | None = No
                 cai.cai_denoise_step(ctx, h)
             torch.cuda.synchronize()
             post = cai.cai_state_download(ctx)
-            check_step(ocfg, W_host, h, pre, post, blk, t, rep)
+            check_step(ocfg, W_host, h, pre, post, blk, t, rep, ctx.norm_weight, ctx.norm_eps)
             pre = post
             steps += 1
             if max_steps is not None and steps >= max_steps:

@@ -103,6 +103,69 @@ def test_head_bruteforce_tiny(seed):
     assert idx == idx_ref
 
 
+def _q(x):
+    """float32 array -> (bf16 bits, the exact float values they decode to)."""
+    b = bf16_from_float(np.asarray(x, np.float32))
+    return b, (b.astype(np.uint32) << 16).view(np.float32).reshape(np.shape(x))
+
+
+@pytest.mark.parametrize("seed", range(8))
+def test_head_rmsnorm_bruteforce_tiny(seed):
+    # The final RMSNorm in the head: x = g h / sqrt(mean h^2 + eps), z = W x,
+    # in 60-digit arithmetic on tiny random inputs.
+    rng = np.random.default_rng(100 + seed)
+    V, H = int(rng.integers(2, 9)), int(rng.integers(1, 6))
+    Wb, Wq = _q(rng.normal(0, 1.5, (V, H)))
+    hb, hq = _q(rng.normal(0, 2.0, (H,)))
+    gb, gq = _q(rng.normal(1, 0.3, (H,)))
+    eps = float(rng.choice([0.0, 1e-6, 0.3]))
+    mpmath.mp.dps = 60
+    r = mpmath.sqrt(mpmath.fsum(mpmath.mpf(float(v)) ** 2 for v in hq) / H + mpmath.mpf(eps))
+    x = [mpmath.mpf(float(gq[k])) * mpmath.mpf(float(hq[k])) / r for k in range(H)]
+    z = [mpmath.fsum(mpmath.mpf(float(Wq[v, k])) * x[k] for k in range(H)) for v in range(V)]
+    m = max(z)
+    idx = min(v for v in range(V) if z[v] == m)
+    c = float(1 / mpmath.fsum(mpmath.e ** (zv - m) for zv in z))
+    out = oracle.head_rows(Wb, hb.reshape(1, H), norm_weight=gb, eps=eps)
+    assert out["idx"][0] == idx
+    assert abs(out["conf"][0] - c) < 1e-12
+
+
+def test_head_rmsnorm_reductions():
+    rng = np.random.default_rng(7)
+    V, H = 41, 64
+    Wb, Wq = _q(rng.normal(0, 0.5, (V, H)))
+    h = np.where(rng.random((3, H)) < 0.5, -1.0, 1.0)  # mean square exactly 1
+    hb, _ = _q(h)
+    one, _ = _q(np.ones(H))
+    plain = oracle.head_rows(Wb, hb)
+    # g = 1, eps = 0 and unit mean square: the norm is the identity
+    same = oracle.head_rows(Wb, hb, norm_weight=one, eps=0.0)
+    np.testing.assert_array_equal(same["idx"], plain["idx"])
+    np.testing.assert_allclose(same["conf"], plain["conf"], rtol=1e-15, atol=0)
+    # scale invariance (eps = 0): 2h and h/4 are exact in bf16
+    for s in (2.0, 0.25):
+        hs, _ = _q(h * s)
+        o = oracle.head_rows(Wb, hs, norm_weight=one, eps=0.0)
+        np.testing.assert_allclose(o["conf"], plain["conf"], rtol=1e-15, atol=0)
+        np.testing.assert_array_equal(o["idx"], plain["idx"])
+    # the weight scales the k-th input, not the v-th output: with powers of
+    # two, W g is exact in bf16 and the normed head equals the plain head on W g
+    gpow = 2.0 ** rng.integers(-2, 3, H)
+    gb, _ = _q(gpow)
+    Wg, _ = _q(Wq * gpow[None, :])
+    folded = oracle.head_rows(Wg, hb)
+    normed = oracle.head_rows(Wb, hb, norm_weight=gb, eps=0.0)
+    np.testing.assert_array_equal(normed["idx"], folded["idx"])
+    np.testing.assert_allclose(normed["conf"], folded["conf"], rtol=1e-14, atol=0)
+    # eps, closed form on V = 2: c = sigmoid(|z0 - z1| / sqrt(1 + eps))
+    W2b, W2q = _q(rng.normal(0, 0.3, (2, H)))
+    for eps in (0.0, 0.5, 3.0):
+        o = oracle.head_rows(W2b, hb[:1], norm_weight=one, eps=eps)
+        d = abs(float(np.dot(W2q[0].astype(np.float64) - W2q[1], h[0]))) / math.sqrt(1 + eps)
+        assert abs(o["conf"][0] - 1.0 / (1.0 + math.exp(-d))) < 1e-14
+
+
 def test_head_transposed_operand_is_caught():
     # W is deliberately non-square and asymmetric: z = W h differs from any
     # use of W's columns.  h picks column 1 only, so z_v = W[v, 1].

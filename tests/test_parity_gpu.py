@@ -127,6 +127,55 @@ def test_fixed_threshold_rule(theta):
             cai.cai_free(ctx)
 
 
+@pytest.mark.parametrize("B,P,gen", [(4, 16, 64), (5, 64, 128)])
+def test_rmsnorm_in_head(B, P, gen):
+    # Final RMSNorm folded into the head, on a single-kernel context (B P = 64)
+    # and a multi-kernel one (B P = 320: gather scales, pair and swapped kernels).
+    wl = _wl("toy", B=B, P=P, a0="bimodal", gen_len=gen)
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    g = synth.final_norm_weight(wl.H, seed=9, device="cuda")
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    ctx = cai.cai_init_rmsnorm(cfg, W, g, 1e-5)
+    try:
+        hs = synth.HiddenStates(wl, W, "calibrated", seed=13)
+        rep, _ = parity.run_checked_trajectory(ctx, W, synth.PreNormHidden(hs, seed=21))
+        assert rep.rows >= B * P
+    finally:
+        cai.cai_free(ctx)
+
+
+def test_rmsnorm_identity_matches_plain_head():
+    # g = 1, eps = 0 on rows of unit mean square: the norm is the identity, so
+    # the normed context takes the plain context's decisions step for step.
+    wl = _wl("toy", B=2)
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    one = torch.ones(wl.H, dtype=torch.bfloat16, device="cuda")
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    gen_ = torch.Generator(device="cpu").manual_seed(4)
+    signs = (torch.randint(0, 2, (wl.T * wl.n_blocks, wl.B, wl.P, wl.H), generator=gen_) * 2 - 1)
+    hid = lambda blk, t: (signs[blk * wl.T + t] * 1.0).to(torch.bfloat16).to("cuda")
+    a = cai.cai_init(cfg, W)
+    b = cai.cai_init_rmsnorm(cfg, W, one, 0.0)
+    try:
+        for blk in range(wl.n_blocks):
+            if blk:
+                cai.cai_block_advance(a)
+                cai.cai_block_advance(b)
+            for t in range(3):
+                step = cai.cai_first_step if t == 0 else cai.cai_denoise_step
+                step(a, hid(blk, t))
+                step(b, hid(blk, t))
+                torch.cuda.synchronize()
+                sa, sb = cai.cai_state_download(a), cai.cai_state_download(b)
+                np.testing.assert_allclose(sa["conf"], sb["conf"], rtol=0, atol=2e-3)
+                np.testing.assert_array_equal(sa["cand"], sb["cand"])
+                if cai.cai_poll(a, 0, 5000) or cai.cai_poll(b, 0, 5000):
+                    break
+    finally:
+        cai.cai_free(a)
+        cai.cai_free(b)
+
+
 def test_fraction_eta_mode():
     wl = _wl("toy", B=2)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")

@@ -291,7 +291,7 @@ def main():
 
     # Timed region 2 (the roofline figure): the same K generations with CUDA
     # events around every LM-head launch on its stream.
-    head_ms, head_launches = 0.0, 0
+    head_ms, head_launches, step_ms = 0.0, 0, 0.0
     if not args.no_profile:
         cai.cai_profile(ctx, True)
         torch.cuda.synchronize()
@@ -303,6 +303,7 @@ def main():
         stats2 = cai.cai_get_stats(ctx)
         head_launches = stats2["head_launches"] - stats1["head_launches"]
         head_ms = stats2["head_ms"] - stats1["head_ms"]
+        step_ms = stats2["step_ms"] - stats1["step_ms"]
 
     ms, total_positions = aggregate(ms, positions * args.steps, dist, dev)
     value = total_positions / (ms / 1e3)
@@ -319,7 +320,14 @@ def main():
     t_hbm = sum(b / (hbm * 1e9) for b in bytes_t)
     t_tc = sum(f / (tf * 1e12) for f in flops_t)
     t_roof = sum(max(b / (hbm * 1e9), f / (tf * 1e12)) for b, f in zip(bytes_t, flops_t))
-    head_s = max(head_ms, 1e-9) / 1e3 / args.steps       # LM-head time per generation
+    # LM-head time per generation.  Live: the timed region (no events between
+    # kernels, steps overlapping as they run) times the LM head's share of step
+    # time; the share comes from the event-profiled pass (LM-head launches over
+    # whole steps; 1 for single-kernel steps).  Isolated: the profiled pass's
+    # own LM-head time, each launch bracketed by events and run alone.
+    share = min(1.0, head_ms / step_ms) if step_ms > 0 else 1.0
+    head_s = ms / 1e3 / args.steps * share
+    head_iso_s = max(head_ms, 1e-9) / 1e3 / args.steps
     tr = _traffic_record(wl.name)
     per_launch = max(1, head_launches // max(1, args.steps))
     kps = int(stats1["kernels_per_step"])
@@ -328,11 +336,18 @@ def main():
               "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows), "
               "with reduce_partials_kernel" if kps == 5 else "lm_head_softmax_kernel")
     common = {"kernel": kernel, "head_launches": head_launches,
-              "head_ms_total": round(head_ms, 3),
+              "head_share_of_step_time": round(share, 4),
               "roofline_time_frac": round(t_roof / head_s, 4),
-              "timing": "CUDA events around every step's LM-head launch(es) (multi-kernel "
-                        "steps: both LM-head kernels and the row merge, not gather or commit), "
-                        "second pass of the same K generations"}
+              "isolated": {"head_ms_total": round(head_ms, 3),
+                           "achieved_frac": round((sum(bytes_t) / head_iso_s / 1e9 / hbm)
+                                                  if t_hbm >= t_tc else
+                                                  (sum(flops_t) / head_iso_s / 1e12 / tf), 4),
+                           "roofline_time_frac": round(t_roof / head_iso_s, 4)},
+              "timing": "live: CUDA events around the timed region (K generations back to "
+                        "back) x the LM head's share of step time; the share and the isolated "
+                        "figures come from a second pass of the same K generations with events "
+                        "around every step and its LM-head launch(es) (multi-kernel steps: both "
+                        "LM-head kernels and the row merge)"}
     traffic = tr["dram_bytes_per_launch"] if tr else None
     traffic_basis = ("ncu dram read+write of one launch with M = %d (%s); algorithmic bytes of "
                      "that launch %d" % (tr["captured_M"], tr["summary"],

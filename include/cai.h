@@ -166,6 +166,7 @@ typedef struct cai_stats {
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
   int32_t kernels_per_step; /* 1: single-kernel step (B P <= 256); 5 with the CTA-pair
                                LM head and its row merge, 3 without them           */
+  double step_ms;           /* summed device time of profiled steps, every kernel  */
 } cai_stats;
 
 /* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")
@@ -260,8 +261,10 @@ int cai_state_upload(cai_ctx* ctx, const cai_host_state* src);
  * the stream (pinned memory for a truly asynchronous copy). */
 int cai_read_tokens(cai_ctx* ctx, int32_t* host_tokens, void* stream);
 
-/* Time every LM-head launch with CUDA events on its stream (enable = 1) or
- * stop (0).  cai_get_stats synchronises the events and reports the sum. */
+/* Time every step with CUDA events on its stream (enable = 1) or stop (0):
+ * the LM-head launch(es) (head_ms) and the whole step (step_ms).  The events
+ * sit between kernels, so profiled steps run without programmatic overlap.
+ * cai_get_stats synchronises the events and reports the sums. */
 int cai_profile(cai_ctx* ctx, int32_t enable);
 int cai_get_stats(cai_ctx* ctx, cai_stats* out);
 

@@ -182,7 +182,7 @@ struct cai_ctx {
   cai_stats stats{};
   bool profiling = false;
   bool pdl = true;
-  std::vector<cudaEvent_t> ev_pool;  // pairs (start, stop)
+  std::vector<cudaEvent_t> ev_pool;  // per profiled step: step start, head start, head end, step end
   size_t ev_used = 0;                // events recorded since the last stats call
   std::vector<void*> allocs;
 };
@@ -317,6 +317,17 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   }
   const int t = c->t_next;
   const int64_t step_id = c->last_step_id + 1;
+  cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  if (c->profiling) {
+    while (c->ev_used + 4 > c->ev_pool.size()) {
+      cudaEvent_t e;
+      if (cudaEventCreate(&e) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+      c->ev_pool.push_back(e);
+    }
+    for (int k = 0; k < 4; ++k) ev[k] = c->ev_pool[c->ev_used + k];
+    c->ev_used += 4;
+    cudaEventRecord(ev[0], stream);
+  }
 
   if (!c->fused) {
     GatherParams gp{};
@@ -380,20 +391,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.inv_r = c->inv_r;
   const CommitParams cp = commit_params(c, t, step_id);
   if (c->fused) hp.cp = cp;
-  cudaEvent_t e0 = nullptr, e1 = nullptr;
-  if (c->profiling) {
-    if (c->ev_used + 2 > c->ev_pool.size()) {
-      for (int k = 0; k < 2; ++k) {
-        cudaEvent_t e;
-        if (cudaEventCreate(&e) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
-        c->ev_pool.push_back(e);
-      }
-    }
-    e0 = c->ev_pool[c->ev_used];
-    e1 = c->ev_pool[c->ev_used + 1];
-    c->ev_used += 2;
-    cudaEventRecord(e0, stream);
-  }
+  if (c->profiling) cudaEventRecord(ev[1], stream);
   if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream,
                  c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
     return check_launch(c);
@@ -427,7 +425,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       return check_launch(c);
     c->stats.launches++;
   }
-  if (c->profiling) cudaEventRecord(e1, stream);
+  if (c->profiling) cudaEventRecord(ev[2], stream);
   c->stats.head_launches++;
 
   if (!c->fused) {
@@ -437,6 +435,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       return check_launch(c);
     c->stats.launches++;
   }
+  if (c->profiling) cudaEventRecord(ev[3], stream);
   c->stats.steps++;
   int r = check_launch(c);
   if (r != CAI_OK) return r;
@@ -982,16 +981,19 @@ int cai_profile(cai_ctx* c, int32_t enable) {
 int cai_get_stats(cai_ctx* c, cai_stats* out) {
   if (!c || !out) return CAI_ERR_ARG;
   if (c->sticky) return c->sticky;
-  double ms = 0.0;
-  for (size_t i = 0; i < c->ev_used; i += 2) {
-    if (cudaEventSynchronize(c->ev_pool[i + 1]) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
-    float m = 0.f;
-    if (cudaEventElapsedTime(&m, c->ev_pool[i], c->ev_pool[i + 1]) != cudaSuccess)
+  double ms = 0.0, step_ms = 0.0;
+  for (size_t i = 0; i < c->ev_used; i += 4) {
+    if (cudaEventSynchronize(c->ev_pool[i + 3]) != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+    float m = 0.f, s = 0.f;
+    if (cudaEventElapsedTime(&m, c->ev_pool[i + 1], c->ev_pool[i + 2]) != cudaSuccess ||
+        cudaEventElapsedTime(&s, c->ev_pool[i], c->ev_pool[i + 3]) != cudaSuccess)
       return fail(c, CAI_ERR_CUDA);
     ms += m;
+    step_ms += s;
   }
   c->stats.head_ms += ms;
-  c->stats.head_profiled += static_cast<int64_t>(c->ev_used / 2);
+  c->stats.step_ms += step_ms;
+  c->stats.head_profiled += static_cast<int64_t>(c->ev_used / 4);
   c->ev_used = 0;
   *out = c->stats;
   return CAI_OK;

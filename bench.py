@@ -182,6 +182,23 @@ def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0, norm=None):
                       f"fp64, one thread per row), {dt:.1f} s"}
 
 
+def _diagnostics_summary(st: dict) -> dict:
+    """Stability step t_i^* against the first-step confidence s_i (the shape of
+    Section 2.1's token pattern), and the mean drift D^(t) per block."""
+    s0, stable = st["s0"].reshape(-1), st["stable"].reshape(-1).astype(np.int64)
+    out = {}
+    for name, sel in (("s0>0.50", s0 > 0.5), ("0.25<=s0<=0.50", (s0 >= 0.25) & (s0 <= 0.5)),
+                      ("s0<0.25", (s0 < 0.25) & (s0 > 0))):
+        ts = stable[sel & (stable >= 0)]
+        out[name] = {"tokens": int(sel.sum()), "stable": int(ts.size),
+                     "mean_t_star": round(float(ts.mean()), 2) if ts.size else None}
+    d = st["drift"]
+    out["mean_drift_per_block"] = [round(float(np.nanmean(d[:, b, :])), 4)
+                                   if np.isfinite(d[:, b, :]).any() else None
+                                   for b in range(d.shape[1])]
+    return out
+
+
 def aggregate(ms: float, positions: int, dist=None, device=None):
     """Whole-job figures over ranks: the slowest rank's time and the sum of
     every rank's decoded positions (each rank decodes its own batch)."""
@@ -207,6 +224,9 @@ def main():
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-profile", action="store_true",
                     help="time the region without per-kernel events (no roofline figure)")
+    ap.add_argument("--diagnostics", action="store_true",
+                    help="track stability steps and hidden-state drift (CAI_DIAGNOSTICS) and "
+                         "summarise them in the line")
     ap.add_argument("--final-norm", action="store_true",
                     help="the model's final RMSNorm inside the head (cai_init_rmsnorm): inputs "
                          "are the rows before that norm")
@@ -254,6 +274,8 @@ def main():
     torch.cuda.synchronize()
 
     cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    if args.diagnostics:
+        cfg.flags |= cai.CAI_DIAGNOSTICS
     ctx = cai.cai_init_rmsnorm(cfg, W, *norm) if norm else cai.cai_init(cfg, W)
 
     for _ in range(args.warmup):
@@ -383,6 +405,9 @@ def main():
         "clocks": clk.summary(),
     }
 
+    if args.diagnostics:
+        line["config"]["diagnostics"] = True
+        line["diagnostics"] = _diagnostics_summary(st0)
     if not args.no_e2e:
         line["e2e"] = e2e_run(cai, ctx, hs, wl, args, dist, dev)
     if rank == 0 and world == 1 and not args.no_cpu_baseline:

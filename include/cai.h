@@ -68,6 +68,7 @@ extern "C" {
 #define CAI_QUARTER_BLOCKS 16u  /* theta_e^(b) indexed by the quarter of the output block b is in */
 #define CAI_NO_BLOCK_SCHEDULE 32u /* Box 3 alone: every block ends at theta_e1 (ablation "APD") */
 #define CAI_FIXED_THRESHOLD 64u /* fixed-threshold rule (Fast-dLLM): theta^(b)(t) = theta_s      */
+#define CAI_DIAGNOSTICS 128u    /* track stability steps t_i^* and drift D^(t) (Section 2.1)     */
 
 #define CAI_PRESET_LLADA 0      /* gating ON  (Section 5: LLaDA-8B-Instruct) */
 #define CAI_PRESET_DREAM 1      /* gating OFF (Section 5: Dream-7B-Instruct) */
@@ -129,6 +130,15 @@ typedef struct cai_state_view {
   int32_t* exit_step;   /* [B, n_blocks] local step of the exit, -1                 */
   int32_t* unresolved;  /* [B, n_blocks] tokens left masked at the exit             */
   int32_t* m_hist;      /* [n_blocks, T] masked rows decoded by each step (M_t)     */
+  /* CAI_DIAGNOSTICS (Section 2.1); left at their reset values otherwise: */
+  uint8_t* run;         /* [B, L] consecutive decoded steps with the same argmax    */
+  int16_t* stable;      /* [B, L] stability step t_i^*: the local step at which the
+                           argmax has been the same for 3 consecutive decoded steps,
+                           -1 until then (and for tokens committed earlier)        */
+  float* drift;         /* [B, n_blocks, T] relative L2 drift D^(t) of the hidden
+                           states between steps t-1 and t of a block, mean over
+                           the block's P positions (Eq. relative_drift); NaN at
+                           t = 0 and for steps not run                             */
 } cai_state_view;
 
 /*
@@ -150,6 +160,9 @@ typedef struct cai_host_state {
   int32_t* exit_step;
   int32_t* unresolved;
   int32_t* m_hist;
+  uint8_t* run;
+  int16_t* stable;
+  float* drift;
   int32_t blk;
   int32_t t_next;
 } cai_host_state;

@@ -32,6 +32,7 @@ QUARTER_POS = 8
 QUARTER_BLOCKS = 16
 NO_BLOCK_SCHEDULE = 32   # Box 3 alone: theta_e1 in every block ("APD" ablation row)
 FIXED_THRESHOLD = 64     # fixed-threshold rule (Fast-dLLM): theta = theta_s always
+DIAGNOSTICS = 128        # stability step t_i^* and drift D^(t) (Section 2.1)
 
 MASK = -1
 RUNNING, EXIT_DONE, EXIT_GRIND, EXIT_TMAX = 0, 1, 2, 3
@@ -64,7 +65,7 @@ class _Cfg(ctypes.Structure):
 class _State(ctypes.Structure):
     _fields_ = [(n, ctypes.c_void_p) for n in (
         "tok", "conf", "s0", "budget", "cstep", "cand", "ell", "eta",
-        "exit_reason", "exit_step", "unresolved")]
+        "exit_reason", "exit_step", "unresolved", "run", "stable")]
 
 
 _lib = None
@@ -84,6 +85,8 @@ def lib():
         _lib.cai_o_head_rows_norm.restype = i32
         _lib.cai_o_head_rows_norm.argtypes = [u16p, i32, i32, u16p, i32, u16p, d, i32,
                                               u16p, u16p, u16p, u16p, u16p]
+        _lib.cai_o_drift.restype = d
+        _lib.cai_o_drift.argtypes = [u16p, u16p, i32, i32]
         _lib.cai_o_softmax_row.restype = i32
         _lib.cai_o_softmax_row.argtypes = [u16p, i32, i32, u16p, u16p, u16p]
         for name in ("cai_o_theta_e",):
@@ -236,6 +239,8 @@ class State:
     exit_reason: np.ndarray = field(init=False)
     exit_step: np.ndarray = field(init=False)
     unresolved: np.ndarray = field(init=False)
+    run: np.ndarray = field(init=False)
+    stable: np.ndarray = field(init=False)
 
     def __post_init__(self):
         B, L, nb = self.cfg.B, self.cfg.n_blocks * self.cfg.P, self.cfg.n_blocks
@@ -250,9 +255,11 @@ class State:
         self.exit_reason = np.zeros((B, nb), np.int32)
         self.exit_step = np.full((B, nb), -1, np.int32)
         self.unresolved = np.zeros((B, nb), np.int32)
+        self.run = np.zeros((B, L), np.int32)
+        self.stable = np.full((B, L), -1, np.int32)
 
     FIELDS = ("tok", "conf", "s0", "budget", "cstep", "cand", "ell", "eta",
-              "exit_reason", "exit_step", "unresolved")
+              "exit_reason", "exit_step", "unresolved", "run", "stable")
 
     def copy(self) -> "State":
         s = State(self.cfg)
@@ -269,6 +276,16 @@ class State:
         m = self.tok[:, blk * P:(blk + 1) * P] == MASK
         running = self.exit_reason[:, blk] == RUNNING
         return m & running[:, None]
+
+
+def drift(h_prev, h_cur) -> float:
+    """Eq. relative_drift for one sequence: mean over positions of
+    ||h_cur - h_prev|| / ||h_prev||; rows [P, H] bf16."""
+    a, b = bf16_bits(h_prev), bf16_bits(h_cur)
+    H = a.shape[-1]
+    a, b = a.reshape(-1, H), b.reshape(-1, H)
+    assert a.shape == b.shape
+    return float(lib().cai_o_drift(_ptr(a), _ptr(b), a.shape[0], H))
 
 
 def controller_step(st: State, blk: int, t: int, conf_bp: np.ndarray, idx_bp: np.ndarray):

@@ -53,6 +53,16 @@
  *     theta_e1 = 0.70 instead of Box 4's theta_e^(b).
  *   - CAI_O_FIXED_THRESHOLD: the fixed-threshold rule of Fast-dLLM that the
  *     paper compares with: theta^(b)(t) = theta_s for every step and block.
+ *
+ * Diagnostics (Section 2.1, CAI_O_DIAGNOSTICS):
+ *   - the stability step t_i^*: a token is stable once its top prediction has
+ *     been the same at three consecutive steps; t_i^* is the local step of the
+ *     third of them (read here as the step at which stability is first
+ *     observed).  Only steps that decode the token count: a token committed
+ *     before that has no t_i^* (-1).
+ *   - the relative L2 drift D^(t) = mean over the block's positions of
+ *     ||h^(t) - h^(t-1)|| / ||h^(t-1)|| (Eq. relative_drift), per sequence,
+ *     from the hidden states of consecutive steps of one block (cai_o_drift).
  */
 #include <math.h>
 #include <pthread.h>
@@ -67,6 +77,7 @@
 #define CAI_O_QUARTER_BLOCKS 16u
 #define CAI_O_NO_BLOCK_SCHEDULE 32u
 #define CAI_O_FIXED_THRESHOLD 64u
+#define CAI_O_DIAGNOSTICS 128u
 
 #define CAI_O_MASK (-1)
 
@@ -321,6 +332,8 @@ typedef struct {
   int32_t* exit_reason; /* [B, n_blocks] 0 running, 1 done, 2 grinding, 3 T exhausted */
   int32_t* exit_step;   /* [B, n_blocks] local step at which the block exited, -1 */
   int32_t* unresolved;  /* [B, n_blocks] tokens left masked at exit */
+  int32_t* run;         /* [B, L] consecutive decoded steps with the same top prediction */
+  int32_t* stable;      /* [B, L] stability step t_i^*, -1 = not (yet) stable */
 } cai_o_state;
 
 /* One denoising step of Algorithm 1 for every running sequence of the batch,
@@ -346,6 +359,10 @@ void cai_o_controller_step(const cai_o_cfg* c, cai_o_state* st, int32_t blk, int
       if (t == 0) {
         st->s0[g] = ci;
         st->budget[g] = cai_o_budget(c, ci, p);
+      }
+      if (c->flags & CAI_O_DIAGNOSTICS) {
+        st->run[g] = (t > 0 && st->cand[g] == xi) ? st->run[g] + 1 : 1;
+        if (st->run[g] >= 3 && st->stable[g] < 0) st->stable[g] = t;
       }
       st->conf[g] = ci;
       st->cand[g] = xi;
@@ -401,4 +418,21 @@ void cai_o_controller_step(const cai_o_cfg* c, cai_o_state* st, int32_t blk, int
       st->unresolved[eb] = left;
     }
   }
+}
+
+/* Eq. relative_drift for one sequence: the mean over the P positions of
+ * ||h_cur[p] - h_prev[p]||_2 / ||h_prev[p]||_2 (bf16 rows [P, H], fp64). */
+double cai_o_drift(const uint16_t* h_prev, const uint16_t* h_cur, int32_t P, int32_t H) {
+  double sum = 0.0;
+  for (int32_t p = 0; p < P; ++p) {
+    double num = 0.0, den = 0.0;
+    for (int32_t k = 0; k < H; ++k) {
+      const double a = cai_o_bf16_to_double(h_prev[(size_t)p * H + k]);
+      const double d = cai_o_bf16_to_double(h_cur[(size_t)p * H + k]) - a;
+      num += d * d;
+      den += a * a;
+    }
+    sum += sqrt(num) / sqrt(den);
+  }
+  return sum / (double)P;
 }

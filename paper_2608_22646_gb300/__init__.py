@@ -37,6 +37,7 @@ CAI_QUARTER_POS = 8
 CAI_QUARTER_BLOCKS = 16
 CAI_NO_BLOCK_SCHEDULE = 32
 CAI_FIXED_THRESHOLD = 64
+CAI_DIAGNOSTICS = 128
 
 CAI_PRESET_LLADA = 0
 CAI_PRESET_DREAM = 1
@@ -72,7 +73,7 @@ class cai_config(ctypes.Structure):
 
 
 _STATE_FIELDS = ("tok", "conf", "s0", "budget", "cstep", "cand", "ell", "eta", "exit_reason",
-                 "exit_step", "unresolved", "m_hist")
+                 "exit_step", "unresolved", "m_hist", "run", "stable", "drift")
 
 
 class cai_state_view(ctypes.Structure):
@@ -241,6 +242,8 @@ def _host_arrays(ctx: Ctx) -> dict:
         "ell": np.zeros(B, np.int32), "eta": np.zeros(B, np.int32),
         "exit_reason": np.zeros((B, nb), np.int32), "exit_step": np.zeros((B, nb), np.int32),
         "unresolved": np.zeros((B, nb), np.int32), "m_hist": np.zeros((nb, c.T), np.int32),
+        "run": np.zeros((B, L), np.uint8), "stable": np.zeros((B, L), np.int16),
+        "drift": np.zeros((B, nb, c.T), np.float32),
     }
 
 

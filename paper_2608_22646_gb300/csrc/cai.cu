@@ -164,6 +164,7 @@ struct cai_ctx {
   bool norm = false;     // the model's final RMSNorm is part of the head (cai_init_rmsnorm)
   float norm_eps = 0.0f;
   float* inv_r = nullptr;  // [rows_cap] 1 / sqrt(mean h^2 + eps) of this step's rows
+  __nv_bfloat16* h_prev = nullptr;  // [B P, H] previous step's rows (CAI_DIAGNOSTICS)
   void (*head_kernel)(CUtensorMap, HeadParams) = nullptr;
   void (*pair_kernel)(CUtensorMap, CUtensorMap, PairParams) = nullptr;
   int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0, reduce_grid = 0;
@@ -210,7 +211,7 @@ int validate(const cai_config* c) {
       c->n_blocks > 32767 || static_cast<int64_t>(c->n_blocks) * c->P > (1 << 24))
     return CAI_ERR_SHAPE;
   if (c->warmup_pct < 0 || c->warmup_pct > 100 || c->K < 1 || (c->eta_mode != 0 && c->eta_mode != 1) ||
-      !(c->clip_lo <= c->clip_hi) || (c->flags & ~127u) != 0)
+      !(c->clip_lo <= c->clip_hi) || (c->flags & ~255u) != 0)
     return CAI_ERR_ARG;
   return CAI_OK;
 }
@@ -318,6 +319,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   const int t = c->t_next;
   const int64_t step_id = c->last_step_id + 1;
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
+  const bool diag = (cfg.flags & CAI_DIAGNOSTICS) != 0;
   if (c->profiling) {
     while (c->ev_used + 4 > c->ev_pool.size()) {
       cudaEvent_t e;
@@ -327,6 +329,21 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     for (int k = 0; k < 4; ++k) ev[k] = c->ev_pool[c->ev_used + k];
     c->ev_used += 4;
     cudaEventRecord(ev[0], stream);
+  }
+  if (diag) {
+    DriftParams dp{};
+    dp.hidden = static_cast<const __nv_bfloat16*>(hid);
+    dp.prev = c->h_prev;
+    dp.drift = c->st.drift;
+    dp.P = cfg.P;
+    dp.H = cfg.H;
+    dp.n_blocks = cfg.n_blocks;
+    dp.T = cfg.T;
+    dp.blk = c->blk;
+    dp.t = t;
+    if (launch_pdl(c->pdl, drift_kernel, cfg.B, kGatherThreads, 0, stream, dp) != cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
   }
 
   if (!c->fused) {
@@ -638,6 +655,11 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   CAI_ALLOC(c->st.exit_step, int, BN)
   CAI_ALLOC(c->st.unresolved, int, BN)
   CAI_ALLOC(c->st.m_hist, int, static_cast<size_t>(cfg->n_blocks) * cfg->T)
+  CAI_ALLOC(c->st.run, uint8_t, BL)
+  CAI_ALLOC(c->st.stable, int16_t, BL)
+  CAI_ALLOC(c->st.drift, float, BN * cfg->T)
+  if (cfg->flags & CAI_DIAGNOSTICS)
+    CAI_ALLOC(c->h_prev, __nv_bfloat16, static_cast<size_t>(c->BP) * cfg->H)
   CAI_ALLOC(c->list, int, c->BP)
   CAI_ALLOC(c->row_of, int, c->BP)
   CAI_ALLOC(c->d_M, int, 1)
@@ -804,6 +826,9 @@ int cai_reset(cai_ctx* c, void* stream_v) {
             cudaMemsetAsync(c->st.unresolved, 0, BN * 4, s) == cudaSuccess &&
             cudaMemsetAsync(c->st.m_hist, 0, static_cast<size_t>(cfg.n_blocks) * cfg.T * 4, s) ==
                 cudaSuccess &&
+            cudaMemsetAsync(c->st.run, 0, BL, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.stable, 0xFF, BL * 2, s) == cudaSuccess &&
+            cudaMemsetAsync(c->st.drift, 0xFF, BN * cfg.T * 4, s) == cudaSuccess &&  // NaN
             cudaMemsetAsync(c->ticket, 0, 4, s) == cudaSuccess &&
             cudaMemsetAsync(c->pub, 0, 8, s) == cudaSuccess &&
             cudaMemsetAsync(c->err, 0, 4, s) == cudaSuccess &&
@@ -889,6 +914,9 @@ int cai_get_state(cai_ctx* c, cai_state_view* v) {
   v->exit_step = c->st.exit_step;
   v->unresolved = c->st.unresolved;
   v->m_hist = c->st.m_hist;
+  v->run = c->st.run;
+  v->stable = c->st.stable;
+  v->drift = c->st.drift;
   return CAI_OK;
 }
 
@@ -908,6 +936,9 @@ static int transfer(cai_ctx* c, const cai_host_state* h, bool down) {
       {h->exit_reason, c->st.exit_reason, BN * 4}, {h->exit_step, c->st.exit_step, BN * 4},
       {h->unresolved, c->st.unresolved, BN * 4},
       {h->m_hist, c->st.m_hist, static_cast<size_t>(cfg.n_blocks) * cfg.T * 4},
+      {h->run, c->st.run, BL},
+      {h->stable, c->st.stable, BL * 2},
+      {h->drift, c->st.drift, BN * cfg.T * 4},
   };
   if (cudaDeviceSynchronize() != cudaSuccess) return fail(c, CAI_ERR_CUDA);
   for (const F& x : f) {

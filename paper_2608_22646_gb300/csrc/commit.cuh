@@ -19,7 +19,8 @@ enum : uint32_t {
   kFlagPosFactor = 2u,
   kFlagFlush = 4u,
   kFlagQuarterPos = 8u,
-  kFlagQuarterBlocks = 16u
+  kFlagQuarterBlocks = 16u,
+  kFlagDiag = 128u
 };
 constexpr int kMaxP = 256;
 constexpr int kPosPerWarp = 6;   // positions whose partials a warp loads at once
@@ -54,6 +55,9 @@ struct StateArrays {
   int* exit_step;
   int* unresolved;
   int* m_hist;
+  uint8_t* run;     // diagnostics: consecutive decoded steps with the same argmax
+  int16_t* stable;  // diagnostics: stability step t_i^*, -1
+  float* drift;     // diagnostics: [B, n_blocks, T] relative drift D^(t)
 };
 
 struct CommitParams {
@@ -102,9 +106,11 @@ __device__ __forceinline__ int budget_tier(float s, int p, int half, int late) {
 // caller provides (the LM-head kernel lends its drained W ring).
 struct CommitSmem {
   int tok[kMaxP];      // token after this step (kMask while masked)
-  int cand[kMaxP];     // argmax of this step
+  int cand[kMaxP];     // argmax of the previous decoded step, then of this step
   float conf[kMaxP];   // confidence of this step
   uint8_t bud[kMaxP];  // budget before this step
+  uint8_t run[kMaxP];  // diagnostics: same-argmax run before this step
+  int16_t stable[kMaxP];  // diagnostics: stability step before this step
 };
 
 __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs,
@@ -126,9 +132,15 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
     s_running = __ldcg(&p.st.exit_reason[eb]) == kRunning;
     s_ell = __ldcg(&p.st.ell[b]);
   }
+  const bool diag = (p.flags & kFlagDiag) != 0;
   for (int pp = tid; pp < p.P; pp += blockDim.x) {
     s_tok[pp] = __ldcg(&p.st.tok[g0 + pp]);
     s_bud[pp] = p.st.budget[g0 + pp];
+    if (diag) {
+      s_cand[pp] = __ldcg(&p.st.cand[g0 + pp]);
+      cs.run[pp] = __ldcg(&p.st.run[g0 + pp]);
+      cs.stable[pp] = __ldcg(&p.st.stable[g0 + pp]);
+    }
   }
   __syncthreads();
   const bool running = s_running != 0;
@@ -189,6 +201,12 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
             bud = budget_tier(c, pp, p.budget_half, p.budget_late);
             p.st.s0[g] = c;
             p.st.budget[g] = static_cast<uint8_t>(bud);
+          }
+          if (diag) {
+            // Section 2.1: stable once the argmax has held for three decoded steps.
+            const int run = (p.t > 0 && s_cand[pp] == ix) ? cs.run[pp] + 1 : 1;
+            p.st.run[g] = static_cast<uint8_t>(run < 255 ? run : 255);
+            if (run >= 3 && cs.stable[pp] < 0) p.st.stable[g] = static_cast<int16_t>(p.t);
           }
           p.st.conf[g] = c;
           p.st.cand[g] = ix;

@@ -87,6 +87,63 @@ __global__ void __launch_bounds__(kGatherThreads)
   }
 }
 
+// ----------------------------------------------------------- diagnostics --
+
+struct DriftParams {
+  const __nv_bfloat16* hidden;  // [B P, H] this step's rows (every position of the block)
+  __nv_bfloat16* prev;          // [B P, H] the previous step's rows (kept by this kernel)
+  float* drift;                 // [B, n_blocks, T]
+  int P, H, n_blocks, T, blk, t;
+};
+
+// One CTA per sequence: D^(t) = mean over the block's positions of
+// ||h^(t) - h^(t-1)|| / ||h^(t-1)|| (Eq. relative_drift; fp32 sums of the bf16
+// rows), then this step's rows become the previous ones.  At t = 0 only the
+// copy is made.
+__global__ void __launch_bounds__(kGatherThreads) drift_kernel(const DriftParams p) {
+  __shared__ float s_sum[kGatherThreads / 32];
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // the previous step's drift kernel wrote prev
+  const int b = blockIdx.x, warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+  const int nw = blockDim.x >> 5, nvec = p.H / 8;
+  float acc = 0.0f;
+  for (int pp = warp; pp < p.P; pp += nw) {
+    const size_t row = static_cast<size_t>(b) * p.P + pp;
+    const uint4* cur = reinterpret_cast<const uint4*>(p.hidden + row * p.H);
+    uint4* prv = reinterpret_cast<uint4*>(p.prev + row * p.H);
+    float num = 0.0f, den = 0.0f;
+    for (int v = lane; v < nvec; v += 32) {
+      const uint4 x = __ldg(cur + v);
+      if (p.t > 0) {
+        const uint4 y = prv[v];
+        const __nv_bfloat16* xe = reinterpret_cast<const __nv_bfloat16*>(&x);
+        const __nv_bfloat16* ye = reinterpret_cast<const __nv_bfloat16*>(&y);
+#pragma unroll
+        for (int i = 0; i < 8; ++i) {
+          const float a = __bfloat162float(ye[i]);
+          const float d = __bfloat162float(xe[i]) - a;
+          num = fmaf(d, d, num);
+          den = fmaf(a, a, den);
+        }
+      }
+      prv[v] = x;
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      num += __shfl_xor_sync(0xffffffffu, num, off);
+      den += __shfl_xor_sync(0xffffffffu, den, off);
+    }
+    acc += sqrtf(num) / sqrtf(den);
+  }
+  if (lane == 0) s_sum[warp] = acc;
+  __syncthreads();
+  if (threadIdx.x == 0 && p.t > 0) {
+    float tot = 0.0f;
+    for (int w = 0; w < nw; ++w) tot += s_sum[w];
+    p.drift[(static_cast<size_t>(b) * p.n_blocks + p.blk) * p.T + p.t] = tot / static_cast<float>(p.P);
+  }
+}
+
 // ------------------------------------------------ final-norm row scales --
 
 struct RmsParams {

@@ -28,7 +28,8 @@ GAP_TOL = 1e-2
 DEC_TOL = 2e-3
 
 INT_FIELDS = ("tok", "cstep", "budget", "cand", "ell", "eta", "exit_reason", "exit_step",
-              "unresolved")
+              "unresolved", "run", "stable")
+DRIFT_RTOL = 1e-4  # fp32 sums of H products against the fp64 oracle
 
 
 def oracle_config(c: cai.cai_config) -> oracle.Config:
@@ -52,6 +53,8 @@ def to_oracle_state(ocfg: oracle.Config, g: dict) -> oracle.State:
     st.exit_reason[:] = g["exit_reason"]
     st.exit_step[:] = g["exit_step"]
     st.unresolved[:] = g["unresolved"]
+    st.run[:] = g["run"].astype(np.int32)
+    st.stable[:] = g["stable"].astype(np.int32)
     return st
 
 
@@ -133,9 +136,11 @@ def run_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_blocks: int | None = No
     W_host = oracle.bf16_bits(W)
     pre = cai.cai_state_download(ctx)
     steps = 0
+    diag = (c.flags & cai.CAI_DIAGNOSTICS) != 0
     for blk in range(nb):
         if blk:
             cai.cai_block_advance(ctx)
+        h_prev = None
         for t in range(c.T):
             h = hidden_fn(blk, t)
             if t == 0:
@@ -145,6 +150,16 @@ def run_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_blocks: int | None = No
             torch.cuda.synchronize()
             post = cai.cai_state_download(ctx)
             check_step(ocfg, W_host, h, pre, post, blk, t, rep, ctx.norm_weight, ctx.norm_eps)
+            if diag:
+                hb = h.reshape(c.B, c.P, -1)
+                for b in range(c.B):
+                    d = post["drift"][b, blk, t]
+                    if t == 0:
+                        assert np.isnan(d)
+                    else:
+                        od = oracle.drift(h_prev[b], hb[b])
+                        assert abs(d - od) <= DRIFT_RTOL * max(od, 1e-6), (b, blk, t, d, od)
+                h_prev = hb
             pre = post
             steps += 1
             if max_steps is not None and steps >= max_steps:

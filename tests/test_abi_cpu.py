@@ -99,7 +99,7 @@ def test_config_default_values():
     ("n_blocks", 40000, cai.CAI_ERR_SHAPE),
     ("K", 0, cai.CAI_ERR_ARG),
     ("eta_mode", 2, cai.CAI_ERR_ARG),
-    ("flags", 1 << 7, cai.CAI_ERR_ARG),
+    ("flags", 1 << 8, cai.CAI_ERR_ARG),
 ])
 def test_init_validates_before_any_cuda_call(field, value, status):
     c = cai.cai_config_default(0, 1, 16, 256, 4096, 8, 4)

@@ -323,6 +323,48 @@ def test_fixed_threshold_trajectory_commits_exactly_above_threshold():
                 break
 
 
+def test_drift_closed_forms():
+    # Eq. relative_drift on rows whose norms are exact: equal -> 0, doubled ->
+    # 1, negated -> 2, orthogonal unit rows -> sqrt(2); the mean over positions.
+    H = 16
+    e = np.eye(H, dtype=np.float32)
+    prev_b, prev = _q(np.stack([e[0], 2 * e[1] + 2 * e[2], e[3], e[4]]))
+    cur_b, _ = _q(np.stack([e[0], 4 * e[1] + 4 * e[2], -e[3], e[5]]))
+    assert oracle.drift(prev_b[:1], prev_b[:1]) == 0.0
+    assert oracle.drift(prev_b[1:2], cur_b[1:2]) == pytest.approx(1.0, abs=1e-15)
+    assert oracle.drift(prev_b[2:3], cur_b[2:3]) == pytest.approx(2.0, abs=1e-15)
+    assert oracle.drift(prev_b[3:4], cur_b[3:4]) == pytest.approx(math.sqrt(2.0), abs=1e-15)
+    assert oracle.drift(prev_b, cur_b) == pytest.approx((0 + 1 + 2 + math.sqrt(2)) / 4, abs=1e-15)
+
+
+def test_stability_step_hand_trajectory():
+    # t_i^*: the step at which a token's top prediction has been the same for
+    # three consecutive decoded steps.  Gating off and a high fixed threshold
+    # keep tokens masked unless their confidence is set above it.
+    cfg = oracle.Config(B=1, P=4, T=8, n_blocks=2, theta_s=0.9,
+                        flags=oracle.FIXED_THRESHOLD | oracle.DIAGNOSTICS)
+    st = oracle.State(cfg)
+    seq = [  # argmax per position at t = 0..4
+        (5, 5, 5, 7),
+        (5, 6, 6, 7),
+        (5, 6, 5, 8),
+        (5, 6, 6, 8),
+        (5, 6, 5, 8),
+    ]
+    for t, idx in enumerate(seq):
+        conf = np.full((1, 4), 0.01)
+        if t == 1:
+            conf[0, 3] = 0.95  # position 3 commits at t = 1, before it can be stable
+        oracle.controller_step(st, 0, t, conf, np.array([idx], np.int32))
+    assert list(st.stable[0, :4]) == [2, 3, -1, -1]
+    assert list(st.run[0, :3]) == [5, 4, 1]
+    # without the flag nothing is tracked
+    plain = oracle.State(oracle.Config(B=1, P=4, T=8, n_blocks=2, flags=oracle.FIXED_THRESHOLD))
+    for t, idx in enumerate(seq):
+        oracle.controller_step(plain, 0, t, np.full((1, 4), 0.01), np.array([idx], np.int32))
+    assert np.all(plain.stable == -1) and np.all(plain.run == 0)
+
+
 def test_position_factor_printed():
     cfg = oracle.Config(P=64)
     for p, r in _rows("position_factors.txt"):

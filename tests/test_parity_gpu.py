@@ -176,6 +176,23 @@ def test_rmsnorm_identity_matches_plain_head():
         cai.cai_free(b)
 
 
+@pytest.mark.parametrize("B,P,gen", [(4, 16, 64), (5, 64, 128)])
+def test_diagnostics_stability_and_drift(B, P, gen):
+    # Section 2.1 diagnostics on a single- and a multi-kernel context: the
+    # stability steps and same-argmax runs bit-exact against the oracle, the
+    # drift of every step within 1e-4 relative (checked in parity).
+    wl = _wl("toy", B=B, P=P, a0="bimodal", gen_len=gen)
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks,
+                  flags=cai.CAI_GATING | cai.CAI_POS_FACTOR | cai.CAI_DIAGNOSTICS)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=31)
+    try:
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert (final["stable"] >= 2).any()
+        assert np.isfinite(final["drift"][:, 0, 1]).all()
+    finally:
+        cai.cai_free(ctx)
+
+
 def test_fraction_eta_mode():
     wl = _wl("toy", B=2)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")

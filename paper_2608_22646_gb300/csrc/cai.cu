@@ -267,6 +267,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   cp.part = c->part;
   cp.n_part = c->G;
   cp.rowres = c->rowres;
+  cp.pair_pairs = c->pair_grid / 2;
   cp.pair_min_M = c->use_pair ? c->pair_min_M : INT_MAX;
   cp.identity_rows = c->fused ? 1 : 0;
   cp.st = c->st;
@@ -437,6 +438,7 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     rp.d_M = c->d_M;
     rp.n_part = c->n_vt;
     rp.min_M = c->pair_min_M;
+    rp.n_pairs = c->pair_grid / 2;
     if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream, rp) !=
         cudaSuccess)
       return check_launch(c);
@@ -667,8 +669,14 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   CAI_ALLOC(c->pub, unsigned long long, 1)
   CAI_ALLOC(c->err, uint32_t, 1)
   CAI_ALLOC(c->hc, __nv_bfloat16, static_cast<size_t>(c->rows_cap) * cfg->H)
-  CAI_ALLOC(c->part, float4,
-            static_cast<size_t>(c->rows_cap) * (c->use_pair && c->n_vt > c->G ? c->n_vt : c->G))
+  // Partials per row: G (swapped-operand kernel), and with the pair kernel
+  // n_vt (one per vocabulary tile) or up to n_pairs (one per pair).
+  int part_cols = c->G;
+  if (c->use_pair) {
+    part_cols = c->n_vt > part_cols ? c->n_vt : part_cols;
+    part_cols = c->pair_grid / 2 > part_cols ? c->pair_grid / 2 : part_cols;
+  }
+  CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * part_cols)
   if (c->use_pair) {
     CAI_ALLOC(c->wt, uint8_t, static_cast<size_t>(2 * c->n_vt) * kPairHalf * 2 * cfg->H)
     CAI_ALLOC(c->rowres, float4, c->rows_cap)

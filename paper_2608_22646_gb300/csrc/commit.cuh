@@ -65,6 +65,7 @@ struct CommitParams {
   int n_part;             // partial slots per row (one per LM-head CTA)
   const float4* rowres;   // [rows] merged triple per row when the pair kernel decoded the step
   int pair_min_M;         // steps with at least this many rows ran the pair kernel
+  int pair_pairs;         // pairs of the pair kernel's grid
   int identity_rows;      // 1: row of (b, p) is b P + p; 0: row_of[b P + p]
   StateArrays st;
   int* list;

@@ -297,6 +297,14 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
   const CtaPlan pl = cta_plan(cta, p.units, G, p.gmax);
   const int KB = p.H / kBlockK;
 
+  // Multi-kernel step with the pair kernel on: most steps belong to the pair
+  // kernel, so read M first and leave before any setup when it is one of them.
+  if (!p.fused && p.max_M != INT_MAX) {
+    grid_launch_dependents();
+    grid_dependency_wait();
+    if (*p.d_M > p.max_M) return;
+  }
+
   // Prologue (overlaps the previous kernel under programmatic dependent launch).
   if (threadIdx.x == 0) {
     for (int s = 0; s < p.n_stages; ++s) {

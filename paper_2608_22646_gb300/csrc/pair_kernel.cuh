@@ -15,9 +15,13 @@
 // per flop of a single-CTA 128 x 256 tile.
 //
 // A tensor-memory lane holds one row's logits, so the epilogue is a serial
-// online softmax per thread over the 256 columns of a tile, no shuffles.  It
-// writes one partial (max * log2 e, sum of 2^(z log2 e - max), argmax) per
-// row and vocabulary tile; the merge kernel combines a row's partials.
+// online softmax per thread over the 256 columns of a tile, no shuffles.  When
+// the number of pairs is a multiple of the number of row tiles n_rt, every
+// tile of a pair has the same row tile, and the epilogue folds its tiles into
+// one partial (max * log2 e, sum of 2^(z log2 e - max), argmax) per row and
+// pair, which the commit reads directly (pair_partials_per_row); otherwise it
+// writes one partial per row and vocabulary tile, merged per row by
+// reduce_partials_kernel.
 //
 // Work: tiles (v, j) of 256 vocabulary rows x 256 masked rows, numbered
 // t = v * n_rt + j and dealt round-robin to the pairs of a persistent grid.
@@ -61,6 +65,14 @@ struct PairParams {
   int n_stages;
   const float* inv_r;  // final-norm row scales [rows] (kNorm only)
 };
+
+// Partials per row written by a pair step with M rows on n_pairs pairs: one
+// per pair of the row's tile when n_pairs is a multiple of the row-tile
+// count, else 0 (one per vocabulary tile, to be merged by the reduce kernel).
+__host__ __device__ inline int pair_partials_per_row(int M, int n_pairs) {
+  const int n_rt = (M + kPairTileRows - 1) / kPairTileRows;
+  return (n_rt > 0 && n_pairs % n_rt == 0) ? n_pairs / n_rt : 0;
+}
 
 __host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
   return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes +
@@ -273,6 +285,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     const int quarter = warp & 3;  // tensor-memory lanes 32 quarter .. 32 quarter + 31
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
     const uint32_t acce_remote = mapa_shared(sm.acce, 0);
+    const int per_row = pair_partials_per_row(M, n_pairs);  // > 0: one partial per pair
+    float am = kNegBig, as = 0.0f;
+    int aix = INT_MAX;
     for (int i = 0; i < my_tiles; ++i) {
       const int t = pair + i * n_pairs;
       const int v = t / n_rt, j = t - v * n_rt;
@@ -326,8 +341,19 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
         else
           mbar_arrive_cluster(acce_remote + static_cast<uint32_t>(acc * 8));
       }
-      if (row < M)
+      if (per_row > 0)
+        merge_tri(am, as, aix, m, s, ix);  // tiles in increasing v: ties keep the lower index
+      else if (row < M)
         p.part[static_cast<size_t>(row) * p.n_vt + v] = make_float4(m, s, __int_as_float(ix), 0.0f);
+    }
+    if (per_row > 0) {
+      // The pair's row tile is fixed (pair mod n_rt); a pair without tiles
+      // writes the empty triple.
+      const int row = (pair % n_rt) * kPairTileRows + static_cast<int>(rank) * kPairHalf +
+                      quarter * 32 + lane;
+      if (row < M)
+        p.part[static_cast<size_t>(row) * per_row + pair / n_rt] =
+            make_float4(am, as, __int_as_float(aix), 0.0f);
     }
   }
 
@@ -350,6 +376,8 @@ struct ReduceParams {
   const int* d_M;
   int n_part;
   int min_M;
+  int n_pairs;         // the pair kernel's grid / 2 (its partials need no merge when
+                       // pair_partials_per_row > 0)
 };
 
 constexpr int kReduceThreads = 256;
@@ -358,7 +386,7 @@ __global__ void __launch_bounds__(kReduceThreads) reduce_partials_kernel(const R
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // the pair kernel's partials
   const int M = *p.d_M;
-  if (M < p.min_M) return;
+  if (M < p.min_M || pair_partials_per_row(M, p.n_pairs) > 0) return;
   const int lane = threadIdx.x & 31;
   const int nw = (gridDim.x * blockDim.x) >> 5;
   for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < M; row += nw) {

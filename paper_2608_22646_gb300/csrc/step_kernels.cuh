@@ -9,6 +9,7 @@
 
 #include <cuda_bf16.h>
 #include "head_kernel.cuh"
+#include "pair_kernel.cuh"
 
 namespace cai {
 
@@ -201,10 +202,16 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
   // This step's M (d_M is rewritten only by the last CTA, after every CTA's
   // merge) tells which LM-head kernel decoded it: the pair kernel's tile
   // partials were already merged into one triple per row.
-  if (*p.d_M >= p.pair_min_M)
-    merge_commit_sequence(p, blockIdx.x, cs, p.rowres, 1);
-  else
+  const int M = *p.d_M;
+  if (M >= p.pair_min_M) {
+    const int per_row = pair_partials_per_row(M, p.pair_pairs);
+    if (per_row > 0)
+      merge_commit_sequence(p, blockIdx.x, cs, p.part, per_row);
+    else
+      merge_commit_sequence(p, blockIdx.x, cs, p.rowres, 1);
+  } else {
     merge_commit_sequence(p, blockIdx.x, cs, p.part, p.n_part);
+  }
   if (gridDim.x > 1) {
     if (threadIdx.x == 0) {
       __threadfence();

@@ -225,7 +225,11 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
  * hidden: the block's final hidden states [B, P, H] bf16, row-major; row
  * (b, p) is the one that predicts position p of the block.  Device pointer:
  * read on the stream, must stay valid until the stream passes this call.
- * Host pointer (pinned or pageable): copied to the device inside the call.
+ * Host pointer: with B P > 256 and page-locked, device-mapped memory (e.g.
+ * cudaHostAlloc), the gather reads the masked rows in place over the host
+ * link, on the stream (valid until the stream passes this call); otherwise
+ * (pageable memory, or B P <= 256) the rows are copied to the device inside
+ * the call.
  * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call
  * cai_block_advance or cai_reset first).
  */

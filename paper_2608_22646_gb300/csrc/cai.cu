@@ -137,6 +137,16 @@ bool is_device_ptr(const void* p) {
   return a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged;
 }
 
+// Device address of page-locked, device-mapped host memory, or null.
+const void* host_mapped_ptr(const void* p) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  return a.type == cudaMemoryTypeHost ? a.devicePointer : nullptr;
+}
+
 }  // namespace
 
 struct cai_ctx {
@@ -312,10 +322,18 @@ int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   const cai_config& cfg = c->cfg;
   const void* hid = hidden;
   if (!is_device_ptr(hidden)) {
-    if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
-                        cudaMemcpyHostToDevice, stream) != cudaSuccess)
-      return fail(c, CAI_ERR_CUDA);
-    hid = c->hidden_stage;
+    // Multi-kernel step on page-locked host rows: the gather reads the masked
+    // rows in place over the host link (only they cross it).  Otherwise the
+    // rows are copied to the device first.
+    const void* mapped = c->fused ? nullptr : host_mapped_ptr(hidden);
+    if (mapped) {
+      hid = mapped;
+    } else {
+      if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
+                          cudaMemcpyHostToDevice, stream) != cudaSuccess)
+        return fail(c, CAI_ERR_CUDA);
+      hid = c->hidden_stage;
+    }
   }
   const int t = c->t_next;
   const int64_t step_id = c->last_step_id + 1;

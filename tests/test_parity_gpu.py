@@ -292,8 +292,14 @@ def test_teacher_forced_random_states():
         cai.cai_free(ctx)
 
 
-def test_host_hidden_and_host_weight_match_device():
+@pytest.mark.parametrize("shape,host", [("toy", "pinned"), ("multi", "pinned"),
+                                        ("multi", "pageable")])
+def test_host_hidden_and_host_weight_match_device(shape, host):
+    # Host inputs: copied in the call (single-kernel steps, or pageable memory)
+    # or, for multi-kernel steps on page-locked memory, read in place by the gather.
     wl = synth.WORKLOADS["toy"]
+    if shape == "multi":
+        wl = _wl("toy", B=5, P=64, gen_len=128)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
     hs = synth.HiddenStates(wl, W, "calibrated")
     cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
@@ -309,8 +315,13 @@ def test_host_hidden_and_host_weight_match_device():
                 h = hs(blk, t)
                 step = cai.cai_first_step if t == 0 else cai.cai_denoise_step
                 step(a, h)
-                step(b, h.cpu().pin_memory())
+                hh = h.cpu()
+                if host == "pinned":
+                    hh = hh.pin_memory()
+                step(b, hh)
                 torch.cuda.synchronize()
+                if cai.cai_poll(a, 0, 5000):
+                    break
         sa, sb = cai.cai_state_download(a), cai.cai_state_download(b)
         for k in ("tok", "conf", "cand", "exit_reason", "m_hist"):
             assert np.array_equal(sa[k], sb[k]), k

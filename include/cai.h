@@ -188,12 +188,12 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
                        int32_t V, int32_t T, int32_t n_blocks);
 
 /*
- * Create a context.  W is the LM-head weight [V, H] bf16, row-major.  If W is
- * a device pointer it must stay valid and unchanged until cai_free (the
- * library reads it in place and never frees it); if it is host memory the
- * library copies it into an owned device buffer before returning.  All state
- * starts at block 0, t = 0, every token masked.  Allocates device memory and
- * one page of mapped pinned host memory.  Synchronous.
+ * Create a context.  W is the LM-head weight [V, H] bf16, row-major, host or
+ * device memory.  It is read once, during this call, into the library's
+ * packed copies (2 V H bytes each: one copy when B P <= 256, two otherwise);
+ * the caller may free or change it afterwards.  All state starts at block 0,
+ * t = 0, every token masked.  Allocates device memory and one page of mapped
+ * pinned host memory.  Synchronous.
  * Errors: CAI_ERR_ARG (NULL cfg/W/out), CAI_ERR_SHAPE, CAI_ERR_UNSUPPORTED,
  * CAI_ERR_NOMEM, CAI_ERR_CUDA.
  */

@@ -180,7 +180,7 @@ class Ctx:
     def __init__(self, handle: int, cfg: cai_config, W, norm_weight=None, norm_eps: float = 0.0):
         self.handle = handle
         self.cfg = cfg
-        self._W = W  # the weight must outlive the context
+        self._W = W  # read into the library's packed copies during cai_init
         self.norm_weight = norm_weight
         self.norm_eps = norm_eps
 

@@ -152,7 +152,6 @@ const void* host_mapped_ptr(const void* p) {
 struct cai_ctx {
   cai_config cfg{};
   int L = 0, BP = 0, rows_cap = 0;
-  const void* W = nullptr;
   StateArrays st{};
   int* list = nullptr;
   int* row_of = nullptr;
@@ -765,7 +764,6 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
       return CAI_ERR_CUDA;
     }
   }
-  c->W = W;
 #undef CAI_ALLOC
   if (cudaHostAlloc(reinterpret_cast<void**>(&c->hf_host), sizeof(HostFlag), cudaHostAllocMapped) !=
           cudaSuccess ||

@@ -23,13 +23,18 @@
  * use programmatic dependent launch: each may be scheduled while the kernel
  * before it in the stream still runs, and waits for that kernel to complete
  * before touching anything it produces (setting CAI_PDL=0 in the environment
- * before cai_init launches them plainly instead).  With B P > 256 a step is
- * gather, LM head, merge + commit; the LM head is then two kernels, of which
- * only one decodes a step: the swapped-operand kernel below 32 masked rows,
- * the CTA-pair kernel (tcgen05 cta_group::2, the masked rows as MMA M) from
- * 32 rows on, followed by a kernel that merges each row's per-tile partials
+ * before cai_init launches them plainly instead).  With B P <= 256 a step is
+ * one kernel: the LM head over every row of the block, whose last CTA applies
+ * the commit rule; it streams W before the previous step has committed and
+ * waits for it only to write its partials and to commit.  With B P > 256 a
+ * step is gather, LM head, merge + commit; the LM head is then two kernels,
+ * of which only one decodes a step: the swapped-operand kernel below 32
+ * masked rows, the CTA-pair kernel (tcgen05 cta_group::2, the masked rows as
+ * MMA M) from 32 rows on, followed by a kernel that merges each row's
+ * per-tile partials when the pair kernel left more than one per pair
  * (CAI_PAIR=0 keeps every step on the first, CAI_PAIR_MIN_M=n moves the
- * threshold; both read at cai_init).  The batch runs
+ * threshold; both read at cai_init).  cai_init_rmsnorm and CAI_DIAGNOSTICS
+ * add one small kernel each to a single-kernel step.  The batch runs
  * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
  * per sequence) and contribute no rows afterwards.  A context is not thread
  * safe; use one context per host thread.

@@ -338,6 +338,13 @@ int cai_test_fail_alloc_after(int32_t n);
  */
 int cai_test_head_grid_limit(int32_t n);
 
+/*
+ * Testing hook: every device buffer of a context is followed by 256 guard
+ * bytes of a fixed pattern.  Synchronises the device, then sets *n_bad to the
+ * number of buffers whose guard bytes changed (a write past their end).
+ */
+int cai_test_check_guards(cai_ctx* ctx, int32_t* n_bad);
+
 #ifdef __cplusplus
 }
 #endif

@@ -51,6 +51,7 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
+           "cai_test_check_guards",
            "cai_head_rows_static")
 
 
@@ -118,6 +119,7 @@ def _load():
         "cai_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
         "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
+        "cai_test_check_guards": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
         "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
     }
     for name, (res, args) in sig.items():
@@ -295,6 +297,13 @@ def cai_test_fail_alloc_after(n: int) -> None:
 
 def cai_test_head_grid_limit(n: int) -> None:
     _check(lib().cai_test_head_grid_limit(n), "cai_test_head_grid_limit")
+
+
+def cai_test_check_guards(ctx: Ctx) -> int:
+    """Number of the context's device buffers written past their end."""
+    n = ctypes.c_int32(0)
+    _check(lib().cai_test_check_guards(ctx.handle, ctypes.byref(n)), "cai_test_check_guards")
+    return n.value
 
 
 def cai_head_rows_static(W, rows, conf, argmax, stream=None) -> None:

@@ -195,6 +195,7 @@ struct cai_ctx {
   std::vector<cudaEvent_t> ev_pool;  // per profiled step: step start, head start, head end, step end
   size_t ev_used = 0;                // events recorded since the last stats call
   std::vector<void*> allocs;
+  std::vector<size_t> alloc_bytes;   // usable bytes of each allocation (guard bytes follow)
 };
 
 namespace {
@@ -225,15 +226,26 @@ int validate(const cai_config* c) {
   return CAI_OK;
 }
 
+// Every context buffer is followed by kGuardBytes of a fixed pattern; a write
+// past the end of a buffer shows up in cai_test_check_guards.
+constexpr size_t kGuardBytes = 256;
+constexpr unsigned char kGuardByte = 0xC3;
+
 int alloc_into(cai_ctx* c, void** dst, size_t bytes) {
-  int r = dev_alloc(dst, bytes);
-  if (r == CAI_OK) c->allocs.push_back(*dst);
-  return r;
+  const size_t padded = (bytes + 255) / 256 * 256;
+  int r = dev_alloc(dst, padded + kGuardBytes);
+  if (r != CAI_OK) return r;
+  c->allocs.push_back(*dst);
+  c->alloc_bytes.push_back(padded);
+  if (cudaMemset(static_cast<char*>(*dst) + padded, kGuardByte, kGuardBytes) != cudaSuccess)
+    return CAI_ERR_CUDA;
+  return CAI_OK;
 }
 
 void release(cai_ctx* c) {
   for (void* p : c->allocs) cudaFree(p);
   c->allocs.clear();
+  c->alloc_bytes.clear();
   if (c->hf_host) cudaFreeHost(c->hf_host);
   c->hf_host = nullptr;
   for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
@@ -1074,6 +1086,26 @@ const char* cai_strerror(int s) {
     case CAI_ERR_NOMEM: return "out of memory";
     default: return "unknown status";
   }
+}
+
+int cai_test_check_guards(cai_ctx* c, int32_t* n_bad) {
+  if (!c || !n_bad) return CAI_ERR_ARG;
+  if (cudaDeviceSynchronize() != cudaSuccess) return fail(c, CAI_ERR_CUDA);
+  unsigned char buf[kGuardBytes];
+  int bad = 0;
+  for (size_t i = 0; i < c->allocs.size(); ++i) {
+    if (cudaMemcpy(buf, static_cast<char*>(c->allocs[i]) + c->alloc_bytes[i], kGuardBytes,
+                   cudaMemcpyDeviceToHost) != cudaSuccess)
+      return fail(c, CAI_ERR_CUDA);
+    for (size_t k = 0; k < kGuardBytes; ++k) {
+      if (buf[k] != kGuardByte) {
+        ++bad;
+        break;
+      }
+    }
+  }
+  *n_bad = bad;
+  return CAI_OK;
 }
 
 int cai_test_head_grid_limit(int32_t n) {

@@ -163,8 +163,10 @@ def run_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_blocks: int | None = No
             pre = post
             steps += 1
             if max_steps is not None and steps >= max_steps:
+                assert cai.cai_test_check_guards(ctx) == 0, "a device buffer was written past its end"
                 return rep, post
             if np.all(post["exit_reason"][:, blk] != 0):
                 assert cai.cai_poll(ctx, 0, 5000)
                 break
+    assert cai.cai_test_check_guards(ctx) == 0, "a device buffer was written past its end"
     return rep, pre

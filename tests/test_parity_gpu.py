@@ -193,6 +193,34 @@ def test_diagnostics_stability_and_drift(B, P, gen):
         cai.cai_free(ctx)
 
 
+def test_guard_bytes_detect_a_write_past_a_buffer():
+    # The guard check itself: a host-issued memset of one byte just past the
+    # token buffer (inside its guard region, memory the context owns) must be
+    # reported; nothing else is touched.
+    import ctypes
+    cudart = None
+    for name in ("libcudart.so", "libcudart.so.13", "/usr/local/cuda/lib64/libcudart.so"):
+        try:
+            cudart = ctypes.CDLL(name)
+            break
+        except OSError:
+            continue
+    if cudart is None:
+        pytest.skip("libcudart not found")
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    try:
+        assert cai.cai_test_check_guards(ctx) == 0
+        tok = cai.cai_get_state(ctx)["tok"]
+        used = wl.B * wl.n_blocks * wl.P * 4
+        padded = (used + 255) // 256 * 256
+        cudart.cudaMemset.argtypes = [ctypes.c_void_p, ctypes.c_int, ctypes.c_size_t]
+        assert cudart.cudaMemset(ctypes.c_void_p(tok + padded), 0, 1) == 0
+        assert cai.cai_test_check_guards(ctx) == 1
+    finally:
+        cai.cai_free(ctx)
+
+
 def test_fraction_eta_mode():
     wl = _wl("toy", B=2)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")

@@ -182,6 +182,18 @@ def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0, norm=None):
                       f"fp64, one thread per row), {dt:.1f} s"}
 
 
+def _trajectory_summary(st: dict) -> dict:
+    """One generation of the workload: steps per block (max over the batch),
+    exits by reason, tokens left unresolved, and the step-zero budgets."""
+    ex = st["exit_reason"]
+    reasons = {"done": 1, "grinding": 2, "t_exhausted": 3}
+    bud = st["budget"].reshape(-1)
+    return {"steps_per_block": [int(x) for x in (st["exit_step"].max(axis=0) + 1)],
+            "exits": {k: int((ex == v).sum()) for k, v in reasons.items()},
+            "unresolved_tokens": int(st["unresolved"].sum()),
+            "budgets": {str(b): int((bud == b).sum()) for b in (8, 32, 64)}}
+
+
 def _diagnostics_summary(st: dict) -> dict:
     """Stability step t_i^* against the first-step confidence s_i (the shape of
     Section 2.1's token pattern), and the mean drift D^(t) per block."""
@@ -401,6 +413,7 @@ def main():
                    "denoising_steps_per_generation": nonzero_launch,
                    "step_calls_per_generation": int(steps_issued)},
         "roofline": roof,
+        "trajectory": _trajectory_summary(st0),
         "gpu_launches": int(gpu_launches),
         "clocks": clk.summary(),
     }

@@ -33,7 +33,8 @@
  * MMA M) from 32 rows on, followed by a kernel that merges each row's
  * per-tile partials when the pair kernel left more than one per pair
  * (CAI_PAIR=0 keeps every step on the first, CAI_PAIR_MIN_M=n moves the
- * threshold; both read at cai_init).  cai_init_rmsnorm and CAI_DIAGNOSTICS
+ * threshold; both read at cai_init; CAI_NVTX=1 wraps every step call in an
+ * NVTX range).  cai_init_rmsnorm and CAI_DIAGNOSTICS
  * add one small kernel each to a single-kernel step.  The batch runs
  * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
  * per sequence) and contribute no rows afterwards.  A context is not thread

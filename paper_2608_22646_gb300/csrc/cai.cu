@@ -5,6 +5,7 @@
 // state transfer.
 #include <cuda.h>
 #include <cuda_runtime.h>
+#include <nvtx3/nvToolsExt.h>
 
 #include <atomic>
 #include <chrono>
@@ -33,6 +34,13 @@ std::atomic<int> g_head_grid_limit{0};
 bool pdl_enabled() {
   const char* e = std::getenv("CAI_PDL");
   return !(e && e[0] == '0');
+}
+
+// NVTX ranges around every step call (CAI_NVTX=1), for profilers that show
+// them (ncu --nvtx); without a profiler attached the calls do nothing.
+bool nvtx_enabled() {
+  const char* e = std::getenv("CAI_NVTX");
+  return e && e[0] == '1';
 }
 
 bool pair_enabled() {
@@ -192,6 +200,7 @@ struct cai_ctx {
   cai_stats stats{};
   bool profiling = false;
   bool pdl = true;
+  bool nvtx = false;
   std::vector<cudaEvent_t> ev_pool;  // per profiled step: step start, head start, head end, step end
   size_t ev_used = 0;                // events recorded since the last stats call
   std::vector<void*> allocs;
@@ -328,7 +337,19 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
 // One denoising step.  Single-kernel step (B P <= 256): the LM-head kernel
 // reads the hidden states in place and its last CTA commits.  Otherwise:
 // gather -> LM head -> merge + commit.
+int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first);
+
 int step(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
+  if (!c->nvtx) return step_impl(c, hidden, stream_v, first);
+  char name[48];
+  std::snprintf(name, sizeof name, "cai step b%d t%d", c->blk, c->t_next);
+  nvtxRangePushA(name);
+  const int r = step_impl(c, hidden, stream_v, first);
+  nvtxRangePop();
+  return r;
+}
+
+int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
   const cai_config& cfg = c->cfg;
   const void* hid = hidden;
@@ -552,6 +573,7 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   c->BP = cfg->B * cfg->P;
   c->rows_cap = round_up(c->BP, 16);
   c->pdl = pdl_enabled();
+  c->nvtx = nvtx_enabled();
   c->fused = c->BP <= kChunkN;
   c->norm = g != nullptr;
   c->norm_eps = static_cast<float>(eps);

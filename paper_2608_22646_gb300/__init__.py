@@ -18,7 +18,8 @@ import os
 import numpy as np
 
 _PKG = os.path.dirname(os.path.abspath(__file__))
-LIB_PATH = os.path.join(_PKG, "libcai.so")
+# CAI_LIB selects another build of the library (e.g. libcai_debug.so).
+LIB_PATH = os.environ.get("CAI_LIB") or os.path.join(_PKG, "libcai.so")
 
 CAI_OK = 0
 CAI_ERR_ARG = -1

@@ -409,6 +409,7 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     gp.H = cfg.H;
     gp.first = first ? 1 : 0;
     gp.inv_r = c->norm ? c->inv_r : nullptr;
+    gp.err = c->err;
     gp.eps = c->norm_eps;
     const int g_grid = c->rows_cap / kGatherRowsPerCta;
     if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) !=

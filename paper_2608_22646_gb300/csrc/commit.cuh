@@ -157,6 +157,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
         row[j] = -1;
         if (pp < p.P && s_tok[pp] == kMask) {
           row[j] = p.identity_rows ? b * p.P + pp : p.row_of[b * p.P + pp];
+          if (!CAI_IN_RANGE(row[j] < p.B * p.P, p.err)) row[j] = -2;
           if (row[j] < 0) {
             if (lane == 0) atomicOr(p.err, kErrBadRow);
             row[j] = -2;

@@ -343,7 +343,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       }
       if (per_row > 0)
         merge_tri(am, as, aix, m, s, ix);  // tiles in increasing v: ties keep the lower index
-      else if (row < M)
+      else if (row < M && CAI_IN_RANGE(v < p.n_vt, p.err))
         p.part[static_cast<size_t>(row) * p.n_vt + v] = make_float4(m, s, __int_as_float(ix), 0.0f);
     }
     if (per_row > 0) {

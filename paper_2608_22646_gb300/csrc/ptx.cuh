@@ -22,7 +22,17 @@ enum : uint32_t {
   kErrDrain = 1u << 4,       // drain of in-flight copies on the abort path
   kErrBadRow = 1u << 5,      // a masked token had no row in this step's list
   kErrWaitEpi = 1u << 6,     // epilogue warps waiting for each other's slices
+  kErrBounds = 1u << 7,      // CAI_DEBUG builds: an index list or partial offset out of range
 };
+
+// CAI_DEBUG builds check index lists and partial offsets before use: a value
+// out of range sets kErrBounds in the error word and the access is skipped.
+// Other builds compile the checks out.
+#ifdef CAI_DEBUG
+#define CAI_IN_RANGE(cond, err) ((cond) ? true : (atomicOr((err), kErrBounds), false))
+#else
+#define CAI_IN_RANGE(cond, err) true
+#endif
 
 __device__ __forceinline__ uint32_t smem_addr(const void* p) {
   return static_cast<uint32_t>(__cvta_generic_to_shared(p));

@@ -25,6 +25,7 @@ struct GatherParams {
   int* list;                    // [B P] token (b P + p) of each masked row
   int* row_of;                  // [B P] row of each token in this step's list, -1
   int* d_M;                     // masked rows of this step
+  uint32_t* err;                // error word (CAI_DEBUG range checks)
   int B, BP, H;
   int first;                    // step zero: every position of every sequence
   float* inv_r;                 // final norm: 1 / sqrt(mean h^2 + eps) per row, or null
@@ -63,7 +64,8 @@ __global__ void __launch_bounds__(kGatherThreads)
   if (r < rows_pad) {
     uint4* dst = reinterpret_cast<uint4*>(p.hc + static_cast<size_t>(r) * p.H);
     if (r < M) {
-      const int src_row = p.first ? r : p.list[r];
+      int src_row = p.first ? r : p.list[r];
+      if (!CAI_IN_RANGE(src_row >= 0 && src_row < p.BP, p.err)) src_row = 0;
       const uint4* src =
           reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(src_row) * p.H);
       for (int v = t; v < nvec; v += 64) {

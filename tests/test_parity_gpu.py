@@ -475,3 +475,32 @@ def test_batched_multi_chunk_step_sampled():
         assert st["m_hist"][0, 0] == wl.B * wl.P
     finally:
         cai.cai_free(ctx)
+
+
+def test_debug_build_range_checks_stay_quiet():
+    # The CAI_DEBUG build checks index lists and partial offsets before every
+    # use (a value out of range sets an error bit and the access is skipped).
+    # Single- and multi-kernel trajectories run clean on it; any flagged
+    # access would surface as CAI_ERR_DEVICE in the state download.
+    import os
+    import subprocess
+    import sys
+    from paper_2608_22646_gb300 import build as cai_build
+    lib = cai_build.build(debug=True)
+    code = (
+        "import synth, torch, paper_2608_22646_gb300 as cai\n"
+        "from tests import parity\n"
+        "for B, P, gen in ((1, 16, 64), (5, 64, 128)):\n"
+        "    wl = synth.Workload('dbg', B=B, H=256, V=4096, gen_len=gen, P=P, T=8, a0='u04')\n"
+        "    W = synth.lm_head_weight(wl.V, wl.H, device='cuda')\n"
+        "    cfg = cai.cai_config_default(0, B, P, wl.H, wl.V, wl.T, wl.n_blocks)\n"
+        "    ctx = cai.cai_init(cfg, W)\n"
+        "    assert cai.LIB_PATH.endswith('libcai_debug.so')\n"
+        "    parity.run_checked_trajectory(ctx, W, synth.HiddenStates(wl, W, 'calibrated', seed=2))\n"
+        "    cai.cai_free(ctx)\n"
+        "print('debug build clean')\n")
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, "-c", code], cwd=root, env={**os.environ, "CAI_LIB": lib},
+                         capture_output=True, text=True, timeout=900)
+    assert out.returncode == 0, out.stdout[-2000:] + out.stderr[-2000:]
+    assert "debug build clean" in out.stdout

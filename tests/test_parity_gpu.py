@@ -504,3 +504,42 @@ def test_debug_build_range_checks_stay_quiet():
                          capture_output=True, text=True, timeout=900)
     assert out.returncode == 0, out.stdout[-2000:] + out.stderr[-2000:]
     assert "debug build clean" in out.stdout
+
+
+def test_long_dream_full_size_steps_sampled():
+    # Long-generation Dream shape (B = 8, P = 64, H = 3584, V = 152064): the
+    # first steps of block 0 run on the pair kernel with two row tiles and
+    # then one (per-pair partials), and the swapped-operand kernel once M < 32;
+    # at every step a sample of the rows it decoded is recomputed by the oracle.
+    wl = synth.WORKLOADS["dream_long"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    rng = np.random.default_rng(5)
+    try:
+        pre = cai.cai_state_download(ctx)
+        seen = set()
+        for t in range(wl.T):
+            h = hs(0, t)
+            (cai.cai_first_step if t == 0 else cai.cai_denoise_step)(ctx, h)
+            torch.cuda.synchronize()
+            post = cai.cai_state_download(ctx)
+            M = int(post["m_hist"][0, t])
+            masked = np.argwhere(pre["tok"][:, :wl.P] == cai.CAI_MASK_TOKEN)
+            masked = [tuple(x) for x in masked if pre["exit_reason"][x[0], 0] == 0]
+            assert len(masked) == M
+            pick = [masked[i] for i in rng.choice(len(masked), size=min(3, len(masked)),
+                                                  replace=False)]
+            rows = oracle.bf16_bits(h)[[b for b, _ in pick], [p for _, p in pick]]
+            o = oracle.head_rows(W, rows)
+            for k, (b, p) in enumerate(pick):
+                assert abs(post["conf"][b, p] - o["conf"][k]) <= parity.CONF_TOL, (t, b, p)
+                if o["gap"][k] > parity.GAP_TOL:
+                    assert post["cand"][b, p] == o["idx"][k], (t, b, p)
+            seen.add("pair2" if M > 256 else "pair1" if M >= 32 else "swap")
+            pre = post
+            if cai.cai_poll(ctx, 0, 5000) or len(seen) == 3:
+                break
+        assert seen == {"pair2", "pair1", "swap"}
+        assert cai.cai_test_check_guards(ctx) == 0
+    finally:
+        cai.cai_free(ctx)

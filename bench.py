@@ -363,7 +363,8 @@ def main():
     head_s = ms / 1e3 / args.steps * share
     head_iso_s = max(head_ms, 1e-9) / 1e3 / args.steps
     tr = _traffic_record(wl.name)
-    per_launch = max(1, head_launches // max(1, args.steps))
+    per_launch = max(1, (head_launches if head_launches else int(steps_issued) * args.steps)
+                     // max(1, args.steps))
     kps = int(stats1["kernels_per_step"])
     kernel = ("lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
               if kps == 1 else
@@ -372,7 +373,8 @@ def main():
     common = {"kernel": kernel, "head_launches": head_launches,
               "head_share_of_step_time": round(share, 4),
               "roofline_time_frac": round(t_roof / head_s, 4),
-              "isolated": {"head_ms_total": round(head_ms, 3),
+              "isolated": None if args.no_profile else
+                          {"head_ms_total": round(head_ms, 3),
                            "achieved_frac": round((sum(bytes_t) / head_iso_s / 1e9 / hbm)
                                                   if t_hbm >= t_tc else
                                                   (sum(flops_t) / head_iso_s / 1e12 / tf), 4),

@@ -366,10 +366,15 @@ def main():
     per_launch = max(1, (head_launches if head_launches else int(steps_issued) * args.steps)
                      // max(1, args.steps))
     kps = int(stats1["kernels_per_step"])
-    kernel = ("lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
-              if kps == 1 else
-              "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows), "
-              "with reduce_partials_kernel" if kps == 5 else "lm_head_softmax_kernel")
+    if kps == 1:
+        kernel = "lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
+    elif stats1["pair_swap_max_n"] >= 32:
+        kernel = (f"lm_head_pair_kernel (every step; swapped orientation for tiles up to "
+                  f"{stats1['pair_swap_max_n']} rows wide)")
+    elif stats1["pair_grid"]:
+        kernel = "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows)"
+    else:
+        kernel = "lm_head_softmax_kernel"
     common = {"kernel": kernel, "head_launches": head_launches,
               "head_share_of_step_time": round(share, 4),
               "roofline_time_frac": round(t_roof / head_s, 4),

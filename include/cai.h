@@ -27,14 +27,19 @@
  * one kernel: the LM head over every row of the block, whose last CTA applies
  * the commit rule; it streams W before the previous step has committed and
  * waits for it only to write its partials and to commit.  With B P > 64 a
- * step is gather, LM head, merge + commit; the LM head is then two kernels,
- * of which only one decodes a step: the swapped-operand kernel below 32
- * masked rows, the CTA-pair kernel (tcgen05 cta_group::2, the masked rows as
- * MMA M) from 32 rows on, followed by a kernel that merges each row's
- * per-tile partials when the pair kernel left more than one per pair
- * (CAI_PAIR=0 keeps every step on the first, CAI_PAIR_MIN_M=n moves the
- * threshold; both read at cai_init; CAI_NVTX=1 wraps every step call in an
- * NVTX range).  cai_init_rmsnorm and CAI_DIAGNOSTICS
+ * step is gather, LM head, merge + commit.  The LM head is the CTA-pair
+ * kernel (tcgen05 cta_group::2), which picks its orientation per step from
+ * the masked-row count M: the rows as MMA N in row tiles of equal width (a
+ * multiple of 32) while that width is at most 192, else as MMA M in 256-row
+ * tiles.  A kernel that merges each row's per-tile partials follows it only
+ * in contexts where some step size leaves more than one partial per pair and
+ * CTA to merge.  CAI_PAIR_SWAP=0 keeps the pair kernel unswapped and moves
+ * the steps below 32 rows to the single-CTA swapped-operand kernel (launched
+ * on every step, returning at once on the others); CAI_PAIR_SWAP_MAX_N=n sets
+ * the widest swapped tile; CAI_PAIR=0 runs every step on the single-CTA
+ * kernel; CAI_PAIR_MIN_M=n sets the smallest step of the pair kernel (all
+ * read at cai_init; CAI_NVTX=1 wraps every step call in an NVTX range).
+ * cai_init_rmsnorm and CAI_DIAGNOSTICS
  * add one small kernel each to a single-kernel step.  The batch runs
  * blocks and steps in lockstep; sequences exit independently (Algorithm 1,
  * per sequence) and contribute no rows afterwards.  A context is not thread
@@ -183,9 +188,14 @@ typedef struct cai_stats {
   int32_t grid;             /* CTAs of the LM-head kernel                          */
   int32_t stages;           /* pipeline stages of the LM-head kernel               */
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
-  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 64); 5 with the CTA-pair
-                               LM head and its row merge, 3 without them           */
+  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 64); else gather,
+                               LM head(s), row merge if needed, commit (2 to 5)    */
   double step_ms;           /* summed device time of profiled steps, every kernel  */
+  int32_t pair_grid;        /* CTAs of the CTA-pair LM head (0: not used)          */
+  int32_t pair_swap_max_n;  /* steps whose tile width in the swapped orientation
+                               (masked rows in the MMA N dimension) is at most
+                               this run swapped on the pair LM head (0: never)     */
+  int32_t pair_stages;      /* pipeline stages of the pair LM head                 */
 } cai_stats;
 
 /* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")

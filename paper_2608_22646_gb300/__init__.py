@@ -92,7 +92,9 @@ class cai_stats(ctypes.Structure):
                 ("head_launches", ctypes.c_int64), ("head_ms", ctypes.c_double),
                 ("head_profiled", ctypes.c_int64), ("grid", ctypes.c_int32),
                 ("stages", ctypes.c_int32), ("n_max", ctypes.c_int32),
-                ("kernels_per_step", ctypes.c_int32), ("step_ms", ctypes.c_double)]
+                ("kernels_per_step", ctypes.c_int32), ("step_ms", ctypes.c_double),
+                ("pair_grid", ctypes.c_int32), ("pair_swap_max_n", ctypes.c_int32),
+                ("pair_stages", ctypes.c_int32)]
 
 
 def _load():

@@ -51,6 +51,17 @@ bool pair_enabled() {
   return !(e && e[0] == '0');
 }
 
+// Widest tile the pair kernel runs in the swapped orientation (masked rows in
+// the MMA N dimension, 32-row granularity): CAI_PAIR_SWAP_MAX_N (32..256), or
+// 0 with CAI_PAIR_SWAP=0; default 192.
+int pair_swap_max_n() {
+  const char* e = std::getenv("CAI_PAIR_SWAP");
+  if (e && e[0] == '0') return 0;
+  const char* n = std::getenv("CAI_PAIR_SWAP_MAX_N");
+  const int v = n ? std::atoi(n) : 0;
+  return v >= 32 && v <= 256 ? v : 192;
+}
+
 // Optional caps on the LM head's W ring depth (CAI_HEAD_STAGES) and tile
 // group size (CAI_HEAD_GMAX), read once per context at cai_init; 0 or unset
 // keeps the defaults.  Tuning knobs only: results do not depend on them.
@@ -179,14 +190,18 @@ struct cai_ctx {
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
   void* wt = nullptr;    // tile-major packed copy of W (pack_w_tiles_kernel), pair kernel
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
+  PairRowMaps tm_rows{};  // ... in 128-, 64-, 32-, 16-row boxes (swapped pair kernel)
   CUtensorMap tm_w{};    // wt as [2 n_vt (H / 64) 128, 64], 16 KiB unswizzled boxes
   bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
+  int swap_max_n = 0;       // ... swapped when its tile width is at most this (pair_swapped)
+  bool head_in_step = true; // the swapped-operand kernel is launched in multi-kernel steps
+  bool need_reduce = false; // some step size leaves per-tile partials to reduce_partials_kernel
   bool norm = false;     // the model's final RMSNorm is part of the head (cai_init_rmsnorm)
   float norm_eps = 0.0f;
   float* inv_r = nullptr;  // [rows_cap] 1 / sqrt(mean h^2 + eps) of this step's rows
   __nv_bfloat16* h_prev = nullptr;  // [B P, H] previous step's rows (CAI_DIAGNOSTICS)
   void (*head_kernel)(CUtensorMap, HeadParams) = nullptr;
-  void (*pair_kernel)(CUtensorMap, CUtensorMap, PairParams) = nullptr;
+  void (*pair_kernel)(CUtensorMap, CUtensorMap, PairRowMaps, PairParams) = nullptr;
   int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0, reduce_grid = 0;
   size_t pair_smem = 0;
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
@@ -301,6 +316,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   cp.n_part = c->G;
   cp.rowres = c->rowres;
   cp.pair_pairs = c->pair_grid / 2;
+  cp.pair_swap_max_n = c->swap_max_n;
   cp.pair_min_M = c->use_pair ? c->pair_min_M : INT_MAX;
   cp.identity_rows = c->fused ? 1 : 0;
   cp.st = c->st;
@@ -464,13 +480,16 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   const CommitParams cp = commit_params(c, t, step_id);
   if (c->fused) hp.cp = cp;
   if (c->profiling) cudaEventRecord(ev[1], stream);
-  if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream,
-                 c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
-    return check_launch(c);
-  c->stats.launches++;
+  if (c->head_in_step) {
+    if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream,
+                   c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
+  }
   if (c->use_pair) {
     // Only one of the two LM-head kernels decodes a step: the other reads
-    // this step's M and returns at once.
+    // this step's M and returns at once (with pair_min_M = 1 the pair kernel
+    // decodes every step and the other one is not launched).
     PairParams pp{};
     pp.d_M = c->d_M;
     pp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
@@ -480,23 +499,27 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     pp.H = cfg.H;
     pp.n_vt = c->n_vt;
     pp.min_M = c->pair_min_M;
+    pp.swap_max_n = c->swap_max_n;
     pp.n_stages = c->pair_stages;
     pp.inv_r = c->inv_r;
     if (launch_pdl(c->pdl, c->pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
-                   c->tm_a, c->tm_w, pp) != cudaSuccess)
+                   c->tm_a, c->tm_w, c->tm_rows, pp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
-    ReduceParams rp{};
-    rp.part = c->part;
-    rp.rowres = c->rowres;
-    rp.d_M = c->d_M;
-    rp.n_part = c->n_vt;
-    rp.min_M = c->pair_min_M;
-    rp.n_pairs = c->pair_grid / 2;
-    if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream, rp) !=
-        cudaSuccess)
-      return check_launch(c);
-    c->stats.launches++;
+    if (c->need_reduce) {
+      ReduceParams rp{};
+      rp.part = c->part;
+      rp.rowres = c->rowres;
+      rp.d_M = c->d_M;
+      rp.n_vt = c->n_vt;
+      rp.min_M = c->pair_min_M;
+      rp.n_pairs = c->pair_grid / 2;
+      rp.swap_max_n = c->swap_max_n;
+      if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream,
+                     rp) != cudaSuccess)
+        return check_launch(c);
+      c->stats.launches++;
+    }
   }
   if (c->profiling) cudaEventRecord(ev[2], stream);
   c->stats.head_launches++;
@@ -589,6 +612,8 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   c->norm = g != nullptr;
   c->norm_eps = static_cast<float>(eps);
   c->head_kernel = c->norm ? lm_head_softmax_kernel<true> : lm_head_softmax_kernel<false>;
+  c->use_pair = !c->fused && pair_enabled();
+  c->swap_max_n = c->use_pair ? pair_swap_max_n() : 0;
   c->pair_kernel = c->norm ? lm_head_pair_kernel<true> : lm_head_pair_kernel<false>;
 
   // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
@@ -598,12 +623,14 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   // Pair kernel (multi-kernel steps only): steps with at least pair_min_M
   // masked rows run on CTA pairs (CAI_PAIR=0 disables it, CAI_PAIR_MIN_M sets
   // the threshold); the swapped-operand kernel then needs N < pair_min_M only,
-  // which keeps its tile groups large.
-  c->use_pair = !c->fused && pair_enabled();
+  // which keeps its tile groups large.  When narrow steps run swapped the pair
+  // kernel decodes every step (pair_min_M = 1: a 32-column tile is as cheap as
+  // the W stream it rides on), and the swapped-operand kernel is not launched.
   if (c->use_pair) {
     const int mset = env_int("CAI_PAIR_MIN_M");
-    c->pair_min_M = mset > 0 ? mset : 32;
+    c->pair_min_M = mset > 0 ? mset : (c->swap_max_n >= kSwapColStep ? 1 : 32);
   }
+  c->head_in_step = !c->use_pair || c->pair_min_M > 1;
   c->n_max = c->rows_cap < kChunkN ? c->rows_cap : kChunkN;
   if (c->use_pair) {
     const int cap = round_up(c->pair_min_M > 1 ? c->pair_min_M - 1 : 1, 16);
@@ -671,9 +698,9 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
     }
     const size_t plimit = static_cast<size_t>(smem_optin) - pa.sharedSizeBytes;
     int ps = 6;
-    while (ps > 2 && pair_smem_bytes(ps) > plimit) --ps;
+    while (ps > 2 && pair_smem_bytes(ps, c->swap_max_n > 0) > plimit) --ps;
     c->pair_stages = ps;
-    c->pair_smem = pair_smem_bytes(ps);
+    c->pair_smem = pair_smem_bytes(ps, c->swap_max_n > 0);
     int clusters = 0;
     if (cudaFuncSetAttribute(c->pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(c->pair_smem)) != cudaSuccess) {
@@ -691,7 +718,15 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
       delete c;
       return CAI_ERR_CUDA;
     }
+    // CAI_PAIR_CLUSTERS caps the grid (tests: per-tile partials at small M).
+    const int cset = env_int("CAI_PAIR_CLUSTERS");
+    if (cset > 0 && cset < clusters) clusters = cset;
     c->pair_grid = 2 * clusters;
+    // Steps whose row-tile count does not divide the pairs leave one partial
+    // per row and vocabulary tile to the reduce kernel; if no step size up to
+    // B P does, that kernel is never launched.
+    for (int rt = 1; rt <= (c->rows_cap + kPairTileRows - 1) / kPairTileRows; ++rt)
+      if (clusters % rt != 0) c->need_reduce = true;
     const int warps_per_cta = kReduceThreads / 32;
     const int want = (c->rows_cap + warps_per_cta - 1) / warps_per_cta;
     c->reduce_grid = want < 4 * sms ? want : 4 * sms;
@@ -735,8 +770,9 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   // n_vt (one per vocabulary tile) or up to n_pairs (one per pair).
   int part_cols = c->G;
   if (c->use_pair) {
-    part_cols = c->n_vt > part_cols ? c->n_vt : part_cols;
-    part_cols = c->pair_grid / 2 > part_cols ? c->pair_grid / 2 : part_cols;
+    const int k = c->swap_max_n > 0 ? 2 : 1;  // swapped steps: one partial per CTA of a pair
+    part_cols = k * c->n_vt > part_cols ? k * c->n_vt : part_cols;
+    part_cols = k * (c->pair_grid / 2) > part_cols ? k * (c->pair_grid / 2) : part_cols;
   }
   CAI_ALLOC(c->part, float4, static_cast<size_t>(c->rows_cap) * part_cols)
   if (c->use_pair) {
@@ -821,6 +857,10 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   std::memset(c->hf_host, 0, sizeof(HostFlag));
   if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB) ||
       (c->use_pair && !make_map(&c->tm_a, c->hc, c->rows_cap, cfg->H, kPairHalf)) ||
+      (c->swap_max_n && !make_map(&c->tm_rows.box[0], c->hc, c->rows_cap, cfg->H, 128)) ||
+      (c->swap_max_n && !make_map(&c->tm_rows.box[1], c->hc, c->rows_cap, cfg->H, 64)) ||
+      (c->swap_max_n && !make_map(&c->tm_rows.box[2], c->hc, c->rows_cap, cfg->H, 32)) ||
+      (c->swap_max_n && !make_map(&c->tm_rows.box[3], c->hc, c->rows_cap, cfg->H, 16)) ||
       (c->use_pair &&
        !make_map(&c->tm_w, c->wt, static_cast<uint64_t>(2 * c->n_vt) * (cfg->H / kPairBlockK) *
                                       kPairHalf,
@@ -850,7 +890,12 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   c->stats.grid = c->G;
   c->stats.stages = c->n_stages;
   c->stats.n_max = c->n_max;
-  c->stats.kernels_per_step = c->fused ? 1 : c->use_pair ? 5 : 3;
+  c->stats.pair_grid = c->use_pair ? c->pair_grid : 0;
+  c->stats.pair_swap_max_n = c->swap_max_n;
+  c->stats.pair_stages = c->use_pair ? c->pair_stages : 0;
+  c->stats.kernels_per_step =
+      c->fused ? 1
+               : 2 + (c->head_in_step ? 1 : 0) + (c->use_pair ? 1 : 0) + (c->need_reduce ? 1 : 0);
   r = cai_reset(c, stream);
   if (r != CAI_OK) {
     release(c);

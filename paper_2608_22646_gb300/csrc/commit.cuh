@@ -66,6 +66,7 @@ struct CommitParams {
   const float4* rowres;   // [rows] merged triple per row when the pair kernel decoded the step
   int pair_min_M;         // steps with at least this many rows ran the pair kernel
   int pair_pairs;         // pairs of the pair kernel's grid
+  int pair_swap_max_n;    // the pair kernel's orientation rule (pair_swapped)
   int identity_rows;      // 1: row of (b, p) is b P + p; 0: row_of[b P + p]
   StateArrays st;
   int* list;

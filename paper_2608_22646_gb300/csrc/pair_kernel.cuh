@@ -29,6 +29,22 @@
 // and by the n_rt pairs of its row tiles from L2; the gathered hidden rows
 // (at most 2 x 65536 x 16384 bytes, in practice tens of MB) stay in L2.
 //
+// Swapped orientation (chosen per step, pair_swapped): the vocabulary fills the MMA M dimension (256
+// rows per pair, 128 per CTA: the W half is the A operand) and the masked rows
+// the N dimension.  The M rows are split into n_rt = ceil(M / 256) row tiles
+// of equal width N (a multiple of 32, at most 256), so a step pads at most 31
+// rows per tile instead of up to 255: M = 305 runs as two 160-column tiles,
+// M = 159 as one of 160.  A tensor-memory lane then holds one vocabulary row
+// of every column; the epilogue reduces across lanes (transpose_merge32) and
+// across the four epilogue warps (a shared-memory exchange), and each CTA
+// writes the triples of its 128 vocabulary rows: two partials per pair.  Each
+// CTA loads N / 2 of a tile's rows per K block (16-row boxes), so a narrow
+// tile also moves fewer bytes through shared memory.  The cross-lane
+// reduction costs more instructions than the unswapped epilogue, so full-width
+// tiles stay unswapped: a step runs swapped when its tile width N is at most
+// swap_max_n (192 by default; measured, Dream shape: N = 64..192 5 % faster
+// than the padded unswapped tile, N = 224, 256 4 to 8 % slower).
+//
 // Roles per CTA (192 threads): warp 0 producer (hidden half and W half, each
 // one TMA box; W from a tile-major packed copy in which every box is one
 // contiguous 16 KiB block); warp 1 allocates tensor memory and, in the even
@@ -53,6 +69,16 @@ constexpr int kPairBlockK = 64;       // K per stage (one 128-byte swizzled row)
 constexpr int kPairHalfBytes = kPairHalf * kPairBlockK * 2;  // 16 KiB
 constexpr int kPairStageBytes = 2 * kPairHalfBytes;          // A half + B half
 constexpr int kPairTmemCols = 2 * kPairTileVocab;            // two accumulators
+constexpr int kSwapColStep = 32;    // swapped orientation: granularity of N
+constexpr int kSwapXchBytes = 2 * 4 * kPairTileVocab * 16;  // cross-warp exchange, two buffers
+
+// Tensor maps of the gathered rows with boxes of 128, 64, 32 and 16 rows
+// (swapped orientation: a CTA's N / 2 rows of a tile, a multiple of 16 up to
+// 128, load as at most four boxes, the binary digits of N / 32; TMA copies
+// of many small boxes cost more than the bytes they move).
+struct PairRowMaps {
+  CUtensorMap box[4];  // box[q]: 128 >> q rows
+};
 
 struct PairParams {
   const int* d_M;      // masked rows of this step (device)
@@ -61,22 +87,44 @@ struct PairParams {
   uint32_t* err;
   int V, H;
   int n_vt;            // ceil(V / 256)
-  int min_M;           // smaller steps are left to lm_head_softmax_kernel
+  int min_M;           // smaller steps are left to lm_head_softmax_kernel (<= 1: this
+                       // kernel decodes every step and records M = 0 too)
+  int swap_max_n;      // steps whose swapped tile width is at most this run swapped
   int n_stages;
   const float* inv_r;  // final-norm row scales [rows] (kNorm only)
 };
 
-// Partials per row written by a pair step with M rows on n_pairs pairs: one
-// per pair of the row's tile when n_pairs is a multiple of the row-tile
-// count, else 0 (one per vocabulary tile, to be merged by the reduce kernel).
-__host__ __device__ inline int pair_partials_per_row(int M, int n_pairs) {
-  const int n_rt = (M + kPairTileRows - 1) / kPairTileRows;
-  return (n_rt > 0 && n_pairs % n_rt == 0) ? n_pairs / n_rt : 0;
+// Row tiles of a pair step with M rows (both orientations).
+__host__ __device__ inline int pair_row_tiles(int M) {
+  return (M + kPairTileRows - 1) / kPairTileRows;
 }
 
-__host__ __device__ inline size_t pair_smem_bytes(int n_stages) {
-  return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes +
-         static_cast<size_t>(2 * n_stages + 5) * 8 + 16;
+// Swapped orientation: width N of each of the n_rt row tiles; tile j covers
+// rows [j N, j N + N), the last one possibly past M (padding, never written).
+__host__ __device__ inline int swap_tile_cols(int M, int n_rt) {
+  const int per = (M + n_rt - 1) / n_rt;
+  return (per + kSwapColStep - 1) / kSwapColStep * kSwapColStep;
+}
+
+// Orientation of a pair step with M rows: swapped when the tile width of the
+// swapped orientation is at most swap_max_n (0: never).
+__host__ __device__ inline bool pair_swapped(int M, int swap_max_n) {
+  return M > 0 && swap_tile_cols(M, pair_row_tiles(M)) <= swap_max_n;
+}
+
+// Partials per row written by a pair step with M rows on n_pairs pairs: one
+// per pair of the row's tile (two in the swapped orientation, one per CTA)
+// when n_pairs is a multiple of the row-tile count, else 0 (one per
+// vocabulary tile, two when swapped, merged by the reduce kernel).
+__host__ __device__ inline int pair_partials_per_row(int M, int n_pairs, bool swap) {
+  const int n_rt = pair_row_tiles(M);
+  if (n_rt <= 0 || n_pairs % n_rt != 0) return 0;
+  return (swap ? 2 : 1) * (n_pairs / n_rt);
+}
+
+__host__ __device__ inline size_t pair_smem_bytes(int n_stages, bool swap) {
+  return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes + (swap ? kSwapXchBytes : 0) +
+         static_cast<size_t>(2 * n_stages + 7) * 8 + 16;
 }
 
 // Pack W [V, H] (row-major bf16) tile-major for the pair kernel: 128-row
@@ -107,26 +155,32 @@ __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restri
 
 struct PairSmem {
   uint8_t* stage;      // n_stages x (A half, B half)
+  float4* xch;         // swapped orientation: 2 x [4 warps][256 columns] triples
   uint64_t* full;      // n_stages (even CTA): both CTAs' halves of the stage landed
   uint64_t* empty;     // n_stages: the pair's MMAs are done with the stage
   uint64_t* accf;      // 2: accumulator ready
   uint64_t* acce;      // 2 (even CTA): accumulator drained by both epilogues
   uint64_t* drain;     // 1 (even CTA): abort path, issued MMAs complete
+  uint64_t* xchb;      // 2 (swapped): the four epilogue warps wrote xch[buffer]
   uint32_t* tmem_slot;
   volatile int* abort;
 };
 
-__device__ __forceinline__ PairSmem pair_carve(uint8_t* raw, int n_stages) {
+__device__ __forceinline__ PairSmem pair_carve(uint8_t* raw, int n_stages, bool swap) {
   PairSmem s;
   uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(raw) + 1023) &
                                              ~static_cast<uintptr_t>(1023));
   s.stage = base;
-  s.full = reinterpret_cast<uint64_t*>(base + static_cast<size_t>(n_stages) * kPairStageBytes);
+  uint8_t* after = base + static_cast<size_t>(n_stages) * kPairStageBytes;
+  s.xch = reinterpret_cast<float4*>(after);
+  if (swap) after += kSwapXchBytes;
+  s.full = reinterpret_cast<uint64_t*>(after);
   s.empty = s.full + n_stages;
   s.accf = s.empty + n_stages;
   s.acce = s.accf + 2;
   s.drain = s.acce + 2;
-  s.tmem_slot = reinterpret_cast<uint32_t*>(s.drain + 1);
+  s.xchb = s.drain + 1;
+  s.tmem_slot = reinterpret_cast<uint32_t*>(s.xchb + 2);
   s.abort = reinterpret_cast<volatile int*>(s.tmem_slot + 1);
   return s;
 }
@@ -153,11 +207,13 @@ __device__ __forceinline__ void pair_drain(uint64_t* bar, uint32_t parity, uint3
 }
 
 // kNorm: as in lm_head_softmax_kernel, row n's logits are scaled by inv_r[n]
-// (written by the gather).
+// (written by the gather).  Swapped steps (pair_swapped) load a tile's rows
+// through hm instead of tm_a.
 template <bool kNorm>
 __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
     lm_head_pair_kernel(const __grid_constant__ CUtensorMap tm_a,
-                        const __grid_constant__ CUtensorMap tm_w, const PairParams p) {
+                        const __grid_constant__ CUtensorMap tm_w,
+                        const __grid_constant__ PairRowMaps hm, const PairParams p) {
   extern __shared__ uint8_t smem_raw[];
   const int warp = threadIdx.x >> 5;
   const int lane = threadIdx.x & 31;
@@ -168,12 +224,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // d_M and the gathered rows of this step
   const int M = *p.d_M;
-  if (M < p.min_M) return;  // both CTAs of every pair take the same branch
-  if (p.m_hist_slot && blockIdx.x == 0 && threadIdx.x == 0) *p.m_hist_slot = M;
+  if (p.m_hist_slot && blockIdx.x == 0 && threadIdx.x == 0 && (M >= p.min_M || p.min_M <= 1))
+    *p.m_hist_slot = M;
+  if (M < p.min_M || M < 1) return;  // both CTAs of every pair take the same branch
+  const bool swap = pair_swapped(M, p.swap_max_n);  // the same in every CTA
 
-  PairSmem sm = pair_carve(smem_raw, p.n_stages);
+  PairSmem sm = pair_carve(smem_raw, p.n_stages, p.swap_max_n > 0);
   const int KB = p.H / kPairBlockK;
-  const int n_rt = (M + kPairTileRows - 1) / kPairTileRows;
+  const int n_rt = pair_row_tiles(M);
+  // Rows per row tile: 256 (the MMA M of the pair), or N when swapped.
+  const int rt_rows = swap ? swap_tile_cols(M, n_rt) : kPairTileRows;
   const int n_tiles = p.n_vt * n_rt;
   const int my_tiles = pair < n_tiles ? (n_tiles - pair + n_pairs - 1) / n_pairs : 0;
 
@@ -187,12 +247,20 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       mbar_init(&sm.acce[a], 8);  // four epilogue warps in each CTA
     }
     mbar_init(sm.drain, 1);
+    if (swap) {
+      mbar_init(&sm.xchb[0], 4);  // the four epilogue warps of this CTA
+      mbar_init(&sm.xchb[1], 4);
+    }
     *sm.abort = 0;
     fence_mbar_init();
   }
   if (warp == 0 && lane == 0) {
-    prefetch_tmap(&tm_a);
     prefetch_tmap(&tm_w);
+    if (swap) {
+      for (int q = 0; q < 4; ++q) prefetch_tmap(&hm.box[q]);
+    } else {
+      prefetch_tmap(&tm_a);
+    }
   }
   if (warp == 1) {
     tmem_alloc_pair(sm.tmem_slot, kPairTmemCols);
@@ -211,10 +279,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       PairRing r;
       long long issued = 0;
       bool ok = true;
+      // Bytes of one stage, both CTAs (the even CTA arms its barrier for them).
+      const uint32_t stage_tx =
+          swap ? 2u * static_cast<uint32_t>(kPairHalfBytes + (rt_rows / 2) * kPairBlockK * 2)
+                : 2u * kPairStageBytes;
       for (int i = 0; i < my_tiles && ok; ++i) {
         const int t = pair + i * n_pairs;
         const int v = t / n_rt, j = t - v * n_rt;
-        const int a_row = j * kPairTileRows + static_cast<int>(rank) * kPairHalf;
+        // First row of this CTA's half of the tile's rows.
+        const int a_row = j * rt_rows + static_cast<int>(rank) * (swap ? rt_rows / 2 : kPairHalf);
         const int w_box = (2 * v + static_cast<int>(rank)) * KB;
         for (int kb = 0; kb < KB; ++kb) {
           if (!mbar_wait(&sm.empty[r.slot], r.phase ^ 1u, sm.abort, p.err, kErrWaitEmpty)) {
@@ -225,9 +298,25 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
           const uint32_t bar = full0 + static_cast<uint32_t>(r.slot * 8);
           // The even CTA arms the stage for the bytes of both CTAs; a copy of
           // the odd CTA that completes first leaves the phase open until then.
-          if (rank == 0) mbar_arrive_expect_tx(&sm.full[r.slot], 2 * kPairStageBytes);
-          tma_load_2d_pair(dst, &tm_a, bar, kb * kPairBlockK, a_row, pol_a);
-          tma_load_2d_pair_nohint(dst + kPairHalfBytes, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
+          if (rank == 0) mbar_arrive_expect_tx(&sm.full[r.slot], stage_tx);
+          if (swap) {
+            // A: the W half; B: rt_rows / 2 gathered rows (a multiple of 16,
+            // at most 128) as boxes of 128, 64, 32, 16 rows.
+            tma_load_2d_pair_nohint(dst, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
+            int off = 0;
+#pragma unroll
+            for (int q = 0; q < 4; ++q) {
+              const int rows = kPairHalf >> q;
+              if ((rt_rows / 2) & rows) {
+                tma_load_2d_pair(dst + kPairHalfBytes + off * (kPairBlockK * 2), &hm.box[q], bar,
+                                 kb * kPairBlockK, a_row + off, pol_a);
+                off += rows;
+              }
+            }
+          } else {
+            tma_load_2d_pair(dst, &tm_a, bar, kb * kPairBlockK, a_row, pol_a);
+            tma_load_2d_pair_nohint(dst + kPairHalfBytes, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
+          }
           ++issued;
           r.next(p.n_stages);
         }
@@ -242,7 +331,10 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   } else if (warp == 1) {
     if (lane == 0 && rank == 0) {
       // -------------------------------------------- MMA issuer (even CTA) --
-      const uint32_t idesc = idesc_bf16_f32(kPairTileRows, kPairTileVocab);
+      // Swapped: M = 256 vocabulary rows, N = the tile's rows; else M = 256
+      // rows, N = 256 vocabulary rows.
+      const uint32_t idesc =
+          idesc_bf16_f32(256, swap ? static_cast<uint32_t>(rt_rows) : kPairTileVocab);
       PairRing r;
       bool ok = true;
       for (int i = 0; i < my_tiles && ok; ++i) {
@@ -280,12 +372,106 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       }
     }
     __syncwarp();
+  } else if (swap) {
+    // ----------------------------------------------- epilogue (swapped) --
+    // Lane l of warp `quarter` holds vocabulary row 256 v + 128 rank + 32
+    // quarter + l of all rt_rows columns (the tile's rows).  Per 32 columns the
+    // warp's 32 rows are merged across lanes (lane l then holds column l), the
+    // four warps' slices through xch, and thread et of the four warps keeps
+    // columns et and et + 128.
+    const int quarter = warp & 3;  // tensor-memory lanes 32 quarter .. 32 quarter + 31
+    const int ew = warp - 2;       // 0..3: slot in the cross-warp exchange
+    const int et = ew * 32 + lane;
+    const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+    const uint32_t acce_remote = mapa_shared(sm.acce, 0);
+    const int per_row = pair_partials_per_row(M, n_pairs, true);  // > 0: two partials per pair
+    const int nch = rt_rows / 32;
+    float am[2] = {kNegBig, kNegBig}, as[2] = {0.0f, 0.0f};
+    int aix[2] = {INT_MAX, INT_MAX};
+    for (int i = 0; i < my_tiles; ++i) {
+      const int t = pair + i * n_pairs;
+      const int v = t / n_rt, j = t - v * n_rt;
+      const int acc = i & 1;
+      if (!mbar_wait(&sm.accf[acc], (i >> 1) & 1, sm.abort, p.err, kErrWaitAccFull)) break;
+      tc_fence_after();
+      const uint32_t tbase = tmem_base + lane_base + static_cast<uint32_t>(acc * kPairTileVocab);
+      const int vrow = v * kPairTileVocab + static_cast<int>(rank) * kPairHalf + quarter * 32 + lane;
+      const bool valid = vrow < p.V;  // vocabulary rows past V are zero padding
+      const bool pvalid = (vrow ^ 16) < p.V;
+      const int row0 = j * rt_rows;
+      // Buffer i & 1 is written again at tile i + 2, after every warp has
+      // arrived for tile i + 1, which each does after reading tile i.  One
+      // chunk of 32 columns at a time (the reduction is not unrolled over
+      // chunks: its code stays small enough for the instruction cache).
+      float4* xb = sm.xch + (i & 1) * 4 * kPairTileVocab;
+#pragma unroll 1
+      for (int c = 0; c < nch; ++c) {
+        uint32_t x[32];
+        tmem_ld_32cols(tbase + static_cast<uint32_t>(32 * c), x);
+        tmem_ld_wait();
+        float z[32];
+#pragma unroll
+        for (int k = 0; k < 32; ++k) {
+          float sc = kLog2e;
+          if constexpr (kNorm) {
+            const int row = row0 + 32 * c + k;
+            if (row < M) sc = kLog2e * __ldg(p.inv_r + row);
+          }
+          z[k] = valid ? __uint_as_float(x[k]) * sc : kNegBig;
+        }
+        float m, s;
+        int ix;
+        transpose_logits32(z, valid, pvalid, vrow, lane, m, s, ix);
+        xb[ew * kPairTileVocab + 32 * c + lane] = make_float4(m, s, __int_as_float(ix), 0.0f);
+      }
+      tc_fence_before();
+      __syncwarp();
+      if (lane == 0) {
+        if (rank == 0)
+          mbar_arrive(&sm.acce[acc]);
+        else
+          mbar_arrive_cluster(acce_remote + static_cast<uint32_t>(acc * 8));
+      }
+      if (lane == 0) mbar_arrive(&sm.xchb[i & 1]);
+      if (!mbar_wait(&sm.xchb[i & 1], (i >> 1) & 1, sm.abort, p.err, kErrWaitEpi)) break;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int col = et + 128 * h;
+        if (col < rt_rows) {
+          float m = kNegBig, s = 0.0f;
+          int ix = INT_MAX;
+#pragma unroll
+          for (int w = 0; w < 4; ++w) {
+            const float4 a = xb[w * kPairTileVocab + col];
+            merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+          }
+          const int row = row0 + col;
+          if (per_row > 0)
+            merge_tri(am[h], as[h], aix[h], m, s, ix);
+          else if (row < M && CAI_IN_RANGE(v < p.n_vt, p.err))
+            p.part[static_cast<size_t>(row) * (2 * p.n_vt) + 2 * v + static_cast<int>(rank)] =
+                make_float4(m, s, __int_as_float(ix), 0.0f);
+        }
+      }
+    }
+    if (per_row > 0) {
+      // The pair's row tile is fixed (pair mod n_rt); a pair without tiles
+      // writes the empty triple.
+      const int row0 = (pair % n_rt) * rt_rows;
+#pragma unroll
+      for (int h = 0; h < 2; ++h) {
+        const int col = et + 128 * h;
+        if (col < rt_rows && row0 + col < M)
+          p.part[static_cast<size_t>(row0 + col) * per_row + 2 * (pair / n_rt) +
+                 static_cast<int>(rank)] = make_float4(am[h], as[h], __int_as_float(aix[h]), 0.0f);
+      }
+    }
   } else {
     // --------------------------------------------------------- epilogue --
     const int quarter = warp & 3;  // tensor-memory lanes 32 quarter .. 32 quarter + 31
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
     const uint32_t acce_remote = mapa_shared(sm.acce, 0);
-    const int per_row = pair_partials_per_row(M, n_pairs);  // > 0: one partial per pair
+    const int per_row = pair_partials_per_row(M, n_pairs, false);  // > 0: one partial per pair
     float am = kNegBig, as = 0.0f;
     int aix = INT_MAX;
     for (int i = 0; i < my_tiles; ++i) {
@@ -371,13 +557,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
 // maxima) into one triple, rowres[row], so that the commit reads one value per
 // row.  Returns at once when the step ran on the swapped-operand kernel.
 struct ReduceParams {
-  const float4* part;  // [rows, n_part]
+  const float4* part;  // [rows, n_vt] partials (unswapped step), [rows, 2 n_vt] (swapped)
   float4* rowres;      // [rows]
   const int* d_M;
-  int n_part;
+  int n_vt;
   int min_M;
   int n_pairs;         // the pair kernel's grid / 2 (its partials need no merge when
                        // pair_partials_per_row > 0)
+  int swap_max_n;      // the pair kernel's orientation rule (pair_swapped)
 };
 
 constexpr int kReduceThreads = 256;
@@ -386,15 +573,17 @@ __global__ void __launch_bounds__(kReduceThreads) reduce_partials_kernel(const R
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // the pair kernel's partials
   const int M = *p.d_M;
-  if (M < p.min_M || pair_partials_per_row(M, p.n_pairs) > 0) return;
+  const bool swap = pair_swapped(M, p.swap_max_n);
+  if (M < p.min_M || M < 1 || pair_partials_per_row(M, p.n_pairs, swap) > 0) return;
+  const int n_part = (swap ? 2 : 1) * p.n_vt;
   const int lane = threadIdx.x & 31;
   const int nw = (gridDim.x * blockDim.x) >> 5;
   for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < M; row += nw) {
-    const float4* pr = p.part + static_cast<size_t>(row) * p.n_part;
+    const float4* pr = p.part + static_cast<size_t>(row) * n_part;
     float m = kNegBig, s = 0.0f;
     int ix = INT_MAX;
     int k = lane;
-    for (; k + 96 < p.n_part; k += 128) {  // four loads in flight per lane
+    for (; k + 96 < n_part; k += 128) {  // four loads in flight per lane
       const float4 a = __ldcg(pr + k), b = __ldcg(pr + k + 32), c = __ldcg(pr + k + 64),
                    d = __ldcg(pr + k + 96);
       merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
@@ -402,7 +591,7 @@ __global__ void __launch_bounds__(kReduceThreads) reduce_partials_kernel(const R
       merge_tri(m, s, ix, c.x, c.y, __float_as_int(c.z));
       merge_tri(m, s, ix, d.x, d.y, __float_as_int(d.z));
     }
-    for (; k < p.n_part; k += 32) {
+    for (; k < n_part; k += 32) {
       const float4 a = __ldcg(pr + k);
       merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
     }

@@ -60,6 +60,59 @@ __device__ __forceinline__ void transpose_merge32(float (&m)[32], float (&s)[32]
   }
 }
 
+// 32 rows (one per lane) x 32 columns of logits z (log2 units) -> lane l
+// holds the (max, sum, argmax) of column l over the 32 rows, as
+// transpose_merge32 but with the first halving step specialised: a lane's
+// partner at width 16 holds vocabulary row vrow ^ 16, so only the logits are
+// exchanged (16 shuffles instead of 48).  vrow is this lane's vocabulary row
+// (lane-aligned: vrow % 32 == lane), valid / pvalid whether this lane's and
+// the partner's rows exist.  On return m[0], s[0], ix[0] hold the column's
+// triple; z is clobbered.
+__device__ __forceinline__ void transpose_logits32(float (&z)[32], bool valid, bool pvalid,
+                                                   int vrow, int lane, float& om, float& os,
+                                                   int& oi) {
+  float m[16], s[16];
+  int ix[16];
+  const bool up = (lane & 16) != 0;
+  const float ks = valid ? 1.0f : 0.0f, rs = pvalid ? 1.0f : 0.0f;
+  const int ki = valid ? vrow : INT_MAX, ri = pvalid ? (vrow ^ 16) : INT_MAX;
+#pragma unroll
+  for (int c = 0; c < 16; ++c) {
+    const float keep = up ? z[c + 16] : z[c];
+    const float send = up ? z[c] : z[c + 16];
+    const float rm = __shfl_xor_sync(0xffffffffu, send, 16);
+    float km = keep, kss = ks;
+    int kii = ki;
+    merge_tri(km, kss, kii, rm, rs, ri);
+    m[c] = km;
+    s[c] = kss;
+    ix[c] = kii;
+  }
+#pragma unroll
+  for (int w = 8; w >= 1; w >>= 1) {
+    const bool hi = (lane & w) != 0;
+#pragma unroll
+    for (int c = 0; c < w; ++c) {
+      float km = hi ? m[c + w] : m[c];
+      float kss = hi ? s[c + w] : s[c];
+      int kii = hi ? ix[c + w] : ix[c];
+      const float sm = hi ? m[c] : m[c + w];
+      const float ss = hi ? s[c] : s[c + w];
+      const int si = hi ? ix[c] : ix[c + w];
+      const float rm = __shfl_xor_sync(0xffffffffu, sm, w);
+      const float rss = __shfl_xor_sync(0xffffffffu, ss, w);
+      const int rii = __shfl_xor_sync(0xffffffffu, si, w);
+      merge_tri(km, kss, kii, rm, rss, rii);
+      m[c] = km;
+      s[c] = kss;
+      ix[c] = kii;
+    }
+  }
+  om = m[0];
+  os = s[0];
+  oi = ix[0];
+}
+
 // 32 rows (one per lane) x 32 columns of logits -> lane l holds the
 // (max, sum, argmax) of column l over the 32 rows.  Column c's logits are
 // scaled by log2 e, times col_scale[c] when given (a per-row normalisation

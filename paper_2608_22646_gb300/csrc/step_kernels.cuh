@@ -206,7 +206,8 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
   // partials were already merged into one triple per row.
   const int M = *p.d_M;
   if (M >= p.pair_min_M) {
-    const int per_row = pair_partials_per_row(M, p.pair_pairs);
+    const int per_row =
+        pair_partials_per_row(M, p.pair_pairs, pair_swapped(M, p.pair_swap_max_n));
     if (per_row > 0)
       merge_commit_sequence(p, blockIdx.x, cs, p.part, per_row);
     else

@@ -261,22 +261,79 @@ def test_all_commit_at_step_zero_and_noop_steps():
         cai.cai_free(ctx)
 
 
-@pytest.mark.parametrize("pair", ["1", "0"])
-def test_pair_kernel_steps(pair, monkeypatch):
-    # B P = 320 > 256: multi-kernel steps.  Steps with >= 32 masked rows run
-    # on the CTA-pair LM head (ragged vocabulary tail, two row tiles of 256,
-    # the second mostly padding), smaller ones on the swapped-operand kernel;
+def _expected_kernels(st, rows_cap):
+    """Launches per multi-kernel step: gather, merge + commit, the LM head(s),
+    and the row merge when some step size leaves per-tile partials."""
+    if not st["pair_grid"]:
+        return 3
+    pairs = st["pair_grid"] // 2
+    reduce = any(pairs % rt for rt in range(1, -(-rows_cap // 256) + 1))
+    head = st["pair_swap_max_n"] < 32  # the swapped-operand kernel takes M < 32
+    return 2 + (1 if head else 0) + 1 + (1 if reduce else 0)
+
+
+@pytest.mark.parametrize("pair,swap,max_n", [("1", "1", None), ("1", "1", "256"),
+                                             ("1", "0", None), ("0", "1", None)])
+def test_pair_kernel_steps(pair, swap, max_n, monkeypatch):
+    # B P = 320 > 256: multi-kernel steps.  The pair kernel decodes every step,
+    # swapped while the tile width is at most 192 (default; 256: always):
+    # two row tiles of 160 at M = 320, one narrowing tile below 192 rows, the
+    # unswapped 256-row tile in between.  CAI_PAIR_SWAP=0: steps with >= 32
+    # masked rows run on the unswapped pair kernel (two 256-row tiles, the
+    # second mostly padding), smaller ones on the swapped-operand kernel;
     # CAI_PAIR=0 keeps every step on the latter.
     monkeypatch.setenv("CAI_PAIR", pair)
+    monkeypatch.setenv("CAI_PAIR_SWAP", swap)
+    if max_n:
+        monkeypatch.setenv("CAI_PAIR_SWAP_MAX_N", max_n)
     B, P, H, V, T, nb = 5, 64, 256, 8000, 10, 2
     wl = synth.Workload("pairsteps", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
     ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
     hs = synth.HiddenStates(wl, W, "calibrated", seed=17)
     try:
-        assert cai.cai_get_stats(ctx)["kernels_per_step"] == (5 if pair == "1" else 3)
+        st = cai.cai_get_stats(ctx)
+        want = (int(max_n or 192) if swap == "1" else 0) if pair == "1" else 0
+        assert st["pair_swap_max_n"] == want
+        assert st["kernels_per_step"] == _expected_kernels(st, B * P)
         rep, final = parity.run_checked_trajectory(ctx, W, hs)
         st = cai.cai_state_download(ctx)
         assert int(st["m_hist"].max()) >= 128   # the pair kernel decoded some steps
+    finally:
+        cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("clusters,max_n,shape", [
+    # (pairs, widest swapped tile, (B, P, H, V, T, n_blocks)).  3 pairs: M in
+    # (256, 512] has two row tiles, not a divisor of 3, so partials are written
+    # per vocabulary tile (and CTA, swapped) and merged by the reduce kernel;
+    # M <= 256 and M in (512, 768] keep one partial per pair (and CTA).
+    # V % 256 = 184: the odd CTA's half of the last vocabulary tile is partly
+    # past V; V % 256 = 84: entirely past V.  H = 64: a single K block.
+    # max_n 256: every step swapped; 0: none; 192: both kinds in one
+    # trajectory (M = 576: three 192-wide tiles swapped, M ~ 400 unswapped).
+    (3, "256", (9, 64, 128, 3000, 10, 1)),
+    (3, "0", (9, 64, 128, 3000, 10, 1)),
+    (3, "192", (9, 64, 128, 3000, 10, 1)),
+    (2, "256", (9, 64, 64, 2900, 8, 1)),
+    (1, "256", (6, 50, 192, 4100, 8, 2)),
+    (1, "192", (6, 50, 192, 4100, 8, 2)),
+])
+def test_pair_partial_layouts(clusters, max_n, shape, monkeypatch):
+    monkeypatch.setenv("CAI_PAIR_CLUSTERS", str(clusters))
+    if max_n == "0":
+        monkeypatch.setenv("CAI_PAIR_SWAP", "0")
+    else:
+        monkeypatch.setenv("CAI_PAIR_SWAP_MAX_N", max_n)
+    B, P, H, V, T, nb = shape
+    wl = synth.Workload("swaplayouts", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=23)
+    try:
+        st = cai.cai_get_stats(ctx)
+        assert st["pair_grid"] == 2 * clusters and st["pair_swap_max_n"] == int(max_n)
+        assert st["kernels_per_step"] == _expected_kernels(st, B * P)
+        rep, _ = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P
     finally:
         cai.cai_free(ctx)
 
@@ -509,8 +566,8 @@ def test_debug_build_range_checks_stay_quiet():
 def test_long_dream_full_size_steps_sampled():
     # Long-generation Dream shape (B = 8, P = 64, H = 3584, V = 152064): the
     # first steps of block 0 run on the pair kernel with two row tiles and
-    # then one (per-pair partials), and the swapped-operand kernel once M < 32;
-    # at every step a sample of the rows it decoded is recomputed by the oracle.
+    # then one (per-pair partials), down to narrow steps with M < 32; at every
+    # step a sample of the rows it decoded is recomputed by the oracle.
     wl = synth.WORKLOADS["dream_long"]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
     hs = synth.HiddenStates(wl, W, "calibrated")

@@ -697,7 +697,9 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
       return CAI_ERR_CUDA;
     }
     const size_t plimit = static_cast<size_t>(smem_optin) - pa.sharedSizeBytes;
-    int ps = 6;
+    // CAI_PAIR_STAGES caps the ring depth (tuning knob; results do not depend on it).
+    const int pcap = env_int("CAI_PAIR_STAGES");
+    int ps = pcap >= 2 && pcap < 6 ? pcap : 6;
     while (ps > 2 && pair_smem_bytes(ps, c->swap_max_n > 0) > plimit) --ps;
     c->pair_stages = ps;
     c->pair_smem = pair_smem_bytes(ps, c->swap_max_n > 0);

@@ -38,8 +38,8 @@
 // of every column; the epilogue reduces across lanes (transpose_merge32) and
 // across the four epilogue warps (a shared-memory exchange), and each CTA
 // writes the triples of its 128 vocabulary rows: two partials per pair.  Each
-// CTA loads N / 2 of a tile's rows per K block (16-row boxes), so a narrow
-// tile also moves fewer bytes through shared memory.  The cross-lane
+// CTA loads N / 2 of a tile's rows per K block (one box of the next power of
+// two rows).  The cross-lane
 // reduction costs more instructions than the unswapped epilogue, so full-width
 // tiles stay unswapped: a step runs swapped when its tile width N is at most
 // swap_max_n (192 by default; measured, Dream shape: N = 64..192 5 % faster
@@ -73,9 +73,9 @@ constexpr int kSwapColStep = 32;    // swapped orientation: granularity of N
 constexpr int kSwapXchBytes = 2 * 4 * kPairTileVocab * 16;  // cross-warp exchange, two buffers
 
 // Tensor maps of the gathered rows with boxes of 128, 64, 32 and 16 rows
-// (swapped orientation: a CTA's N / 2 rows of a tile, a multiple of 16 up to
-// 128, load as at most four boxes, the binary digits of N / 32; TMA copies
-// of many small boxes cost more than the bytes they move).
+// (swapped orientation: a CTA's N / 2 rows of a tile load as the smallest of
+// these boxes that holds them; each TMA copy has a fixed cost of the order
+// of a 16 KiB copy's transfer time, so one box beats several exact ones).
 struct PairRowMaps {
   CUtensorMap box[4];  // box[q]: 128 >> q rows
 };
@@ -279,9 +279,15 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       PairRing r;
       long long issued = 0;
       bool ok = true;
+      // Swapped: a CTA's rt_rows / 2 rows load as one box of the next power
+      // of two (16..128 rows; the MMA reads the first rt_rows / 2): one TMA
+      // copy instead of up to four costs less than the extra bytes from L2.
+      int q1 = 3;
+      while (q1 > 0 && (kPairHalf >> q1) < rt_rows / 2) --q1;
+      const int box_rows = kPairHalf >> q1;
       // Bytes of one stage, both CTAs (the even CTA arms its barrier for them).
       const uint32_t stage_tx =
-          swap ? 2u * static_cast<uint32_t>(kPairHalfBytes + (rt_rows / 2) * kPairBlockK * 2)
+          swap ? 2u * static_cast<uint32_t>(kPairHalfBytes + box_rows * kPairBlockK * 2)
                 : 2u * kPairStageBytes;
       for (int i = 0; i < my_tiles && ok; ++i) {
         const int t = pair + i * n_pairs;
@@ -300,19 +306,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
           // the odd CTA that completes first leaves the phase open until then.
           if (rank == 0) mbar_arrive_expect_tx(&sm.full[r.slot], stage_tx);
           if (swap) {
-            // A: the W half; B: rt_rows / 2 gathered rows (a multiple of 16,
-            // at most 128) as boxes of 128, 64, 32, 16 rows.
+            // A: the W half; B: the CTA's rows, one box of box_rows.
             tma_load_2d_pair_nohint(dst, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
-            int off = 0;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-              const int rows = kPairHalf >> q;
-              if ((rt_rows / 2) & rows) {
-                tma_load_2d_pair(dst + kPairHalfBytes + off * (kPairBlockK * 2), &hm.box[q], bar,
-                                 kb * kPairBlockK, a_row + off, pol_a);
-                off += rows;
-              }
-            }
+            tma_load_2d_pair(dst + kPairHalfBytes, &hm.box[q1], bar, kb * kPairBlockK, a_row, pol_a);
           } else {
             tma_load_2d_pair(dst, &tm_a, bar, kb * kPairBlockK, a_row, pol_a);
             tma_load_2d_pair_nohint(dst + kPairHalfBytes, &tm_w, bar, 0, (w_box + kb) * kPairHalf);

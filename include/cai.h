@@ -23,7 +23,7 @@
  * use programmatic dependent launch: each may be scheduled while the kernel
  * before it in the stream still runs, and waits for that kernel to complete
  * before touching anything it produces (setting CAI_PDL=0 in the environment
- * before cai_init launches them plainly instead).  With B P <= 64 a step is
+ * before cai_init launches them plainly instead).  With B P <= 32 a step is
  * one kernel: the LM head over every row of the block, whose last CTA applies
  * the commit rule; it streams W before the previous step has committed and
  * waits for it only to write its partials and to commit.  With B P > 64 a
@@ -188,7 +188,7 @@ typedef struct cai_stats {
   int32_t grid;             /* CTAs of the LM-head kernel                          */
   int32_t stages;           /* pipeline stages of the LM-head kernel               */
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
-  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 64); else gather,
+  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 32); else gather,
                                LM head(s), row merge if needed, commit (2 to 5)    */
   double step_ms;           /* summed device time of profiled steps, every kernel  */
   int32_t pair_grid;        /* CTAs of the CTA-pair LM head (0: not used)          */
@@ -206,7 +206,7 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
 /*
  * Create a context.  W is the LM-head weight [V, H] bf16, row-major, host or
  * device memory.  It is read once, during this call, into the library's
- * packed copies (2 V H bytes each: one copy when B P <= 64, two otherwise);
+ * packed copies (2 V H bytes each: one copy when B P <= 32, two otherwise);
  * the caller may free or change it afterwards.  All state starts at block 0,
  * t = 0, every token masked.  Allocates device memory and one page of mapped
  * pinned host memory.  Synchronous.
@@ -244,7 +244,7 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
  * Host pointer: with B P > 64 and page-locked, device-mapped memory (e.g.
  * cudaHostAlloc), the gather reads the masked rows in place over the host
  * link, on the stream (valid until the stream passes this call); otherwise
- * (pageable memory, or B P <= 64) the rows are copied to the device inside
+ * (pageable memory, or B P <= 32) the rows are copied to the device inside
  * the call.
  * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call
  * cai_block_advance or cai_reset first).

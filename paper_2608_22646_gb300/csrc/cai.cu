@@ -32,7 +32,7 @@ std::atomic<int> g_head_grid_limit{0};
 // Programmatic dependent launch between the step's kernels; CAI_PDL=0 in the
 // environment turns it off (read once per context at cai_init).
 // Largest B P that runs single-kernel steps by default.
-constexpr int kFusedMaxRows = 64;
+constexpr int kFusedMaxRows = 32;
 
 bool pdl_enabled() {
   const char* e = std::getenv("CAI_PDL");
@@ -207,7 +207,7 @@ struct cai_ctx {
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
   const void* hid_mapped = nullptr;
-  bool fused = false;    // single-kernel step (B P <= 64)
+  bool fused = false;    // single-kernel step (B P <= 32)
   int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
   int b_slot_bytes = 0;
   size_t head_smem = 0;
@@ -353,7 +353,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   return cp;
 }
 
-// One denoising step.  Single-kernel step (B P <= 64): the LM-head kernel
+// One denoising step.  Single-kernel step (B P <= 32): the LM-head kernel
 // reads the hidden states in place and its last CTA commits.  Otherwise:
 // gather -> LM head -> merge + commit.
 int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first);
@@ -602,10 +602,11 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   c->pdl = pdl_enabled();
   c->nvtx = nvtx_enabled();
   // Single-kernel steps decode every row of the block each step, through one
-  // N = B P chunk of the swapped-operand kernel: efficient up to 64 rows (full
-  // tile groups).  Larger batches run multi-kernel steps, whose pair kernel
-  // decodes only the masked rows (measured, LLaDA shape: B P = 128, 256 run at
-  // 0.60, 0.29 of the roofline single-kernel and 0.83, 0.80 multi-kernel).
+  // N = B P chunk of the swapped-operand kernel, and save the gather and
+  // commit launches.  Larger batches run multi-kernel steps, whose pair kernel
+  // decodes only the masked rows (measured, LLaDA shape, positions/s: B P = 32
+  // 92.3k single-kernel against 85.3k multi-kernel; B P = 64 161.9k against
+  // 168.0k; B P = 128, 256 ran at 0.60, 0.29 of the roofline single-kernel).
   // CAI_FUSED_MAX_BP overrides the limit (up to 256).
   const int fmax = env_int("CAI_FUSED_MAX_BP");
   c->fused = c->BP <= (fmax > 0 && fmax <= kChunkN ? fmax : kFusedMaxRows);

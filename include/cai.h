@@ -356,6 +356,17 @@ int cai_test_head_grid_limit(int32_t n);
  */
 int cai_test_check_guards(cai_ctx* ctx, int32_t* n_bad);
 
+/*
+ * Testing hook, host only (no device use): the CTA-pair LM head's plan for a
+ * step with M masked rows on n_pairs pairs whose widest swapped tile is
+ * swap_max_n (0: never swapped).  Writes out[0] = 1 if the step runs in the
+ * swapped orientation, out[1] = row tiles, out[2] = rows per row tile (the
+ * MMA N when swapped, 256 otherwise), out[3] = partials per row read by the
+ * commit (0: per-tile partials merged by the row-merge kernel).
+ * CAI_ERR_ARG for M < 1, n_pairs < 1, swap_max_n < 0 or out == NULL.
+ */
+int cai_test_pair_plan(int32_t M, int32_t n_pairs, int32_t swap_max_n, int32_t* out);
+
 #ifdef __cplusplus
 }
 #endif

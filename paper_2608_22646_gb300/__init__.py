@@ -52,6 +52,7 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
+           "cai_test_pair_plan",
            "cai_test_check_guards",
            "cai_head_rows_static")
 
@@ -122,6 +123,7 @@ def _load():
         "cai_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
         "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
+        "cai_test_pair_plan": (ctypes.c_int, [i32, i32, i32, ctypes.POINTER(i32)]),
         "cai_test_check_guards": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
         "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
     }
@@ -296,6 +298,13 @@ def cai_free(ctx: Ctx) -> None:
 
 def cai_test_fail_alloc_after(n: int) -> None:
     _check(lib().cai_test_fail_alloc_after(n), "cai_test_fail_alloc_after")
+
+
+def cai_test_pair_plan(M: int, n_pairs: int, swap_max_n: int) -> dict:
+    out = (ctypes.c_int32 * 4)()
+    _check(lib().cai_test_pair_plan(M, n_pairs, swap_max_n, out), "cai_test_pair_plan")
+    return {"swapped": bool(out[0]), "row_tiles": out[1], "tile_rows": out[2],
+            "partials_per_row": out[3]}
 
 
 def cai_test_head_grid_limit(n: int) -> None:

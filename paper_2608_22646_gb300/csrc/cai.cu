@@ -1195,6 +1195,17 @@ int cai_test_head_grid_limit(int32_t n) {
   return CAI_OK;
 }
 
+int cai_test_pair_plan(int32_t M, int32_t n_pairs, int32_t swap_max_n, int32_t* out) {
+  if (M < 1 || n_pairs < 1 || swap_max_n < 0 || !out) return CAI_ERR_ARG;
+  const bool swap = pair_swapped(M, swap_max_n);
+  const int n_rt = pair_row_tiles(M);
+  out[0] = swap ? 1 : 0;
+  out[1] = n_rt;
+  out[2] = swap ? swap_tile_cols(M, n_rt) : kPairTileRows;
+  out[3] = pair_partials_per_row(M, n_pairs, swap);
+  return CAI_OK;
+}
+
 int cai_test_fail_alloc_after(int32_t n) {
   if (n < 0) return CAI_ERR_ARG;
   g_fail_alloc_after.store(n);

@@ -134,3 +134,32 @@ def test_no_device_is_a_status_not_a_crash():
     h = ctypes.c_void_p()
     r = cai.lib().cai_init(ctypes.byref(c), ctypes.addressof(w), None, ctypes.byref(h))
     assert r in (cai.CAI_ERR_CUDA, cai.CAI_ERR_UNSUPPORTED) and not h.value
+
+
+@pytest.mark.parametrize("n_pairs", [76, 74, 3, 1])
+def test_pair_plan_covers_rows_with_bounded_padding(n_pairs):
+    # The pair LM head's per-step plan (host logic, no device): row tiles of
+    # at most 256 rows cover M; swapped tiles are equal, a multiple of 32
+    # wide, and pad fewer than 32 rows each; a step is swapped exactly when
+    # its tile would be at most swap_max_n wide; one partial per pair (and
+    # CTA when swapped) exactly when the row-tile count divides the pairs.
+    for max_n in (0, 32, 192, 256):
+        for M in range(1, 2049):
+            pl = cai.cai_test_pair_plan(M, n_pairs, max_n)
+            n_rt = -(-M // 256)
+            assert pl["row_tiles"] == n_rt
+            width = -(-(-(-M // n_rt)) // 32) * 32
+            assert 32 <= width <= 256 and n_rt * width >= M
+            assert n_rt * width - M < 32 * n_rt
+            assert pl["swapped"] == (max_n >= 32 and width <= max_n), (M, max_n)
+            assert pl["tile_rows"] == (width if pl["swapped"] else 256)
+            if pl["swapped"]:
+                assert pl["tile_rows"] * n_rt - M < 32 * n_rt
+            want = 0 if n_pairs % n_rt else (2 if pl["swapped"] else 1) * (n_pairs // n_rt)
+            assert pl["partials_per_row"] == want
+    lib = cai.lib()
+    out = (ctypes.c_int32 * 4)()
+    assert lib.cai_test_pair_plan(0, 76, 192, out) == cai.CAI_ERR_ARG
+    assert lib.cai_test_pair_plan(5, 0, 192, out) == cai.CAI_ERR_ARG
+    assert lib.cai_test_pair_plan(5, 76, -1, out) == cai.CAI_ERR_ARG
+    assert lib.cai_test_pair_plan(5, 76, 192, None) == cai.CAI_ERR_ARG

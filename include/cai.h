@@ -241,11 +241,15 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
  * hidden: the block's final hidden states [B, P, H] bf16, row-major; row
  * (b, p) is the one that predicts position p of the block.  Device pointer:
  * read on the stream, must stay valid until the stream passes this call.
- * Host pointer: with B P > 64 and page-locked, device-mapped memory (e.g.
+ * Host pointer: with B P > 32 and page-locked, device-mapped memory (e.g.
  * cudaHostAlloc), the gather reads the masked rows in place over the host
- * link, on the stream (valid until the stream passes this call); otherwise
- * (pageable memory, or B P <= 32) the rows are copied to the device inside
- * the call.
+ * link, on the stream (valid until the stream passes this call).  Otherwise
+ * the rows are copied to the device: with B P <= 32 on a stream of the
+ * context's own into one of two alternating device buffers, which the step
+ * waits for (so the copy for the next step can run during this one), with
+ * B P > 32 on the step's stream; page-locked memory must stay valid until
+ * the stream passes this call, pageable memory is staged by the CUDA runtime
+ * before the call returns.
  * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call
  * cai_block_advance or cai_reset first).
  */

@@ -207,6 +207,17 @@ struct cai_ctx {
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
   const void* hid_mapped = nullptr;
+  // Single-kernel steps on host rows: the rows are copied on copy_stream into
+  // stage2[step id & 1] (hidden_stage and a second buffer), and the step's
+  // stream waits only for that copy, so the copy of step t + 1 overlaps step
+  // t and no copy sits between two step kernels in the step's stream.  A
+  // buffer is refilled after the step that read it (ev_read) has finished.
+  void* stage2[2] = {nullptr, nullptr};
+  CUtensorMap tm_stage[2]{};
+  cudaStream_t copy_stream = nullptr;
+  cudaEvent_t ev_copied[2] = {nullptr, nullptr};
+  cudaEvent_t ev_read[2] = {nullptr, nullptr};
+  bool read_pending[2] = {false, false};
   bool fused = false;    // single-kernel step (B P <= 32)
   int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
   int b_slot_bytes = 0;
@@ -277,6 +288,13 @@ void release(cai_ctx* c) {
   c->hf_host = nullptr;
   for (cudaEvent_t e : c->ev_pool) cudaEventDestroy(e);
   c->ev_pool.clear();
+  for (int k = 0; k < 2; ++k) {
+    if (c->ev_copied[k]) cudaEventDestroy(c->ev_copied[k]);
+    if (c->ev_read[k]) cudaEventDestroy(c->ev_read[k]);
+    c->ev_copied[k] = c->ev_read[k] = nullptr;
+  }
+  if (c->copy_stream) cudaStreamDestroy(c->copy_stream);
+  c->copy_stream = nullptr;
 }
 
 // ---- threshold schedule (Boxes 3, 4, 6), double precision on the host ----
@@ -372,22 +390,36 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
   const cai_config& cfg = c->cfg;
   const void* hid = hidden;
+  const int64_t step_id = c->last_step_id + 1;
+  int stage_slot = -1;  // single-kernel step on host rows: stage2 buffer used
   if (!is_device_ptr(hidden)) {
     // Multi-kernel step on page-locked host rows: the gather reads the masked
     // rows in place over the host link (only they cross it).  Otherwise the
-    // rows are copied to the device first.
+    // rows are copied to the device first: single-kernel steps on the side
+    // stream (see stage2), multi-kernel steps in the step's stream.
     const void* mapped = c->fused ? nullptr : host_mapped_ptr(hidden);
+    const size_t bytes = static_cast<size_t>(c->BP) * cfg.H * 2;
     if (mapped) {
       hid = mapped;
+    } else if (c->fused) {
+      const int k = static_cast<int>(step_id & 1);
+      if ((c->read_pending[k] &&
+           cudaStreamWaitEvent(c->copy_stream, c->ev_read[k], 0) != cudaSuccess) ||
+          cudaMemcpyAsync(c->stage2[k], hidden, bytes, cudaMemcpyHostToDevice, c->copy_stream) !=
+              cudaSuccess ||
+          cudaEventRecord(c->ev_copied[k], c->copy_stream) != cudaSuccess ||
+          cudaStreamWaitEvent(stream, c->ev_copied[k], 0) != cudaSuccess)
+        return fail(c, CAI_ERR_CUDA);
+      hid = c->stage2[k];
+      stage_slot = k;
     } else {
-      if (cudaMemcpyAsync(c->hidden_stage, hidden, static_cast<size_t>(c->BP) * cfg.H * 2,
-                          cudaMemcpyHostToDevice, stream) != cudaSuccess)
+      if (cudaMemcpyAsync(c->hidden_stage, hidden, bytes, cudaMemcpyHostToDevice, stream) !=
+          cudaSuccess)
         return fail(c, CAI_ERR_CUDA);
       hid = c->hidden_stage;
     }
   }
   const int t = c->t_next;
-  const int64_t step_id = c->last_step_id + 1;
   cudaEvent_t ev[4] = {nullptr, nullptr, nullptr, nullptr};
   const bool diag = (cfg.flags & CAI_DIAGNOSTICS) != 0;
   if (c->profiling) {
@@ -436,7 +468,7 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       return check_launch(c);
     c->stats.launches++;
   } else {
-    if (hid != c->hid_mapped) {
+    if (stage_slot < 0 && hid != c->hid_mapped) {
       // The single-kernel step reads the caller's [B P, H] rows through TMA.
       if (!make_map(&c->tm_hid, hid, c->BP, cfg.H, kBoxRowsB)) return CAI_ERR_ARG;
       c->hid_mapped = hid;
@@ -481,10 +513,18 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   if (c->fused) hp.cp = cp;
   if (c->profiling) cudaEventRecord(ev[1], stream);
   if (c->head_in_step) {
-    if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream,
-                   c->fused ? c->tm_hid : c->tm_h, hp) != cudaSuccess)
+    const CUtensorMap& tm_rows =
+        !c->fused ? c->tm_h : stage_slot >= 0 ? c->tm_stage[stage_slot] : c->tm_hid;
+    if (launch_pdl(c->pdl, c->head_kernel, c->G, kHeadThreads, c->head_smem, stream, tm_rows,
+                   hp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
+    if (stage_slot >= 0) {
+      // stage2[stage_slot] may be refilled once this step's kernel is done.
+      if (cudaEventRecord(c->ev_read[stage_slot], stream) != cudaSuccess)
+        return fail(c, CAI_ERR_CUDA);
+      c->read_pending[stage_slot] = true;
+    }
   }
   if (c->use_pair) {
     // Only one of the two LM-head kernels decodes a step: the other reads
@@ -783,6 +823,10 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
     CAI_ALLOC(c->rowres, float4, c->rows_cap)
   }
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
+  if (c->fused) {
+    c->stage2[0] = c->hidden_stage;
+    CAI_ALLOC(c->stage2[1], uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
+  }
   CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   if (c->norm) {
     CAI_ALLOC(c->inv_r, float, c->rows_cap)
@@ -871,6 +915,20 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
     release(c);
     delete c;
     return CAI_ERR_CUDA;
+  }
+  if (c->fused) {
+    bool ok = make_map(&c->tm_stage[0], c->stage2[0], c->BP, cfg->H, kBoxRowsB) &&
+              make_map(&c->tm_stage[1], c->stage2[1], c->BP, cfg->H, kBoxRowsB) &&
+              cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking) == cudaSuccess;
+    for (int k = 0; ok && k < 2; ++k)
+      ok = cudaEventCreateWithFlags(&c->ev_copied[k], cudaEventDisableTiming) == cudaSuccess &&
+           cudaEventCreateWithFlags(&c->ev_read[k], cudaEventDisableTiming) == cudaSuccess;
+    if (!ok) {
+      cudaGetLastError();
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
   }
   // All step kernels ask for the same (largest) shared-memory carveout, so the
   // small gather and merge CTAs can be resident on an SM beside an LM-head

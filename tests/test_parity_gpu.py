@@ -377,8 +377,8 @@ def test_teacher_forced_random_states():
         cai.cai_free(ctx)
 
 
-@pytest.mark.parametrize("shape,host", [("toy", "pinned"), ("multi", "pinned"),
-                                        ("multi", "pageable")])
+@pytest.mark.parametrize("shape,host", [("toy", "pinned"), ("toy", "pageable"),
+                                        ("multi", "pinned"), ("multi", "pageable")])
 def test_host_hidden_and_host_weight_match_device(shape, host):
     # Host inputs: copied in the call (single-kernel steps, or pageable memory)
     # or, for multi-kernel steps on page-locked memory, read in place by the gather.
@@ -414,6 +414,48 @@ def test_host_hidden_and_host_weight_match_device(shape, host):
         cai.cai_read_tokens(a, out)
         torch.cuda.synchronize()
         assert np.array_equal(out.numpy(), sa["tok"])
+    finally:
+        cai.cai_free(a)
+        cai.cai_free(b)
+
+
+@pytest.mark.parametrize("B,host", [(1, "pinned"), (2, "pinned"), (2, "pageable"),
+                                    (5, "pinned")])
+def test_host_rows_pipelined_match_device(B, host):
+    # Whole trajectories issued back to back with no synchronisation between
+    # steps (a one-step-behind poll only), every step reading a different host
+    # buffer: single-kernel steps copy on the context's side stream into two
+    # alternating buffers while the previous step runs, multi-kernel steps
+    # (B = 5) read page-locked rows in place.  The states must equal those of
+    # the same trajectory on device inputs bit for bit.
+    P = 16 if B < 5 else 64
+    wl = _wl("toy", B=B, P=P, gen_len=4 * P)
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=29)
+    dev_in = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    host_in = [[(x.cpu().pin_memory() if host == "pinned" else x.cpu().clone()) for x in row]
+               for row in dev_in]
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    a = cai.cai_init(cfg, W)
+    b = cai.cai_init(cfg, W)
+    try:
+        for ctx, inp in ((a, dev_in), (b, host_in)):
+            for rep in range(2):
+                cai.cai_reset(ctx)
+                for blk in range(wl.n_blocks):
+                    if blk:
+                        cai.cai_block_advance(ctx)
+                    cai.cai_first_step(ctx, inp[blk][0])
+                    for t in range(1, wl.T):
+                        if t >= 2 and cai.cai_poll(ctx, 1, 60000):
+                            break
+                        cai.cai_denoise_step(ctx, inp[blk][t])
+            torch.cuda.synchronize()
+        sa, sb = cai.cai_state_download(a), cai.cai_state_download(b)
+        for k in ("tok", "conf", "cand", "cstep", "exit_reason", "exit_step", "m_hist"):
+            assert np.array_equal(sa[k], sb[k]), k
+        assert int(sa["m_hist"].sum()) > 0
+        assert cai.cai_test_check_guards(b) == 0
     finally:
         cai.cai_free(a)
         cai.cai_free(b)

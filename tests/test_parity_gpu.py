@@ -338,6 +338,31 @@ def test_pair_partial_layouts(clusters, max_n, shape, monkeypatch):
         cai.cai_free(ctx)
 
 
+@pytest.mark.parametrize("shape", [
+    # (B, P, H, V, T, n_blocks), all multi-kernel.  B P = 33: one over the
+    # single-kernel limit, a 64-wide swapped tile whose odd half runs past the
+    # 48-row buffer (TMA fills zeros).  V = 130: the odd CTA's vocabulary half
+    # holds 2 rows; V = 128: none.  B P = 287 (buffer 288): the first step's two
+    # 160-wide swapped tiles end at row 320.  B P = 400: the first steps run
+    # unswapped (224-wide tiles would be needed), later ones swapped.
+    (1, 33, 64, 130, 6, 2),
+    (3, 11, 128, 128, 6, 2),
+    (7, 41, 192, 777, 6, 1),
+    (2, 200, 64, 1000, 5, 1),
+])
+def test_multi_kernel_edge_shapes(shape):
+    B, P, H, V, T, nb = shape
+    wl = synth.Workload("edges", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=37)
+    try:
+        assert cai.cai_get_stats(ctx)["kernels_per_step"] > 1
+        rep, _ = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P
+    finally:
+        cai.cai_free(ctx)
+
+
 def test_teacher_forced_random_states():
     # Random mid-block states uploaded into the context, then one step.
     wl = _wl("toy", B=6, P=16, gen_len=32, T=20)

@@ -1161,7 +1161,7 @@ int cai_state_upload(cai_ctx* c, const cai_host_state* src) {
   lp.L = c->L;
   lp.n_blocks = c->cfg.n_blocks;
   lp.blk = c->blk;
-  rebuild_list_kernel<<<1, kCommitThreads>>>(lp);
+  rebuild_list_kernel<<<1, kListThreads>>>(lp);
   c->stats.launches++;
   r = check_launch(c);
   if (r != CAI_OK) return r;

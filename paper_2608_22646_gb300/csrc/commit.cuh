@@ -97,7 +97,7 @@ __device__ __forceinline__ int budget_tier(float s, int p, int half, int late) {
 // One step of Algorithm 1 for sequence b, by the whole calling CTA (blockDim.x
 // a multiple of 32; every thread must call it).  The sequence's state is read
 // into shared memory in one round of loads; warps then merge the partials of
-// the still-masked positions (kPosPerWarp at a time, all loads issued before
+// the still-masked positions (kPPW at a time, all loads issued before
 // any merge) and lane 0 applies the commit rule (Box 6, Eq. position_commit,
 // with the step-zero init of Boxes 2 and 5); thread 0 updates the low-yield
 // counter and the exit state (Box 7, Algorithm 1).  Global state is only
@@ -115,6 +115,7 @@ struct CommitSmem {
   int16_t stable[kMaxP];  // diagnostics: stability step before this step
 };
 
+template <int kPPW = kPosPerWarp>
 __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs,
                                      const float4* part, int n_part, int* left_after = nullptr) {
   __shared__ int s_eta, s_left, s_reason, s_unres, s_ell, s_running;
@@ -149,11 +150,11 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
   const bool gating = (p.flags & kFlagGating) != 0;
 
   if (running) {
-    for (int base = warp; base < p.P; base += nwarps * kPosPerWarp) {
-      int row[kPosPerWarp];
-      float4 q[kPosPerWarp][kPartPerLane];
+    for (int base = warp; base < p.P; base += nwarps * kPPW) {
+      int row[kPPW];
+      float4 q[kPPW][kPartPerLane];
 #pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
+      for (int j = 0; j < kPPW; ++j) {
         const int pp = base + j * nwarps;
         row[j] = -1;
         if (pp < p.P && s_tok[pp] == kMask) {
@@ -166,7 +167,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
         }
       }
 #pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
+      for (int j = 0; j < kPPW; ++j) {
         const float4* pr = part + static_cast<size_t>(row[j] < 0 ? 0 : row[j]) * n_part;
 #pragma unroll
         for (int u = 0; u < kPartPerLane; ++u) {
@@ -177,7 +178,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
         }
       }
 #pragma unroll
-      for (int j = 0; j < kPosPerWarp; ++j) {
+      for (int j = 0; j < kPPW; ++j) {
         if (row[j] < 0) continue;  // warp-uniform
         const int pp = base + j * nwarps;
         float m = kNegBig, s = 0.0f;

@@ -15,7 +15,13 @@ namespace cai {
 
 constexpr int kGatherRowsPerCta = 4;
 constexpr int kGatherThreads = 256;
-constexpr int kCommitThreads = 256;  // merge kernel: small enough to share an SM with the LM head
+constexpr int kListThreads = 256;    // rebuild_list_kernel
+// Merge kernel: one CTA per sequence, 16 warps of 4 positions each, so that
+// a 64-position block merges in one round of loads and the last CTA builds
+// the next step's list 512 tokens at a time (measured against 256 threads of
+// 6 positions: see the design notes).
+constexpr int kCommitThreads = 512;
+constexpr int kCommitPPW = 4;
 
 // ------------------------------------------------------------ gather (K1) --
 
@@ -185,7 +191,7 @@ struct ListParams {
 };
 
 // Rebuild the masked-row list from the state (after a state upload).
-__global__ void __launch_bounds__(kCommitThreads) rebuild_list_kernel(const ListParams p) {
+__global__ void __launch_bounds__(kListThreads) rebuild_list_kernel(const ListParams p) {
   const int n = build_masked_list(p.tok, p.exit_reason, p.list, p.row_of, p.B, p.P, p.L,
                                   p.n_blocks, p.blk);
   if (threadIdx.x == 0) *p.d_M = n;
@@ -209,11 +215,11 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
     const int per_row =
         pair_partials_per_row(M, p.pair_pairs, pair_swapped(M, p.pair_swap_max_n));
     if (per_row > 0)
-      merge_commit_sequence(p, blockIdx.x, cs, p.part, per_row);
+      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, per_row);
     else
-      merge_commit_sequence(p, blockIdx.x, cs, p.rowres, 1);
+      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.rowres, 1);
   } else {
-    merge_commit_sequence(p, blockIdx.x, cs, p.part, p.n_part);
+    merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, p.n_part);
   }
   if (gridDim.x > 1) {
     if (threadIdx.x == 0) {

@@ -290,9 +290,11 @@ __device__ int build_masked_list(const int* tok, const int* exit_reason, int* li
     const int i = i0 + tid;
     bool mk = false;
     if (i < BP) {
+      // Both loads issued before either is tested (one round trip, not two).
       const int b = i / P, pp = i - b * P;
-      mk = __ldcg(&tok[static_cast<size_t>(b) * L + blk * P + pp]) == kMask &&
-           __ldcg(&exit_reason[b * n_blocks + blk]) == kRunning;
+      const int tk = __ldcg(&tok[static_cast<size_t>(b) * L + blk * P + pp]);
+      const int ex = __ldcg(&exit_reason[b * n_blocks + blk]);
+      mk = (tk == kMask) & (ex == kRunning);
     }
     const unsigned bal = __ballot_sync(0xffffffffu, mk);
     const int wpre = __popc(bal & ((1u << lane) - 1u));

@@ -234,12 +234,16 @@ def test_fraction_eta_mode():
         cai.cai_free(ctx)
 
 
-def test_all_commit_at_step_zero_and_noop_steps():
+@pytest.mark.parametrize("B", [2, 3])
+def test_all_commit_at_step_zero_and_noop_steps(B):
     # Hidden rows equal to a scaled W row make every confidence ~1: every
-    # token commits at t = 0, the block exits DONE, and later steps decode nothing.
-    B, P, H, V, T = 2, 16, 256, 4096, 8
+    # token commits at t = 0, the block exits DONE, and later steps decode
+    # nothing.  B P = 32: single-kernel steps; 48: multi-kernel steps, whose
+    # pair LM head records the empty step's M = 0 itself.
+    P, H, V, T = 16, 256, 4096, 8
     ctx, W = _ctx(B, P, H, V, T, 2)
     try:
+        assert (cai.cai_get_stats(ctx)["kernels_per_step"] == 1) == (B * P <= 32)
         tgt = torch.arange(B * P, device="cuda") * 37 % V
         h = (W[tgt].float() * 400.0).to(torch.bfloat16).reshape(B, P, H)
         cai.cai_first_step(ctx, h)

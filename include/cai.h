@@ -26,8 +26,9 @@
  * before cai_init launches them plainly instead).  With B P <= 32 a step is
  * one kernel: the LM head over every row of the block, whose last CTA applies
  * the commit rule; it streams W before the previous step has committed and
- * waits for it only to write its partials and to commit.  With B P > 64 a
- * step is gather, LM head, merge + commit.  The LM head is the CTA-pair
+ * waits for it only to write its partials and to commit (CAI_FUSED_MAX_BP=n
+ * moves the limit, up to 256).  With B P > 32 a step is gather, LM head,
+ * merge + commit.  The LM head is the CTA-pair
  * kernel (tcgen05 cta_group::2), which picks its orientation per step from
  * the masked-row count M: the rows as MMA N in row tiles of equal width (a
  * multiple of 32) while that width is at most 192, else as MMA M in 256-row

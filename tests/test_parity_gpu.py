@@ -367,6 +367,37 @@ def test_multi_kernel_edge_shapes(shape):
         cai.cai_free(ctx)
 
 
+def _random_shapes(n, seed=2608):
+    rng = np.random.default_rng(seed)
+    out = []
+    while len(out) < n:
+        B = int(rng.integers(1, 13))
+        P = int(rng.choice([8, 16, 24, 32, 48, 64]))
+        H = int(rng.choice([64, 128, 192, 256]))
+        V = int(rng.integers(128, 6000))
+        T = int(rng.integers(4, 11))
+        nb = int(rng.choice([1, 2]))
+        if 8 <= B * P <= 768:
+            out.append((B, P, H, V, T, nb))
+    return out
+
+
+@pytest.mark.parametrize("shape", _random_shapes(14))
+def test_random_shape_trajectories(shape):
+    # Seeded random shapes (mostly multi-kernel: both pair orientations, one to
+    # three row tiles, ragged vocabularies and hidden sizes), each a full
+    # trajectory checked step by step against the oracle.
+    B, P, H, V, T, nb = shape
+    wl = synth.Workload("random", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=B * 1000 + P)
+    try:
+        rep, _ = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P
+    finally:
+        cai.cai_free(ctx)
+
+
 def test_teacher_forced_random_states():
     # Random mid-block states uploaded into the context, then one step.
     wl = _wl("toy", B=6, P=16, gen_len=32, T=20)

@@ -43,6 +43,10 @@
 // the next one learns it from the published step word (CommitParams::pub)
 // while streaming and stops at the next K block.
 //
+// Multi-kernel steps (fused = 0) run on lm_head_pair_kernel; this kernel
+// takes their steps of fewer than pair_min_M rows only when the pair kernel
+// never runs swapped (CAI_PAIR_SWAP=0) or is off (CAI_PAIR=0).
+//
 // Warp roles (192 threads, one CTA per SM):
 //   warp 0      producer (one lane): W stages (bulk copies), hidden stages (TMA)
 //   warp 1      TMEM allocator; one lane issues tcgen05.mma

@@ -1,57 +1,57 @@
-// LM head for steps with many masked rows (M > 128, several sequences), on
-// CTA pairs: the same quantities as lm_head_softmax_kernel (Box 1 of arXiv
-// 2608.22646: c_i = max_v p_theta(x_i = v) and argmax_v p_theta, logits never
-// leaving tensor memory), computed in the orientation a compute-bound
-// contraction wants.
+// LM head of the multi-kernel step, on CTA pairs (tcgen05 cta_group::2): the
+// same quantities as lm_head_softmax_kernel (Box 1 of arXiv 2608.22646:
+// c_i = max_v p_theta(x_i = v) and argmax_v p_theta, logits never leaving
+// tensor memory), for any number M >= 1 of masked rows, in one of two
+// orientations chosen per step from M (pair_swapped).
 //
-// With hundreds to thousands of rows the contraction is tensor-bound (2 V H M
-// flops against 2 V H bytes of W), so it is run without swapping A and B:
-// the masked rows fill the MMA M dimension and the vocabulary the N dimension.
-// One tcgen05.mma of the pair (cta_group::2) computes a 256 x 256 tile:
-// each CTA holds 128 of the rows (its A half) and 128 of the vocabulary rows
-// (its B half) per K block, and keeps its 128 x 256 half of the accumulator
-// in tensor memory.  Per K block a CTA loads 32 KiB (16 KiB of hidden rows,
+// Unswapped, for wide steps: with hundreds to thousands of rows the
+// contraction is tensor-bound (2 V H M flops against 2 V H bytes of W), so
+// the masked rows fill the MMA M dimension and the vocabulary the N
+// dimension.  One tcgen05.mma of the pair computes a 256 x 256 tile: each CTA
+// holds 128 of the rows (its A half) and 128 of the vocabulary rows (its B
+// half) per K block, and keeps its 128 x 256 half of the accumulator in
+// tensor memory.  Per K block a CTA loads 32 KiB (16 KiB of hidden rows,
 // 16 KiB of W) for 2 * 128 * 256 * 64 flops, half the shared-memory traffic
-// per flop of a single-CTA 128 x 256 tile.
+// per flop of a single-CTA 128 x 256 tile.  A tensor-memory lane holds one
+// row's logits, so the epilogue is a serial online softmax per thread over
+// the 256 columns of a tile, no shuffles.
 //
-// A tensor-memory lane holds one row's logits, so the epilogue is a serial
-// online softmax per thread over the 256 columns of a tile, no shuffles.  When
-// the number of pairs is a multiple of the number of row tiles n_rt, every
-// tile of a pair has the same row tile, and the epilogue folds its tiles into
-// one partial (max * log2 e, sum of 2^(z log2 e - max), argmax) per row and
-// pair, which the commit reads directly (pair_partials_per_row); otherwise it
-// writes one partial per row and vocabulary tile, merged per row by
-// reduce_partials_kernel.
+// Swapped, for narrow steps: the vocabulary fills the MMA M dimension (256
+// rows per pair, 128 per CTA: the W half is the A operand) and the masked
+// rows the N dimension.  The M rows are split into n_rt = ceil(M / 256) row
+// tiles of equal width N (a multiple of 32, at most 256), so a step pads at
+// most 31 rows per tile instead of up to 255: M = 305 runs as two 160-column
+// tiles, M = 159 as one of 160, M = 5 as one of 32.  A tensor-memory lane
+// then holds one vocabulary row of every column; the epilogue reduces across
+// lanes (transpose_logits32) and across the four epilogue warps (a
+// shared-memory exchange), and each CTA writes the triples of its 128
+// vocabulary rows: two partials per pair.  Each CTA loads N / 2 of a tile's
+// rows per K block (one box of the next power of two rows).  The cross-lane
+// reduction costs more than the serial one, so wide tiles stay unswapped: a
+// step runs swapped when N is at most swap_max_n (192 by default; measured
+// per step on the Dream shape: N = 64..192 3 to 11 % faster than the padded
+// unswapped tile, N = 224, 256 1 to 7 % slower).
 //
-// Work: tiles (v, j) of 256 vocabulary rows x 256 masked rows, numbered
+// Partials: when the number of pairs is a multiple of the number of row
+// tiles n_rt, every tile of a pair has the same row tile, and the epilogue
+// folds its tiles into one partial (max * log2 e, sum of 2^(z log2 e - max),
+// argmax) per row and pair (and CTA, swapped), which the commit reads
+// directly (pair_partials_per_row); otherwise it writes one partial per row
+// and vocabulary tile (and CTA), merged per row by reduce_partials_kernel.
+//
+// Work: tiles (v, j) of 256 vocabulary rows x one row tile, numbered
 // t = v * n_rt + j and dealt round-robin to the pairs of a persistent grid.
 // The pairs working at one time share few W tiles, each read from HBM once
 // and by the n_rt pairs of its row tiles from L2; the gathered hidden rows
 // (at most 2 x 65536 x 16384 bytes, in practice tens of MB) stay in L2.
 //
-// Swapped orientation (chosen per step, pair_swapped): the vocabulary fills the MMA M dimension (256
-// rows per pair, 128 per CTA: the W half is the A operand) and the masked rows
-// the N dimension.  The M rows are split into n_rt = ceil(M / 256) row tiles
-// of equal width N (a multiple of 32, at most 256), so a step pads at most 31
-// rows per tile instead of up to 255: M = 305 runs as two 160-column tiles,
-// M = 159 as one of 160.  A tensor-memory lane then holds one vocabulary row
-// of every column; the epilogue reduces across lanes (transpose_merge32) and
-// across the four epilogue warps (a shared-memory exchange), and each CTA
-// writes the triples of its 128 vocabulary rows: two partials per pair.  Each
-// CTA loads N / 2 of a tile's rows per K block (one box of the next power of
-// two rows).  The cross-lane
-// reduction costs more instructions than the unswapped epilogue, so full-width
-// tiles stay unswapped: a step runs swapped when its tile width N is at most
-// swap_max_n (192 by default; measured, Dream shape: N = 64..192 5 % faster
-// than the padded unswapped tile, N = 224, 256 4 to 8 % slower).
-//
-// Roles per CTA (192 threads): warp 0 producer (hidden half and W half, each
-// one TMA box; W from a tile-major packed copy in which every box is one
-// contiguous 16 KiB block); warp 1 allocates tensor memory and, in the even
-// CTA, issues the MMAs; warps 2..5 epilogue.  Both CTAs' copies of a stage
-// complete on the even CTA's barrier (cta_group::2 loads), which the even
-// CTA's producer arms with the bytes of both.  Two accumulator buffers let
-// the epilogue of one tile overlap the next tile's MMAs.
+// Roles per CTA (192 threads): warp 0 producer (hidden half and W half by
+// TMA; W from a tile-major packed copy in which every box is one contiguous
+// 16 KiB block); warp 1 allocates tensor memory and, in the even CTA, issues
+// the MMAs; warps 2..5 epilogue.  Both CTAs' copies of a stage complete on
+// the even CTA's barrier (cta_group::2 loads), which the even CTA's producer
+// arms with the bytes of both.  Two accumulator buffers let the epilogue of
+// one tile overlap the next tile's MMAs.
 #pragma once
 
 #include <climits>

@@ -163,3 +163,25 @@ def test_pair_plan_covers_rows_with_bounded_padding(n_pairs):
     assert lib.cai_test_pair_plan(5, 0, 192, out) == cai.CAI_ERR_ARG
     assert lib.cai_test_pair_plan(5, 76, -1, out) == cai.CAI_ERR_ARG
     assert lib.cai_test_pair_plan(5, 76, 192, None) == cai.CAI_ERR_ARG
+
+
+def test_bench_reference_arm_json_line():
+    # The reference arm (the oracle on the host cores) needs no GPU: one JSON
+    # line with the contract's fields, its own cpu_baseline and e2e.
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, "bench.py", "--impl", "reference", "--workload", "toy",
+                          "--steps", "2", "--warmup", "3"], cwd=root, capture_output=True,
+                         text=True, timeout=600)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    assert line["impl"] == "reference" and line["value"] > 0 and line["unit"] == "positions/s"
+    assert line["higher_is_better"] is True and line["steps"] == 2 and line["warmup"] == 3
+    for k in ("metric", "n_gpus", "ms_per_step", "scaling", "dtype", "data", "config"):
+        assert k in line, k
+    cb = line["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"]
+    assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]

@@ -124,6 +124,14 @@ bool make_map(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, ui
 }
 
 int round_up(int x, int m) { return (x + m - 1) / m * m; }
+
+// Swapped pair tiles: one map of the gathered rows per box height 16..128.
+template <typename Ctx>
+bool make_row_maps(Ctx* c, int H) {
+  for (int q = 0; q < 8; ++q)
+    if (!make_map(&c->tm_rows.box[q], c->hc, c->rows_cap, H, 16 * (q + 1))) return false;
+  return true;
+}
 int next_pow2(int x) {
   int p = 1;
   while (p < x) p <<= 1;
@@ -190,7 +198,7 @@ struct cai_ctx {
   void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
   void* wt = nullptr;    // tile-major packed copy of W (pack_w_tiles_kernel), pair kernel
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
-  PairRowMaps tm_rows{};  // ... in 128-, 64-, 32-, 16-row boxes (swapped pair kernel)
+  PairRowMaps tm_rows{};  // ... in 16-, 32-, ..., 128-row boxes (swapped pair kernel)
   CUtensorMap tm_w{};    // wt as [2 n_vt (H / 64) 128, 64], 16 KiB unswizzled boxes
   bool use_pair = false; // steps with >= pair_min_M rows run lm_head_pair_kernel
   int swap_max_n = 0;       // ... swapped when its tile width is at most this (pair_swapped)
@@ -904,10 +912,7 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   std::memset(c->hf_host, 0, sizeof(HostFlag));
   if (!make_map(&c->tm_h, c->hc, c->rows_cap, cfg->H, kBoxRowsB) ||
       (c->use_pair && !make_map(&c->tm_a, c->hc, c->rows_cap, cfg->H, kPairHalf)) ||
-      (c->swap_max_n && !make_map(&c->tm_rows.box[0], c->hc, c->rows_cap, cfg->H, 128)) ||
-      (c->swap_max_n && !make_map(&c->tm_rows.box[1], c->hc, c->rows_cap, cfg->H, 64)) ||
-      (c->swap_max_n && !make_map(&c->tm_rows.box[2], c->hc, c->rows_cap, cfg->H, 32)) ||
-      (c->swap_max_n && !make_map(&c->tm_rows.box[3], c->hc, c->rows_cap, cfg->H, 16)) ||
+      (c->swap_max_n && !make_row_maps(c, cfg->H)) ||
       (c->use_pair &&
        !make_map(&c->tm_w, c->wt, static_cast<uint64_t>(2 * c->n_vt) * (cfg->H / kPairBlockK) *
                                       kPairHalf,

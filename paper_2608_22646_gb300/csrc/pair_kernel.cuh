@@ -26,7 +26,7 @@
 // lanes (transpose_logits32) and across the four epilogue warps (a
 // shared-memory exchange), and each CTA writes the triples of its 128
 // vocabulary rows: two partials per pair.  Each CTA loads N / 2 of a tile's
-// rows per K block (one box of the next power of two rows).  The cross-lane
+// rows per K block as one box of exactly that many rows.  The cross-lane
 // reduction costs more than the serial one, so wide tiles stay unswapped: a
 // step runs swapped when N is at most swap_max_n (192 by default; measured
 // per step on the Dream shape: N = 64..192 3 to 11 % faster than the padded
@@ -72,12 +72,12 @@ constexpr int kPairTmemCols = 2 * kPairTileVocab;            // two accumulators
 constexpr int kSwapColStep = 32;    // swapped orientation: granularity of N
 constexpr int kSwapXchBytes = 2 * 4 * kPairTileVocab * 16;  // cross-warp exchange, two buffers
 
-// Tensor maps of the gathered rows with boxes of 128, 64, 32 and 16 rows
-// (swapped orientation: a CTA's N / 2 rows of a tile load as the smallest of
-// these boxes that holds them; each TMA copy has a fixed cost of the order
-// of a 16 KiB copy's transfer time, so one box beats several exact ones).
+// Tensor maps of the gathered rows with boxes of 16, 32, ..., 128 rows
+// (swapped orientation: a CTA's N / 2 rows of a tile, a multiple of 16, load
+// as one exact box: each TMA copy has a fixed cost, and every byte written
+// to shared memory competes with the MMAs' operand reads).
 struct PairRowMaps {
-  CUtensorMap box[4];  // box[q]: 128 >> q rows
+  CUtensorMap box[8];  // box[q]: 16 (q + 1) rows
 };
 
 struct PairParams {
@@ -257,7 +257,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   if (warp == 0 && lane == 0) {
     prefetch_tmap(&tm_w);
     if (swap) {
-      for (int q = 0; q < 4; ++q) prefetch_tmap(&hm.box[q]);
+      prefetch_tmap(&hm.box[swap_tile_cols(M, n_rt) / 32 - 1]);
     } else {
       prefetch_tmap(&tm_a);
     }
@@ -279,12 +279,9 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       PairRing r;
       long long issued = 0;
       bool ok = true;
-      // Swapped: a CTA's rt_rows / 2 rows load as one box of the next power
-      // of two (16..128 rows; the MMA reads the first rt_rows / 2): one TMA
-      // copy instead of up to four costs less than the extra bytes from L2.
-      int q1 = 3;
-      while (q1 > 0 && (kPairHalf >> q1) < rt_rows / 2) --q1;
-      const int box_rows = kPairHalf >> q1;
+      // Swapped: a CTA's rt_rows / 2 rows (a multiple of 16) load as one box.
+      const int q1 = rt_rows / 32 - 1;
+      const int box_rows = rt_rows / 2;
       // Bytes of one stage, both CTAs (the even CTA arms its barrier for them).
       const uint32_t stage_tx =
           swap ? 2u * static_cast<uint32_t>(kPairHalfBytes + box_rows * kPairBlockK * 2)

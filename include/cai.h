@@ -362,6 +362,16 @@ int cai_test_head_grid_limit(int32_t n);
 int cai_test_check_guards(cai_ctx* ctx, int32_t* n_bad);
 
 /*
+ * Testing hook: launches, on the stream, a kernel that waits through the
+ * step kernels' bounded barrier wait on a barrier nothing arrives at; after
+ * the wait limit (2 s) it records a wait failure in the context's error word
+ * and returns.  The next call that reads the word (cai_poll,
+ * cai_state_download) then returns CAI_ERR_DEVICE and the context is sticky.
+ * No trap and no fault: the device and other contexts stay usable.
+ */
+int cai_test_wait_timeout(cai_ctx* ctx, void* stream);
+
+/*
  * Testing hook, host only (no device use): the CTA-pair LM head's plan for a
  * step with M masked rows on n_pairs pairs whose widest swapped tile is
  * swap_max_n (0: never swapped).  Writes out[0] = 1 if the step runs in the

@@ -52,7 +52,7 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
-           "cai_test_pair_plan",
+           "cai_test_pair_plan", "cai_test_wait_timeout",
            "cai_test_check_guards",
            "cai_head_rows_static")
 
@@ -124,6 +124,7 @@ def _load():
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
         "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
         "cai_test_pair_plan": (ctypes.c_int, [i32, i32, i32, ctypes.POINTER(i32)]),
+        "cai_test_wait_timeout": (ctypes.c_int, [vp, vp]),
         "cai_test_check_guards": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
         "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
     }
@@ -298,6 +299,10 @@ def cai_free(ctx: Ctx) -> None:
 
 def cai_test_fail_alloc_after(n: int) -> None:
     _check(lib().cai_test_fail_alloc_after(n), "cai_test_fail_alloc_after")
+
+
+def cai_test_wait_timeout(ctx: Ctx, stream=None) -> None:
+    _check(lib().cai_test_wait_timeout(ctx.handle, _stream(stream)), "cai_test_wait_timeout")
 
 
 def cai_test_pair_plan(M: int, n_pairs: int, swap_max_n: int) -> dict:

@@ -1258,6 +1258,14 @@ int cai_test_head_grid_limit(int32_t n) {
   return CAI_OK;
 }
 
+int cai_test_wait_timeout(cai_ctx* c, void* stream) {
+  if (!c) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  wait_timeout_probe_kernel<<<1, 32, 0, static_cast<cudaStream_t>(stream)>>>(c->err, kErrWaitFull);
+  c->stats.launches++;
+  return check_launch(c);
+}
+
 int cai_test_pair_plan(int32_t M, int32_t n_pairs, int32_t swap_max_n, int32_t* out) {
   if (M < 1 || n_pairs < 1 || swap_max_n < 0 || !out) return CAI_ERR_ARG;
   const bool swap = pair_swapped(M, swap_max_n);

@@ -179,6 +179,24 @@ __global__ void __launch_bounds__(kGatherThreads) row_rms_kernel(const RmsParams
   if (row < p.rows && lane == 0) p.inv_r[row] = rsqrtf(ss / static_cast<float>(p.H) + p.eps);
 }
 
+// ------------------------------------------------- bounded-wait test hook --
+
+// Waits, through the same bounded mbar_wait every step kernel uses, on a
+// barrier nothing arrives at: after the wait limit it records `site` in the
+// error word and returns (no trap, no fault; the context stays valid until
+// the host reads the word).
+__global__ void wait_timeout_probe_kernel(uint32_t* err, uint32_t site) {
+  __shared__ uint64_t bar;
+  __shared__ int abort_flag;
+  if (threadIdx.x == 0) {
+    mbar_init(&bar, 1);
+    abort_flag = 0;
+    fence_mbar_init();
+  }
+  __syncthreads();
+  if (threadIdx.x == 0) mbar_wait(&bar, 0, &abort_flag, err, site);
+}
+
 // ------------------------------------------------------ list rebuild -----
 
 struct ListParams {

@@ -123,6 +123,7 @@ def test_null_and_status_strings():
     assert cai.cai_strerror(-99) == "unknown status"
     assert lib.cai_test_fail_alloc_after(-1) == cai.CAI_ERR_ARG
     assert lib.cai_test_head_grid_limit(-1) == cai.CAI_ERR_ARG
+    assert lib.cai_test_wait_timeout(None, None) == cai.CAI_ERR_ARG
 
 
 def test_no_device_is_a_status_not_a_crash():

@@ -521,6 +521,39 @@ def test_host_rows_pipelined_match_device(B, host):
         cai.cai_free(b)
 
 
+def test_device_wait_timeout_reports_and_device_stays_usable():
+    # A kernel waits, through the step kernels' bounded barrier wait, on a
+    # barrier nothing arrives at: after the limit it records the failure in
+    # the context's error word and returns.  The host then reads
+    # CAI_ERR_DEVICE, the context stays sticky, and a new context on the same
+    # GPU runs a checked trajectory.
+    import time
+    wl = synth.WORKLOADS["toy"]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=41)
+    try:
+        cai.cai_first_step(ctx, hs(0, 0))
+        torch.cuda.synchronize()
+        cai.cai_state_download(ctx)                      # healthy so far
+        t0 = time.perf_counter()
+        cai.cai_test_wait_timeout(ctx)
+        torch.cuda.synchronize()
+        assert 1.5 < time.perf_counter() - t0 < 30.0     # the wait ran to its limit
+        with pytest.raises(cai.CaiError) as e:
+            cai.cai_state_download(ctx)
+        assert e.value.status == cai.CAI_ERR_DEVICE
+        with pytest.raises(cai.CaiError) as e:
+            cai.cai_denoise_step(ctx, hs(0, 1))
+        assert e.value.status == cai.CAI_ERR_DEVICE
+    finally:
+        cai.cai_free(ctx)
+    ctx2, W2 = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    try:
+        parity.run_checked_trajectory(ctx2, W2, synth.HiddenStates(wl, W2, "calibrated", seed=43))
+    finally:
+        cai.cai_free(ctx2)
+
+
 def test_order_errors_and_poll():
     wl = synth.WORKLOADS["toy"]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, 2)

@@ -211,6 +211,14 @@ def _diagnostics_summary(st: dict) -> dict:
     return out
 
 
+def pg_timeout():
+    """Process-group timeout: a rank that died leaves the others' next barrier
+    or collective failing after this long instead of waiting for ever
+    (CAI_PG_TIMEOUT_S, default 300 s)."""
+    import datetime
+    return datetime.timedelta(seconds=float(os.environ.get("CAI_PG_TIMEOUT_S", "300")))
+
+
 def aggregate(ms: float, positions: int, dist=None, device=None):
     """Whole-job figures over ranks: the slowest rank's time and the sum of
     every rank's decoded positions (each rank decodes its own batch)."""
@@ -254,7 +262,7 @@ def main():
     if world > 1:
         import torch.distributed as dist
         torch.cuda.set_device(local)
-        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local), timeout=pg_timeout())
     wl = synth.WORKLOADS[args.workload]
 
     if args.impl == "reference":

@@ -554,6 +554,56 @@ def test_device_wait_timeout_reports_and_device_stays_usable():
         cai.cai_free(ctx2)
 
 
+@pytest.mark.parametrize("B,P", [(2, 16), (5, 64)])
+def test_checkpoint_resume_in_new_context(B, P):
+    # Checkpoint/resume: a trajectory interrupted after a few steps of its
+    # second block, its state downloaded, freed, uploaded into a new context
+    # and continued, ends exactly where the uninterrupted trajectory does.
+    wl = _wl("toy", B=B, P=P, gen_len=3 * P, a0="bimodal")
+    W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=47)
+    inp = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+
+    def run(ctx, start_blk=0, start_t=0, stop=None):
+        for blk in range(start_blk, wl.n_blocks):
+            if blk > start_blk or (blk == start_blk and start_t == 0 and blk > 0):
+                cai.cai_block_advance(ctx)
+            for t in range(start_t if blk == start_blk else 0, wl.T):
+                if stop == (blk, t):
+                    torch.cuda.synchronize()
+                    return
+                (cai.cai_first_step if t == 0 else cai.cai_denoise_step)(ctx, inp[blk][t])
+                torch.cuda.synchronize()
+                if cai.cai_poll(ctx, 0, 5000):
+                    break
+        torch.cuda.synchronize()
+
+    a = cai.cai_init(cfg, W)
+    try:
+        run(a)
+        full = cai.cai_state_download(a)
+    finally:
+        cai.cai_free(a)
+    b = cai.cai_init(cfg, W)
+    try:
+        run(b, stop=(1, 2))
+        ckpt = cai.cai_state_download(b)
+    finally:
+        cai.cai_free(b)
+    assert ckpt["blk"] == 1 and ckpt["t_next"] == 2
+    c = cai.cai_init(cfg, W)
+    try:
+        cai.cai_state_upload(c, ckpt)
+        run(c, start_blk=1, start_t=2)
+        resumed = cai.cai_state_download(c)
+    finally:
+        cai.cai_free(c)
+    for k in ("tok", "conf", "cand", "cstep", "budget", "s0", "exit_reason", "exit_step",
+              "unresolved", "m_hist"):
+        assert np.array_equal(full[k], resumed[k]), k
+
+
 def test_order_errors_and_poll():
     wl = synth.WORKLOADS["toy"]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, 2)

@@ -246,8 +246,9 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
  * cudaHostAlloc), the gather reads the masked rows in place over the host
  * link, on the stream (valid until the stream passes this call).  Otherwise
  * the rows are copied to the device: with B P <= 32 on a stream of the
- * context's own into one of two alternating device buffers, which the step
- * waits for (so the copy for the next step can run during this one), with
+ * context's own into one of two alternating device buffers, which the step's
+ * kernel waits for on the device (so the copy for the next step runs during
+ * this one and the step's stream itself waits for nothing), with
  * B P > 32 on the step's stream; page-locked memory must stay valid until
  * the stream passes this call, pageable memory is staged by the CUDA runtime
  * before the call returns.

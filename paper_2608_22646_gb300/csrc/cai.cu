@@ -95,6 +95,26 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
+// cuStreamWriteValue64 (driver API), for the staged-rows sequence words;
+// null if the driver does not provide it.
+typedef CUresult (*WriteValue64Fn)(CUstream, CUdeviceptr, cuuint64_t, unsigned int);
+WriteValue64Fn get_write_value64() {
+  static WriteValue64Fn fn = nullptr;
+  static bool tried = false;
+  if (fn || tried) return fn;
+  tried = true;
+  void* ptr = nullptr;
+  cudaDriverEntryPointQueryResult q;
+  if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue64", &ptr, 12000, cudaEnableDefault, &q) !=
+          cudaSuccess ||
+      q != cudaDriverEntryPointSuccess) {
+    cudaGetLastError();
+    return nullptr;
+  }
+  fn = reinterpret_cast<WriteValue64Fn>(ptr);
+  return fn;
+}
+
 EncodeTiledFn get_encoder() {
   static EncodeTiledFn fn = nullptr;
   if (fn) return fn;
@@ -226,6 +246,15 @@ struct cai_ctx {
   cudaEvent_t ev_copied[2] = {nullptr, nullptr};
   cudaEvent_t ev_read[2] = {nullptr, nullptr};
   bool read_pending[2] = {false, false};
+  // After its copy the side stream writes the step's id + 1 into
+  // stage_seq_dev[k]; the step's kernel waits for that word before reading
+  // the rows, so the step's stream waits for nothing and consecutive steps
+  // keep their programmatic overlap.  Used when no other kernel of the step
+  // reads the rows first (no final norm, no diagnostics) and the driver
+  // provides stream memory writes; otherwise the step's stream waits for
+  // ev_copied.
+  unsigned long long* stage_seq_dev = nullptr;
+  bool stage_by_word = false;
   bool fused = false;    // single-kernel step (B P <= 32)
   int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
   int b_slot_bytes = 0;
@@ -414,10 +443,18 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       if ((c->read_pending[k] &&
            cudaStreamWaitEvent(c->copy_stream, c->ev_read[k], 0) != cudaSuccess) ||
           cudaMemcpyAsync(c->stage2[k], hidden, bytes, cudaMemcpyHostToDevice, c->copy_stream) !=
-              cudaSuccess ||
-          cudaEventRecord(c->ev_copied[k], c->copy_stream) != cudaSuccess ||
-          cudaStreamWaitEvent(stream, c->ev_copied[k], 0) != cudaSuccess)
+              cudaSuccess)
         return fail(c, CAI_ERR_CUDA);
+      if (c->stage_by_word) {
+        // Default flags: the write follows the copy and makes its bytes visible.
+        if (get_write_value64()(reinterpret_cast<CUstream>(c->copy_stream),
+                                reinterpret_cast<CUdeviceptr>(c->stage_seq_dev + k),
+                                static_cast<cuuint64_t>(step_id + 1), 0) != CUDA_SUCCESS)
+          return fail(c, CAI_ERR_CUDA);
+      } else if (cudaEventRecord(c->ev_copied[k], c->copy_stream) != cudaSuccess ||
+                 cudaStreamWaitEvent(stream, c->ev_copied[k], 0) != cudaSuccess) {
+        return fail(c, CAI_ERR_CUDA);
+      }
       hid = c->stage2[k];
       stage_slot = k;
     } else {
@@ -503,6 +540,10 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.fused = c->fused ? 1 : 0;
   hp.M_fixed = c->BP;
   hp.max_M = c->use_pair ? c->pair_min_M - 1 : INT_MAX;
+  if (stage_slot >= 0 && c->stage_by_word) {
+    hp.stage_word = c->stage_seq_dev + stage_slot;
+    hp.stage_seq = static_cast<unsigned long long>(step_id + 1);
+  }
   hp.prefetch = c->use_pair ? 0 : 1;
   hp.first = first ? 1 : 0;
   hp.part = c->part;
@@ -834,6 +875,13 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   if (c->fused) {
     c->stage2[0] = c->hidden_stage;
     CAI_ALLOC(c->stage2[1], uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
+    CAI_ALLOC(c->stage_seq_dev, unsigned long long, 2)
+    if (cudaMemset(c->stage_seq_dev, 0, 16) != cudaSuccess) {
+      release(c);
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    c->stage_by_word = !c->norm && !(cfg->flags & CAI_DIAGNOSTICS) && get_write_value64() != nullptr;
   }
   CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   if (c->norm) {

@@ -77,6 +77,8 @@ struct HeadParams {
   int fused;           // 1: single-kernel step (see below), 0: gather / head / merge kernels
   int M_fixed;         // rows decoded by the single-kernel step (all B P positions)
   int max_M;           // multi-kernel step: larger steps are left to lm_head_pair_kernel
+  const unsigned long long* stage_word;  // single-kernel step on staged host rows: the rows
+  unsigned long long stage_seq;          // are read once *stage_word >= stage_seq (or null)
   int prefetch;        // stream the first W stages before the dependency wait
   int first;           // the step is a block's step zero (every position masked)
   float4* part;        // [rows_cap, G] partial (m2, S, idx bits, 0) per CTA
@@ -375,6 +377,10 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
       Ring ra, rb;
       long long a_issued = 0, b_issued = 0;
       bool ok = true, decided = !spec, skipped = false;
+      // Rows copied from the host on the context's side stream: wait (bounded)
+      // for that copy's sequence word before the first row load.
+      if (p.stage_word && !wait_word_ge(p.stage_word, p.stage_seq, sm.abort, p.err, kErrWaitRows))
+        ok = false;
       // The word is loaded one K block ahead of its use, so its latency never
       // holds up the stream of copies.
       unsigned long long pub_w = spec ? load_pub(p.cp.pub) : 0ull;

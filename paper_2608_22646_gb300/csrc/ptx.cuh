@@ -23,6 +23,7 @@ enum : uint32_t {
   kErrBadRow = 1u << 5,      // a masked token had no row in this step's list
   kErrWaitEpi = 1u << 6,     // epilogue warps waiting for each other's slices
   kErrBounds = 1u << 7,      // CAI_DEBUG builds: an index list or partial offset out of range
+  kErrWaitRows = 1u << 8,    // host rows staged by the side-stream copy did not arrive
 };
 
 // CAI_DEBUG builds check index lists and partial offsets before use: a value
@@ -95,6 +96,31 @@ __device__ __forceinline__ bool mbar_wait(uint64_t* bar, uint32_t parity, volati
   for (uint32_t it = 1;; ++it) {
     if (mbar_try_wait(bar, parity)) return true;
     if ((it & 63u) == 0u) {
+      if (*abort) return false;
+      if (global_timer_ns() - t0 > kWaitLimitNs) {
+        *abort = 1;
+        atomicOr(err, site);
+        return false;
+      }
+    }
+  }
+}
+
+// Wait until the 64-bit word at `word` (in global memory, written by a
+// stream memory operation after a copy) reaches `want`, bounded like
+// mbar_wait; on success the copy's bytes are visible to the async proxy
+// (TMA) of this thread.
+__device__ __forceinline__ bool wait_word_ge(const unsigned long long* word, unsigned long long want,
+                                             volatile int* abort, uint32_t* err, uint32_t site) {
+  const uint64_t t0 = global_timer_ns();
+  for (uint32_t it = 0;; ++it) {
+    unsigned long long v;
+    asm volatile("ld.acquire.sys.global.u64 %0, [%1];" : "=l"(v) : "l"(word) : "memory");
+    if (v >= want) {
+      asm volatile("fence.proxy.async.global;" ::: "memory");
+      return true;
+    }
+    if ((it & 63u) == 63u) {
       if (*abort) return false;
       if (global_timer_ns() - t0 > kWaitLimitNs) {
         *abort = 1;

@@ -695,6 +695,26 @@ def test_full_size_first_step_sampled(name):
         cai.cai_free(ctx)
 
 
+@pytest.mark.parametrize("name,n_blocks", [("llada", None), ("dream", 2)])
+def test_full_size_trajectory_every_row(name, n_blocks):
+    # The benchmark's own configuration at full size (B = 1, P = 32, the LLaDA
+    # or Dream weight shape, single-kernel steps, the calibrated generator):
+    # every step of the generation (LLaDA: all eight blocks; Dream: the first
+    # two) is checked teacher-forced on every masked row, confidences,
+    # argmaxes and every integer field of the state.
+    wl = synth.WORKLOADS[name]
+    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks, preset=cai.CAI_PRESET_LLADA)
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    try:
+        assert cai.cai_get_stats(ctx)["kernels_per_step"] == 1
+        rep, st = parity.run_checked_trajectory(ctx, W, hs, n_blocks=n_blocks)
+        blocks = wl.n_blocks if n_blocks is None else n_blocks
+        assert rep.rows >= blocks * wl.P
+        assert np.all(st["exit_reason"][:, :blocks] != 0)
+    finally:
+        cai.cai_free(ctx)
+
+
 def test_batched_multi_chunk_step_sampled():
     # B = 64 sequences, 2048 masked rows (8 MMA chunks of 256) at full LLaDA
     # width; sampled rows across chunks against the oracle.

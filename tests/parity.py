@@ -111,6 +111,22 @@ def check_step(ocfg: oracle.Config, W, hidden_bph, pre: dict, post: dict, blk: i
     near &= mk
     rep.near_ties += int(near.sum())
     conf_in = np.where(near, g_conf, conf_o)
+    # Inside the band the decision is the kernel's, taken in its precision: an
+    # fp32 confidence against the fp32-rounded theta_i (c >= theta_i) and
+    # theta_fb (c > theta_fb).  Where the fp64 comparison of the same value
+    # falls the other way (c within one fp32 ulp of the threshold), the
+    # oracle gets a value on the kernel's side of both thresholds.
+    if near.any():
+        fb = ocfg.theta_fb
+        for b, p in np.argwhere(near):
+            c32 = np.float32(g_conf[b, p])
+            want_th = bool(c32 >= np.float32(th[0, p]))
+            want_fb = bool(c32 > np.float32(fb))
+            for v in (float(c32), th[0, p], np.nextafter(th[0, p], -np.inf), fb,
+                      np.nextafter(fb, np.inf)):
+                if (v >= th[0, p]) == want_th and (v > fb) == want_fb:
+                    conf_in[b, p] = v
+                    break
     idx_in = np.where(mk & (gap_o <= GAP_TOL), g_cand, idx_o)
     oracle.controller_step(st, blk, t, conf_in, idx_in)
     for f in INT_FIELDS:

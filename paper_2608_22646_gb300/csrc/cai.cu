@@ -215,7 +215,7 @@ struct cai_ctx {
   void* hidden_stage = nullptr;
   HostFlag* hf_host = nullptr;
   HostFlag* hf_dev = nullptr;
-  void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout)
+  void* wpk = nullptr;   // packed copy of W (pack_weight_kernel layout), if head_in_step
   void* wt = nullptr;    // tile-major packed copy of W (pack_w_tiles_kernel), pair kernel
   CUtensorMap tm_a{};    // compact gathered rows in 128-row boxes (pair kernel)
   PairRowMaps tm_rows{};  // ... in 16-, 32-, ..., 128-row boxes (swapped pair kernel)
@@ -883,7 +883,9 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
     }
     c->stage_by_word = !c->norm && !(cfg->flags & CAI_DIAGNOSTICS) && get_write_value64() != nullptr;
   }
-  CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
+  // The swapped-operand kernel's packed W, only where that kernel runs (every
+  // single-kernel step; multi-kernel steps with CAI_PAIR_SWAP=0 or CAI_PAIR=0).
+  if (c->head_in_step) CAI_ALLOC(c->wpk, uint8_t, static_cast<size_t>(units) * kUnitRows * 2 * cfg->H)
   if (c->norm) {
     CAI_ALLOC(c->inv_r, float, c->rows_cap)
     if (cudaMemset(c->inv_r, 0, sizeof(float) * c->rows_cap) != cudaSuccess) {
@@ -931,9 +933,10 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   }
   {
     const long long n_chunks = static_cast<long long>(units) * kUnitRows * cfg->H / 8;
-    pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
-        static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units, c->G,
-        c->gmax, n_chunks, g_dev);
+    if (c->head_in_step)
+      pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+          static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units,
+          c->G, c->gmax, n_chunks, g_dev);
     if (c->use_pair)
       pack_w_tiles_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
           static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wt), cfg->V, cfg->H,

@@ -70,6 +70,20 @@ class StepReport:
                 f"near_ties={self.near_ties}, argmax_ties={self.argmax_ties})")
 
 
+def kernel_side_value(c, theta: float, theta_fb: float) -> float:
+    """A double on the same side of theta (c >= theta) and theta_fb (c >
+    theta_fb) as the kernel's fp32 comparisons of c with the fp32-rounded
+    thresholds put c."""
+    c32 = np.float32(c)
+    want_th = bool(c32 >= np.float32(theta))
+    want_fb = bool(c32 > np.float32(theta_fb))
+    for v in (float(c32), theta, np.nextafter(theta, -np.inf), theta_fb,
+              np.nextafter(theta_fb, np.inf)):
+        if (v >= theta) == want_th and (v > theta_fb) == want_fb:
+            return float(v)
+    raise AssertionError(f"no value matches the kernel's decisions for c = {c}")
+
+
 def check_step(ocfg: oracle.Config, W, hidden_bph, pre: dict, post: dict, blk: int, t: int,
                rep: StepReport | None = None, norm_weight=None, eps: float = 0.0) -> StepReport:
     """Teacher-forced check of one GPU step (pre -> post) against the oracle
@@ -116,17 +130,8 @@ def check_step(ocfg: oracle.Config, W, hidden_bph, pre: dict, post: dict, blk: i
     # theta_fb (c > theta_fb).  Where the fp64 comparison of the same value
     # falls the other way (c within one fp32 ulp of the threshold), the
     # oracle gets a value on the kernel's side of both thresholds.
-    if near.any():
-        fb = ocfg.theta_fb
-        for b, p in np.argwhere(near):
-            c32 = np.float32(g_conf[b, p])
-            want_th = bool(c32 >= np.float32(th[0, p]))
-            want_fb = bool(c32 > np.float32(fb))
-            for v in (float(c32), th[0, p], np.nextafter(th[0, p], -np.inf), fb,
-                      np.nextafter(fb, np.inf)):
-                if (v >= th[0, p]) == want_th and (v > fb) == want_fb:
-                    conf_in[b, p] = v
-                    break
+    for b, p in np.argwhere(near):
+        conf_in[b, p] = kernel_side_value(g_conf[b, p], th[0, p], ocfg.theta_fb)
     idx_in = np.where(mk & (gap_o <= GAP_TOL), g_cand, idx_o)
     oracle.controller_step(st, blk, t, conf_in, idx_in)
     for f in INT_FIELDS:

@@ -805,3 +805,34 @@ def test_long_dream_full_size_steps_sampled():
         assert cai.cai_test_check_guards(ctx) == 0
     finally:
         cai.cai_free(ctx)
+
+
+def test_bench_json_line_contract():
+    # The benchmark's own arm on the toy shape: one JSON line with the
+    # contract's keys, a device-timed value, the roofline object, the
+    # end-to-end figure through host buffers, clocks and the launch count.
+    import json
+    import os
+    import subprocess
+    import sys
+    root = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+    out = subprocess.run([sys.executable, "bench.py", "--workload", "toy", "--steps", "3",
+                          "--warmup", "3", "--no-cpu-baseline"], cwd=root, capture_output=True,
+                         text=True, timeout=900)
+    assert out.returncode == 0, out.stderr[-2000:]
+    line = json.loads(out.stdout.strip().splitlines()[-1])
+    for k in ("metric", "value", "unit", "n_gpus", "steps", "warmup", "ms_per_step",
+              "higher_is_better", "scaling", "vs_baseline", "dtype", "data", "config",
+              "roofline", "e2e", "gpu_launches", "clocks"):
+        assert k in line, k
+    assert line["value"] > 0 and line["steps"] == 3 and line["warmup"] == 3 and line["n_gpus"] == 1
+    assert line["config"]["workload"].startswith("toy")
+    roof = line["roofline"]
+    for k in ("bound", "achieved", "peak", "unit", "frac", "traffic"):
+        assert k in roof, k
+    assert abs(roof["frac"] - roof["achieved"] / roof["peak"]) < 1e-3
+    e2e = line["e2e"]
+    assert e2e["value"] > 0 and e2e["unit"] == line["unit"] and e2e["h2d_bytes_per_step"] > 0
+    assert e2e["d2h_bytes_per_step"] > 0
+    assert line["gpu_launches"] > 0
+    assert line["clocks"]["sm_max_mhz"] > 0

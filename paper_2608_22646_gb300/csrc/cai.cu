@@ -95,36 +95,31 @@ typedef CUresult (*EncodeTiledFn)(CUtensorMap*, CUtensorMapDataType, cuuint32_t,
                                   const cuuint32_t*, CUtensorMapInterleave, CUtensorMapSwizzle,
                                   CUtensorMapL2promotion, CUtensorMapFloatOOBfill);
 
-// cuStreamWriteValue64 (driver API), for the staged-rows sequence words;
-// null if the driver does not provide it.
-typedef CUresult (*WriteValue64Fn)(CUstream, CUdeviceptr, cuuint64_t, unsigned int);
-WriteValue64Fn get_write_value64() {
-  static WriteValue64Fn fn = nullptr;
-  static bool tried = false;
-  if (fn || tried) return fn;
-  tried = true;
+// A driver API entry point, or null if the driver does not provide it.
+void* driver_entry(const char* name) {
   void* ptr = nullptr;
   cudaDriverEntryPointQueryResult q;
-  if (cudaGetDriverEntryPointByVersion("cuStreamWriteValue64", &ptr, 12000, cudaEnableDefault, &q) !=
-          cudaSuccess ||
+  if (cudaGetDriverEntryPointByVersion(name, &ptr, 12000, cudaEnableDefault, &q) != cudaSuccess ||
       q != cudaDriverEntryPointSuccess) {
     cudaGetLastError();
     return nullptr;
   }
-  fn = reinterpret_cast<WriteValue64Fn>(ptr);
+  return ptr;
+}
+
+// Each entry point is resolved once; a function-local static is initialised
+// once even when contexts are created on several host threads at a time.
+// cuStreamWriteValue64, for the staged-rows sequence words:
+typedef CUresult (*WriteValue64Fn)(CUstream, CUdeviceptr, cuuint64_t, unsigned int);
+WriteValue64Fn get_write_value64() {
+  static const WriteValue64Fn fn =
+      reinterpret_cast<WriteValue64Fn>(driver_entry("cuStreamWriteValue64"));
   return fn;
 }
 
 EncodeTiledFn get_encoder() {
-  static EncodeTiledFn fn = nullptr;
-  if (fn) return fn;
-  void* ptr = nullptr;
-  cudaDriverEntryPointQueryResult q;
-  if (cudaGetDriverEntryPointByVersion("cuTensorMapEncodeTiled", &ptr, 12000, cudaEnableDefault,
-                                       &q) != cudaSuccess ||
-      q != cudaDriverEntryPointSuccess)
-    return nullptr;
-  fn = reinterpret_cast<EncodeTiledFn>(ptr);
+  static const EncodeTiledFn fn =
+      reinterpret_cast<EncodeTiledFn>(driver_entry("cuTensorMapEncodeTiled"));
   return fn;
 }
 

@@ -160,6 +160,26 @@ def _ptr(x) -> int | None:
     return x.data_ptr()
 
 
+def _buf(x, what: str, dtype: str) -> int | None:
+    """Address of a buffer the library reads or writes as a dense array of
+    ``dtype`` ("bfloat16", "float32" or "int32"): a tensor or array of that
+    element type with a contiguous layout, or a raw address (int).  A wrong
+    element type or a strided view raises instead of being read as garbage."""
+    if x is None or isinstance(x, int):
+        return x
+    if isinstance(x, np.ndarray):
+        # numpy has no bfloat16: such buffers travel as their uint16 bits
+        want = {"bfloat16": np.uint16, "float32": np.float32, "int32": np.int32}[dtype]
+        if x.dtype != want or not x.flags["C_CONTIGUOUS"]:
+            raise ValueError(f"{what}: expected a C-contiguous {np.dtype(want)} array "
+                             f"(got {x.dtype}, contiguous={x.flags['C_CONTIGUOUS']})")
+        return x.ctypes.data
+    if str(x.dtype) != f"torch.{dtype}" or not x.is_contiguous():
+        raise ValueError(f"{what}: expected a contiguous torch.{dtype} tensor "
+                         f"(got {x.dtype}, contiguous={x.is_contiguous()})")
+    return x.data_ptr()
+
+
 def _stream(s) -> int | None:
     if s is None:
         import torch
@@ -196,10 +216,17 @@ class Ctx:
     def L(self) -> int:
         return self.cfg.n_blocks * self.cfg.P
 
+    def __enter__(self) -> "Ctx":
+        return self
+
+    def __exit__(self, *exc) -> None:
+        cai_free(self)
+
 
 def cai_init(cfg: cai_config, W, stream=None) -> Ctx:
     h = ctypes.c_void_p()
-    _check(lib().cai_init(ctypes.byref(cfg), _ptr(W), _stream(stream), ctypes.byref(h)), "cai_init")
+    _check(lib().cai_init(ctypes.byref(cfg), _buf(W, "W", "bfloat16"), _stream(stream),
+                          ctypes.byref(h)), "cai_init")
     return Ctx(h.value, cfg, W)
 
 
@@ -207,17 +234,20 @@ def cai_init_rmsnorm(cfg: cai_config, W, norm_weight, eps: float, stream=None) -
     """cai_init with the model's final RMSNorm (weight ``norm_weight`` [H] bf16,
     epsilon ``eps``) applied to every decoded row inside the head."""
     h = ctypes.c_void_p()
-    _check(lib().cai_init_rmsnorm(ctypes.byref(cfg), _ptr(W), _ptr(norm_weight), float(eps),
+    _check(lib().cai_init_rmsnorm(ctypes.byref(cfg), _buf(W, "W", "bfloat16"),
+                                  _buf(norm_weight, "norm_weight", "bfloat16"), float(eps),
                                   _stream(stream), ctypes.byref(h)), "cai_init_rmsnorm")
     return Ctx(h.value, cfg, W, norm_weight, float(eps))
 
 
 def cai_first_step(ctx: Ctx, hidden, stream=None) -> None:
-    _check(lib().cai_first_step(ctx.handle, _ptr(hidden), _stream(stream)), "cai_first_step")
+    _check(lib().cai_first_step(ctx.handle, _buf(hidden, "hidden", "bfloat16"), _stream(stream)),
+           "cai_first_step")
 
 
 def cai_denoise_step(ctx: Ctx, hidden, stream=None) -> None:
-    _check(lib().cai_denoise_step(ctx.handle, _ptr(hidden), _stream(stream)), "cai_denoise_step")
+    _check(lib().cai_denoise_step(ctx.handle, _buf(hidden, "hidden", "bfloat16"), _stream(stream)),
+           "cai_denoise_step")
 
 
 def cai_block_advance(ctx: Ctx, stream=None) -> None:
@@ -278,7 +308,8 @@ def cai_state_upload(ctx: Ctx, state: dict) -> None:
 
 
 def cai_read_tokens(ctx: Ctx, host_tokens, stream=None) -> None:
-    _check(lib().cai_read_tokens(ctx.handle, _ptr(host_tokens), _stream(stream)), "cai_read_tokens")
+    _check(lib().cai_read_tokens(ctx.handle, _buf(host_tokens, "host_tokens", "int32"),
+                                 _stream(stream)), "cai_read_tokens")
 
 
 def cai_profile(ctx: Ctx, enable: bool) -> None:
@@ -329,8 +360,10 @@ def cai_head_rows_static(W, rows, conf, argmax, stream=None) -> None:
     allocating nothing (see include/cai.h)."""
     V, H = W.shape
     M = rows.shape[0]
-    _check(lib().cai_head_rows_static(_ptr(W), V, H, _ptr(rows), M, _ptr(conf), _ptr(argmax),
-                                      _stream(stream)), "cai_head_rows_static")
+    _check(lib().cai_head_rows_static(_buf(W, "W", "bfloat16"), V, H, _buf(rows, "rows", "bfloat16"),
+                                      M, _buf(conf, "conf", "float32"),
+                                      _buf(argmax, "argmax", "int32"), _stream(stream)),
+           "cai_head_rows_static")
 
 
 def config_from_dict(d: dict) -> cai_config:

@@ -186,3 +186,34 @@ def test_bench_reference_arm_json_line():
     cb = line["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == line["value"]
     assert line["e2e"]["h2d_bytes_per_step"] == 0 and line["e2e"]["value"] == line["value"]
+
+
+def test_binding_rejects_wrong_element_types_and_strided_views():
+    # The library reads W and the hidden states as dense bf16, the tokens as
+    # int32: the binding raises on anything else instead of passing a pointer.
+    import numpy as np
+    import torch
+    from paper_2608_22646_gb300 import _buf
+    w = torch.zeros((8, 64), dtype=torch.bfloat16)
+    assert _buf(w, "W", "bfloat16") == w.data_ptr()
+    assert _buf(1234, "W", "bfloat16") == 1234 and _buf(None, "W", "bfloat16") is None
+    for bad in (w.float(), w.half(), w.t(), w[:, ::2]):
+        with pytest.raises(ValueError):
+            _buf(bad, "W", "bfloat16")
+    bits = np.zeros((8, 64), np.uint16)
+    assert _buf(bits, "W", "bfloat16") == bits.ctypes.data
+    with pytest.raises(ValueError):
+        _buf(bits[:, ::2], "W", "bfloat16")
+    with pytest.raises(ValueError):
+        _buf(np.zeros(8, np.float32), "W", "bfloat16")
+    tok = torch.zeros((2, 5), dtype=torch.int32)
+    assert _buf(tok, "host_tokens", "int32") == tok.data_ptr()
+    with pytest.raises(ValueError):
+        _buf(tok.long(), "host_tokens", "int32")
+
+
+def test_context_handle_frees_on_exit():
+    c = cai.cai_config_default(0, 1, 16, 256, 4096, 8, 4)
+    with cai.Ctx(0, c, None) as ctx:     # a null handle: nothing to free
+        assert ctx.L == 64
+    assert ctx.handle == 0

@@ -5,8 +5,9 @@ decoding head (Box 1) and the confidence-aware controller (Boxes 2-7,
 Algorithm 1) of arXiv 2608.22646, plus the block loop of Algorithm 1 run over a
 batch in lockstep.
 
-Only ``tests/``, ``__graft_entry__.smoke()`` and the CPU-baseline leg of
-``bench.py`` may import this package.  It shares no code with the CUDA path and
+Only ``tests/``, ``__graft_entry__.smoke()``, the CPU-baseline leg and the
+reference arm of ``bench.py``, and ``calibrate_synth.py`` beside this file may
+import this package.  It shares no code with the CUDA path and
 never imports it.  bf16 tensors cross this boundary as ``uint16`` bit patterns.
 
 Parity status of each function (what pins it, beyond itself) is listed in

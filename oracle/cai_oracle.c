@@ -22,8 +22,9 @@
  * each row is computed by one thread from start to end.
  *
  * Nothing under the product package includes, links or calls this file, and
- * this file includes nothing from it.  Only the tests, the smoke check and
- * the CPU-baseline leg of the benchmark load it.
+ * this file includes nothing from it.  Only the tests, the smoke check, the
+ * benchmark's CPU-baseline leg and reference arm, and the generator
+ * calibration script beside this file load it.
  *
  * Readings of points the paper leaves open (each selectable by a flag):
  *   - eta_bar (Box 7): count mode reads "eta < 1.5" as a count of newly

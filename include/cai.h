@@ -383,6 +383,17 @@ int cai_test_wait_timeout(cai_ctx* ctx, void* stream);
  */
 int cai_test_pair_plan(int32_t M, int32_t n_pairs, int32_t swap_max_n, int32_t* out);
 
+/*
+ * Testing hook, host only (no device use): the position thresholds
+ * theta_i(t) (Box 6, Eq. position_threshold: the block threshold of Boxes 3
+ * and 4 times the position factor, clipped to [clip_lo, clip_hi]) that a step
+ * of block blk (0-based) at local step t hands to the commit rule, one fp32
+ * value per position p < P into out[P].  Computed in double and rounded once,
+ * exactly as for the step.  CAI_ERR_ARG for a null pointer, blk outside
+ * [0, n_blocks) or t outside [0, T); otherwise cai_init's configuration checks.
+ */
+int cai_test_theta_table(const cai_config* cfg, int32_t blk, int32_t t, float* out);
+
 #ifdef __cplusplus
 }
 #endif

@@ -52,7 +52,7 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_block_advance", "cai_reset", "cai_poll", "cai_get_state", "cai_state_download",
            "cai_state_upload", "cai_read_tokens", "cai_profile", "cai_get_stats", "cai_free",
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
-           "cai_test_pair_plan", "cai_test_wait_timeout",
+           "cai_test_pair_plan", "cai_test_theta_table", "cai_test_wait_timeout",
            "cai_test_check_guards",
            "cai_head_rows_static")
 
@@ -124,6 +124,8 @@ def _load():
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
         "cai_test_head_grid_limit": (ctypes.c_int, [i32]),
         "cai_test_pair_plan": (ctypes.c_int, [i32, i32, i32, ctypes.POINTER(i32)]),
+        "cai_test_theta_table": (ctypes.c_int, [ctypes.POINTER(cai_config), i32, i32,
+                                                ctypes.POINTER(ctypes.c_float)]),
         "cai_test_wait_timeout": (ctypes.c_int, [vp, vp]),
         "cai_test_check_guards": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
         "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
@@ -341,6 +343,16 @@ def cai_test_pair_plan(M: int, n_pairs: int, swap_max_n: int) -> dict:
     _check(lib().cai_test_pair_plan(M, n_pairs, swap_max_n, out), "cai_test_pair_plan")
     return {"swapped": bool(out[0]), "row_tiles": out[1], "tile_rows": out[2],
             "partials_per_row": out[3]}
+
+
+def cai_test_theta_table(cfg: cai_config, blk: int, t: int) -> np.ndarray:
+    """theta_i(t) of every position of block ``blk`` at local step ``t``, as
+    the step's commit rule receives it (fp32)."""
+    out = np.zeros(cfg.P, np.float32)
+    _check(lib().cai_test_theta_table(ctypes.byref(cfg), blk, t,
+                                      out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))),
+           "cai_test_theta_table")
+    return out
 
 
 def cai_test_head_grid_limit(n: int) -> None:

@@ -359,6 +359,16 @@ double pos_factor_of(const cai_config& c, int p) {
   return p < q1 ? 0.80 : p < q2 ? 0.90 : p < q3 ? 1.05 : 1.10;
 }
 
+// theta_i(t) of position p in block b1 (1-based), Eq. position_threshold:
+// the block's threshold times the position factor, clipped, in double, then
+// rounded once to the fp32 value the commit rule compares against.
+float theta_token_of(const cai_config& c, int b1, int t, int p) {
+  double th = theta_block_of(c, b1, t) * pos_factor_of(c, p);
+  th = th < c.clip_lo ? c.clip_lo : th;
+  th = th > c.clip_hi ? c.clip_hi : th;
+  return static_cast<float>(th);
+}
+
 CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   const cai_config& cfg = c->cfg;
   CommitParams cp{};
@@ -393,13 +403,7 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   cp.budget_half = (cfg.flags & CAI_QUARTER_POS) ? cfg.P / 2 : 32;
   cp.budget_late = (cfg.flags & CAI_QUARTER_POS) ? 3 * cfg.P / 4 : 48;
   cp.flags = cfg.flags;
-  const double tb = theta_block_of(cfg, c->blk + 1, t);
-  for (int p = 0; p < cfg.P; ++p) {
-    double th = tb * pos_factor_of(cfg, p);
-    th = th < cfg.clip_lo ? cfg.clip_lo : th;
-    th = th > cfg.clip_hi ? cfg.clip_hi : th;
-    cp.theta_tab[p] = static_cast<float>(th);
-  }
+  for (int p = 0; p < cfg.P; ++p) cp.theta_tab[p] = theta_token_of(cfg, c->blk + 1, t, p);
   return cp;
 }
 
@@ -1320,6 +1324,15 @@ int cai_test_pair_plan(int32_t M, int32_t n_pairs, int32_t swap_max_n, int32_t* 
   out[1] = n_rt;
   out[2] = swap ? swap_tile_cols(M, n_rt) : kPairTileRows;
   out[3] = pair_partials_per_row(M, n_pairs, swap);
+  return CAI_OK;
+}
+
+int cai_test_theta_table(const cai_config* cfg, int32_t blk, int32_t t, float* out) {
+  if (!cfg || !out) return CAI_ERR_ARG;
+  const int r = validate(cfg);
+  if (r != CAI_OK) return r;
+  if (blk < 0 || blk >= cfg->n_blocks || t < 0 || t >= cfg->T) return CAI_ERR_ARG;
+  for (int p = 0; p < cfg->P; ++p) out[p] = theta_token_of(*cfg, blk + 1, t, p);
   return CAI_OK;
 }
 

@@ -7,6 +7,7 @@ import re
 import subprocess
 import tempfile
 
+import numpy as np
 import pytest
 
 import paper_2608_22646_gb300 as cai
@@ -191,7 +192,6 @@ def test_bench_reference_arm_json_line():
 def test_binding_rejects_wrong_element_types_and_strided_views():
     # The library reads W and the hidden states as dense bf16, the tokens as
     # int32: the binding raises on anything else instead of passing a pointer.
-    import numpy as np
     import torch
     from paper_2608_22646_gb300 import _buf
     w = torch.zeros((8, 64), dtype=torch.bfloat16)
@@ -217,3 +217,63 @@ def test_context_handle_frees_on_exit():
     with cai.Ctx(0, c, None) as ctx:     # a null handle: nothing to free
         assert ctx.L == 64
     assert ctx.handle == 0
+
+
+def _golden(name):
+    out = []
+    with open(os.path.join(os.path.dirname(os.path.abspath(__file__)), "golden", name)) as f:
+        for line in f:
+            line = line.strip()
+            if line and not line.startswith("#"):
+                out.append(line.split())
+    return out
+
+
+def test_theta_table_matches_golden_schedule_and_position_factors():
+    # The product's host-side threshold table (what the commit rule receives)
+    # against the hand-worked Box 3-4 schedule and the printed Box 6 factors.
+    for T, b, t, th in _golden("theta_schedule.txt"):
+        T, b, t, th = int(T), int(b), int(t), float(th)
+        c = cai.cai_config_default(0, 1, 16, 256, 4096, T, max(4, b))
+        c.flags = 0                                   # no position factors
+        tab = cai.cai_test_theta_table(c, b - 1, t)
+        assert abs(float(tab[0]) - th) <= 6e-7, (T, b, t, tab[0], th)
+        assert np.all(tab == tab[0])
+    c = cai.cai_config_default(0, 1, 64, 256, 4096, 32, 4)   # t = 0: theta = theta_s = 0.9
+    tab = cai.cai_test_theta_table(c, 0, 0)
+    for p, r in _golden("position_factors.txt"):
+        want = min(max(0.9 * float(r), 0.20), 0.98)
+        assert abs(float(tab[int(p)]) - want) <= 1e-7, (p, tab[int(p)], want)
+
+
+@pytest.mark.parametrize("flags", [0, 2, 2 | 8, 2 | 16, 2 | 32, 2 | 64, 1 | 2])
+def test_theta_table_matches_oracle(flags):
+    # Every position, block and step of several shapes against the oracle's
+    # fp64 theta_i(t) rounded to fp32 (one rounding on each side).
+    import oracle
+    from tests import parity
+    for P, T, nb in ((16, 8, 3), (32, 32, 8), (50, 20, 6), (64, 64, 16)):
+        c = cai.cai_config_default(0, 2, P, 256, 4096, T, nb)
+        c.flags = flags
+        ocfg = parity.oracle_config(c)
+        for blk in range(nb):
+            for t in range(T):
+                tab = cai.cai_test_theta_table(c, blk, t)
+                want = np.array([oracle.theta_token(ocfg, blk + 1, t, p) for p in range(P)],
+                                np.float32)
+                ulp = np.spacing(want)
+                assert np.all(np.abs(tab - want) <= ulp), (P, T, blk, t, flags)
+
+
+def test_theta_table_arguments():
+    c = cai.cai_config_default(0, 1, 16, 256, 4096, 8, 2)
+    lib = cai.lib()
+    out = np.zeros(16, np.float32)
+    ptr = out.ctypes.data_as(ctypes.POINTER(ctypes.c_float))
+    assert lib.cai_test_theta_table(ctypes.byref(c), 2, 0, ptr) == cai.CAI_ERR_ARG
+    assert lib.cai_test_theta_table(ctypes.byref(c), 0, 8, ptr) == cai.CAI_ERR_ARG
+    assert lib.cai_test_theta_table(ctypes.byref(c), -1, 0, ptr) == cai.CAI_ERR_ARG
+    assert lib.cai_test_theta_table(None, 0, 0, ptr) == cai.CAI_ERR_ARG
+    assert lib.cai_test_theta_table(ctypes.byref(c), 0, 0, None) == cai.CAI_ERR_ARG
+    c.P = 0
+    assert lib.cai_test_theta_table(ctypes.byref(c), 0, 0, ptr) == cai.CAI_ERR_SHAPE

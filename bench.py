@@ -514,10 +514,8 @@ def run_reference(args, wl):
         while True:
             b, t = order[pos % len(order)]
             pos += 1
-            if t == 0:
-                if b == 0:
-                    st.__init__(cfg)
-                st.ell[:] = 0
+            if t == 0 and b == 0:
+                st.__init__(cfg)
             if np.all(st.exit_reason[:, b] != 0):
                 continue
             h = oracle.bf16_bits(hs(b, t))

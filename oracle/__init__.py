@@ -328,7 +328,7 @@ def run_trajectory(cfg: Config, W, hidden_fn, n_threads: int | None = None, on_s
     every step (tests use it to compare or re-synchronise state)."""
     st = State(cfg)
     for blk in range(cfg.n_blocks):
-        st.ell[:] = 0
+        # (the controller itself sets ell <- 0 at each block's step zero)
         for t in range(cfg.T):
             out = step(st, W, hidden_fn(blk, t), blk, t, n_threads)
             if on_step is not None:

@@ -452,6 +452,38 @@ def test_trajectory_G2_counter_reset():
     assert st.exit_reason[0, 0] == oracle.EXIT_GRIND and st.exit_step[0, 0] == 5
 
 
+@pytest.mark.parametrize("T,ending", [(8, oracle.EXIT_DONE), (3, oracle.EXIT_TMAX)])
+def test_low_yield_counter_resets_at_each_block(T, ending):
+    # Algorithm 1 sets ell <- 0 before each block's first step.  Block 0 commits
+    # one token per step (eta = 1 < 1.5: ell = 1, 2, 3) and ends with ell = 3,
+    # by DONE (P = 3, all committed at t = 2) or by T exhaustion (P = 4, T = 3).
+    # Block 1's step zero commits nothing: with the reset ell = 1 and the block
+    # runs on; without it ell = 4 = K and the block would exit by grinding at
+    # t = 0.  The steps are fed to controller_step directly, so no caller-side
+    # reset can stand in for the oracle's own.
+    P = 3 if ending == oracle.EXIT_DONE else 4
+    cfg = oracle.Config(B=1, P=P, T=T, n_blocks=2)
+    idx = np.asarray([list(range(20, 20 + P))], np.int32)
+    st = oracle.State(cfg)
+    for t in range(3):
+        c = np.full((1, P), 0.1)
+        c[0, t] = 0.99                       # one commit per step (theta <= 0.90 * 1.0)
+        oracle.controller_step(st, 0, t, c, idx)
+        assert st.ell[0] == t + 1
+    assert st.exit_reason[0, 0] == ending and st.exit_step[0, 0] == 2 and st.ell[0] == 3
+    ells = []
+    for t in range(min(T, 4)):
+        oracle.controller_step(st, 1, t, np.full((1, P), 0.1), idx)
+        ells.append(int(st.ell[0]))
+        if t == 0:
+            assert st.exit_reason[0, 1] == oracle.RUNNING, "ell carried over from block 0"
+    assert ells == [1, 2, 3, 4][:len(ells)]
+    if T >= 4:
+        assert st.exit_reason[0, 1] == oracle.EXIT_GRIND and st.exit_step[0, 1] == 3
+    # block 0's record is left as it was
+    assert st.exit_reason[0, 0] == ending and list(st.tok[0, :3]) == [20, 21, 22]
+
+
 def _budget_force_seq(P, T):
     # token 0: s = 0.6 at p = 0 -> B = 8; c stays 0.5 < theta.  Tokens 1..P-1
     # commit two per step (c = 0.99) so the low-yield counter stays at 0.

@@ -180,6 +180,29 @@ def head_rows(W, rows, n_threads: int | None = None, norm_weight=None, eps: floa
     return out
 
 
+def head_rows_shard(W_shard, rows, v0: int, n_threads: int | None = None) -> dict:
+    """Box 1's three reductions over one slice of the vocabulary, the rows
+    [v0, v0 + V_shard) of W held as ``W_shard`` [V_shard, H] (bf16): per row
+    m = max_v z_v over the slice, S = sum over the slice of exp(z_v - m), and
+    idx = the lowest (global) index v of the slice with z_v = m.  The
+    vocabulary-parallel head computes these on every shard and merges them
+    (``merge_shards``)."""
+    h = head_rows(W_shard, rows, n_threads)
+    return {"m": h["zmax"], "S": 1.0 / h["conf"], "idx": h["idx"].astype(np.int64) + int(v0)}
+
+
+def merge_shards(parts) -> dict:
+    """Box 1 over the whole vocabulary from the reductions of the slices of
+    any partition of it (``head_rows_shard`` of each): m = max_k m_k,
+    S = sum_k S_k exp(m_k - m), the argmax the lowest idx_k among the slices
+    whose m_k equals m (ties keep the lowest index), c = 1 / S."""
+    m = np.max(np.stack([p["m"] for p in parts]), axis=0)
+    S = np.sum(np.stack([p["S"] * np.exp(p["m"] - m) for p in parts]), axis=0)
+    big = np.iinfo(np.int64).max
+    idx = np.min(np.stack([np.where(p["m"] == m, p["idx"], big) for p in parts]), axis=0)
+    return {"conf": 1.0 / S, "idx": idx.astype(np.int32), "zmax": m, "lse": m + np.log(S)}
+
+
 def softmax_row(W, h):
     """Logits and full probability vector of one row (Box 1)."""
     Wb, hb = bf16_bits(W), bf16_bits(h).reshape(-1)

@@ -18,8 +18,12 @@ Coverage map (function -> pins):
   cai_o_budget             -> Box 5 hand table, boundaries
   cai_o_low_yield          -> count and fraction readings
   cai_o_controller_step    -> hand trajectories G1, G2, budget force,
-                              DONE, T-exhausted, flush, gating OFF, and
+                              DONE, T-exhausted, flush, gating OFF, the
+                              low-yield reset at each block's step zero, and
                               invariants over synthetic trajectories
+  head_rows_shard,         -> equal to the full-vocabulary head for several
+  merge_shards                partitions, a tie across a shard boundary,
+                              the two-row closed form
 """
 import math
 import os
@@ -615,3 +619,64 @@ def test_theta_e_non_increasing_in_trajectory_configs():
         cfg = oracle.Config(n_blocks=nb)
         vals = [oracle.theta_e(cfg, b) for b in range(1, nb + 1)]
         assert all(x >= y for x, y in zip(vals, vals[1:]))
+
+
+# ------------------------------------------------- vocabulary-parallel head --
+
+def _random_bf16(shape, scale, seed):
+    rng = np.random.default_rng(seed)
+    return bf16_from_float(rng.normal(0.0, scale, shape).astype(np.float32))
+
+
+@pytest.mark.parametrize("cuts", [[], [500], [1, 999], [128, 333, 640], [7, 8, 9, 500, 990]])
+def test_vocab_shards_merge_to_the_full_vocabulary(cuts):
+    # Any partition of the vocabulary: the merged slice reductions equal Box 1
+    # over the whole vocabulary (itself pinned by brute force above): the same
+    # maximum and argmax, confidence and log-sum-exp to rounding.
+    V, H, M = 1000, 64, 40
+    W = _random_bf16((V, H), 0.05, 11)
+    rows = _random_bf16((M, H), 1.0, 12)
+    full = oracle.head_rows(W, rows)
+    edges = [0] + cuts + [V]
+    parts = [oracle.head_rows_shard(W[a:b], rows, a) for a, b in zip(edges[:-1], edges[1:])]
+    got = oracle.merge_shards(parts)
+    assert np.array_equal(got["idx"], full["idx"])
+    assert np.array_equal(got["zmax"], full["zmax"])
+    np.testing.assert_allclose(got["conf"], full["conf"], rtol=1e-12, atol=0)
+    np.testing.assert_allclose(got["lse"], full["lse"], rtol=1e-12, atol=0)
+
+
+def test_vocab_shards_tie_across_a_shard_boundary_keeps_the_lower_index():
+    # Rows 37 and 537 of W are equal, and each hidden row points along them:
+    # both logits are the maximum, in different shards.  The argmax is the
+    # lower index (Box 1 with the lowest-index reading of ties), and c = 1/2
+    # up to the other rows' tiny mass.
+    V, H = 1000, 64
+    W = _random_bf16((V, H), 0.02, 21)
+    W[537] = W[37]
+    w37 = np.frombuffer((W[37].astype(np.uint32) << 16).tobytes(), np.float32)
+    rows = np.stack([bf16_from_float(w37 * 400.0 * (1 + 0.1 * k)) for k in range(3)])
+    full = oracle.head_rows(W, rows)
+    assert list(full["idx"]) == [37, 37, 37]
+    parts = [oracle.head_rows_shard(W[:500], rows, 0), oracle.head_rows_shard(W[500:], rows, 500)]
+    assert list(parts[1]["idx"]) == [537, 537, 537]
+    got = oracle.merge_shards(parts)
+    assert list(got["idx"]) == [37, 37, 37]
+    np.testing.assert_allclose(got["conf"], full["conf"], rtol=1e-12)
+    assert np.all(np.abs(got["conf"] - 0.5) < 1e-3)
+    # the same split in the other order of the slices
+    got2 = oracle.merge_shards(parts[::-1])
+    assert list(got2["idx"]) == [37, 37, 37]
+
+
+def test_vocab_shard_two_way_closed_form():
+    # Two one-row slices: z = (a, b), so S over the whole vocabulary is
+    # 1 + exp(-|a - b|) and c = sigma(|a - b|), whatever slice holds the max.
+    H = 4
+    for a, b in ((1.0, 0.0), (0.0, 2.5), (3.0, 3.0)):
+        W = bf16_from_float(np.array([[a, 0, 0, 0], [b, 0, 0, 0]], np.float32))
+        h = bf16_from_float(np.array([[1, 0, 0, 0]], np.float32))
+        got = oracle.merge_shards([oracle.head_rows_shard(W[:1], h, 0),
+                                   oracle.head_rows_shard(W[1:], h, 1)])
+        assert got["conf"][0] == pytest.approx(1.0 / (1.0 + math.exp(-abs(a - b))), rel=1e-15)
+        assert got["idx"][0] == (0 if a >= b else 1)

@@ -232,6 +232,185 @@ def aggregate(ms: float, positions: int, dist=None, device=None):
     return float(t.item()), int(n.item())
 
 
+def _roofline(wl, st0, stats1, head_ms, head_launches, step_ms, ms, steps, steps_issued,
+              profiled):
+    """Roofline of the dominant kernel (the LM head), launch by launch: a
+    launch that decodes M rows reads 2 V H + 2 M H bytes (W once, the rows
+    once) and does 2 M V H flops; its roof is the slower of the two at the
+    measured peaks.  Launches of empty steps (M = 0) have no algorithmic work.
+
+    achieved / frac: algorithmic work per launch / the LM head's average
+    launch duration, from CUDA events around every LM-head launch on its
+    stream (the profiled pass: each launch runs alone, with its launch latency
+    and, in single-kernel steps, the commit tail; this is the figure that
+    carries over to a decoder whose model forward runs between two steps).
+    live: the same work over the timed region of back-to-back generations
+    times the LM head's share of step time (consecutive steps overlap there)."""
+    hbm, tf_burst, tf_sus, peak_kind = _peaks()
+    tf = tf_sus or tf_burst
+    m_t = [int(x) for x in st0["m_hist"].reshape(-1) if x > 0]
+    bytes_t = [2.0 * wl.V * wl.H + 2.0 * m * wl.H for m in m_t]
+    flops_t = [2.0 * m * wl.V * wl.H for m in m_t]
+    t_hbm = sum(b / (hbm * 1e9) for b in bytes_t)
+    t_tc = sum(f / (tf * 1e12) for f in flops_t)
+    t_roof = sum(max(b / (hbm * 1e9), f / (tf * 1e12)) for b, f in zip(bytes_t, flops_t))
+    share = min(1.0, head_ms / step_ms) if step_ms > 0 else 1.0
+    head_live_s = ms / 1e3 / steps * share
+    head_iso_s = (head_ms / 1e3 / steps) if profiled and head_ms > 0 else head_live_s
+    per_launch = max(1, (head_launches if head_launches else int(steps_issued) * steps) // steps)
+    kps = int(stats1["kernels_per_step"])
+    if kps == 1:
+        kernel = "lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
+    elif stats1["pair_swap_max_n"] >= 32:
+        kernel = (f"lm_head_pair_kernel (every step; swapped orientation for tiles up to "
+                  f"{stats1['pair_swap_max_n']} rows wide)")
+    elif stats1["pair_grid"]:
+        kernel = "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows)"
+    else:
+        kernel = "lm_head_softmax_kernel"
+    tr = _traffic_record(wl.name)
+    hb = t_hbm >= t_tc
+    work = sum(bytes_t) if hb else sum(flops_t)
+    scale = 1e9 if hb else 1e12
+    peak = hbm if hb else tf
+    achieved = work / head_iso_s / scale
+    live = work / head_live_s / scale
+    roof = {"bound": "hbm" if hb else "tensor", "achieved": round(achieved, 1), "peak": peak,
+            "unit": "GB/s" if hb else "TFLOP/s", "frac": round(achieved / peak, 4),
+            "traffic": tr["dram_bytes_per_launch"] if tr else None,
+            "traffic_basis": ("ncu dram read+write of one launch with M = %d (%s); algorithmic "
+                              "bytes of that launch %d" % (
+                                  tr["captured_M"], tr["summary"],
+                                  tr["algorithmic_bytes_of_profiled_launch"])) if tr else None,
+            ("algorithmic_bytes_per_launch" if hb else "algorithmic_flops_per_launch"):
+                round(work / per_launch),
+            "peak_source": f"{peak_kind} " + ("hbm_gbs" if hb else "bf16 sustained"),
+            "kernel": kernel, "head_launches": head_launches,
+            "avg_launch_us": round(head_iso_s / per_launch * 1e6, 2),
+            "roofline_time_frac": round(t_roof / head_iso_s, 4),
+            "live": {"achieved": round(live, 1), "frac": round(live / peak, 4),
+                     "roofline_time_frac": round(t_roof / head_live_s, 4),
+                     "head_share_of_step_time": round(share, 4)},
+            "timing": "achieved/frac: CUDA events around every LM-head launch on its stream in a "
+                      "second pass of the same K generations (each launch alone); live: CUDA "
+                      "events around the timed region of K generations back to back times the "
+                      "LM head's share of step time (consecutive steps overlap under "
+                      "programmatic dependent launch)"}
+    return roof
+
+
+def measure(cai, wl, generator, args, dist, dev, steps, warmup, with_e2e=True, cpu_leg=False):
+    """One workload: `warmup` untimed generations, `steps` timed ones (the
+    value), a profiled pass (the roofline), the end-to-end pass through host
+    buffers, and optionally the oracle's CPU baseline."""
+    import torch
+    import synth
+    rank = int(os.environ.get("RANK", "0"))
+    local = dev.index or 0
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device=dev)
+    hs = synth.HiddenStates(wl, W, generator, seed=wl.seed_h + 1000 * rank)
+    norm = None
+    if args.final_norm:
+        norm = (synth.final_norm_weight(wl.H, device=dev), FINAL_NORM_EPS)
+        hs = synth.PreNormHidden(hs)
+    hidden = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    torch.cuda.synchronize()
+
+    cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    if args.diagnostics:
+        cfg.flags |= cai.CAI_DIAGNOSTICS
+    ctx = cai.cai_init_rmsnorm(cfg, W, *norm) if norm else cai.cai_init(cfg, W)
+    stream = torch.cuda.current_stream(dev)
+
+    for _ in range(warmup):
+        cai.cai_reset(ctx)
+        run_trajectory(cai, ctx, hidden, wl)
+    torch.cuda.synchronize()
+    st0 = cai.cai_state_download(ctx)
+    positions = int(st0["m_hist"].sum())
+    nonzero_launch = int((st0["m_hist"] > 0).sum())   # steps that decoded rows
+    stats0 = cai.cai_get_stats(ctx)
+
+    # Timed region 1 (the value): K generations back to back, device time by
+    # CUDA events on the stream, no per-kernel events in between (an event
+    # between two kernels serialises them and would defeat the programmatic
+    # dependent launch the library uses).
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    with Clocks(local) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(steps):
+            cai.cai_reset(ctx)
+            run_trajectory(cai, ctx, hidden, wl)
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    stats1 = cai.cai_get_stats(ctx)
+    st1 = cai.cai_state_download(ctx)
+    assert np.array_equal(st1["m_hist"], st0["m_hist"]), "trajectory changed between runs"
+    gpu_launches = stats1["launches"] - stats0["launches"]
+    steps_issued = (stats1["steps"] - stats0["steps"]) // steps
+
+    # Timed region 2 (the roofline figure): the same K generations with CUDA
+    # events around every step and its LM-head launch(es) on the stream.
+    head_ms, head_launches, step_ms = 0.0, 0, 0.0
+    if not args.no_profile:
+        cai.cai_profile(ctx, True)
+        torch.cuda.synchronize()
+        for _ in range(steps):
+            cai.cai_reset(ctx)
+            run_trajectory(cai, ctx, hidden, wl)
+        torch.cuda.synchronize()
+        cai.cai_profile(ctx, False)
+        stats2 = cai.cai_get_stats(ctx)
+        head_launches = stats2["head_launches"] - stats1["head_launches"]
+        head_ms = stats2["head_ms"] - stats1["head_ms"]
+        step_ms = stats2["step_ms"] - stats1["step_ms"]
+
+    ms, total_positions = aggregate(ms, positions * steps, dist, dev)
+    rec = {
+        "value": round(total_positions / (ms / 1e3), 1), "unit": UNIT,
+        "ms_per_generation": round(ms / steps, 4),
+        "ms_per_step_call": round(ms / steps / max(1, steps_issued), 5),
+        "config": {**_workload_desc(wl, generator),
+                   "final_norm_in_head": bool(args.final_norm),
+                   "positions_per_generation": positions,
+                   "denoising_steps_per_generation": nonzero_launch,
+                   "step_calls_per_generation": int(steps_issued)},
+        "roofline": _roofline(wl, st0, stats1, head_ms, head_launches, step_ms, ms, steps,
+                              steps_issued, not args.no_profile),
+        "trajectory": _trajectory_summary(st0),
+        "gpu_launches": int(gpu_launches),
+        "clocks": clk.summary(),
+    }
+    if args.diagnostics:
+        rec["config"]["diagnostics"] = True
+        rec["diagnostics"] = _diagnostics_summary(st0)
+    if with_e2e and not args.no_e2e:
+        rec["e2e"] = e2e_run(cai, ctx, hs, wl, max(3, steps // 3), dist, dev)
+    if cpu_leg:
+        rec["cpu_baseline"] = cpu_baseline(wl, W, lambda b, t: hidden[b][t], norm=norm)
+    cai.cai_free(ctx)
+    del hidden, W, hs
+    torch.cuda.synchronize()
+    torch.cuda.empty_cache()
+    return rec
+
+
+# The other configurations measured beside the headline workload (N = 1):
+# name in the line -> (workload, hidden-state generator).
+EXTRA_WORKLOADS = {
+    "dream": ("dream", "calibrated"),
+    "llada_batched": ("llada_batched", "calibrated"),
+    "dream_long": ("dream_long", "calibrated"),
+    "llada_literal": ("llada", "literal"),
+}
+
+
 def main():
     ap = argparse.ArgumentParser()
     ap.add_argument("--gpus", type=int, default=1)
@@ -240,6 +419,9 @@ def main():
     ap.add_argument("--impl", default="ours", choices=["ours", "reference"])
     ap.add_argument("--workload", default="llada")
     ap.add_argument("--generator", default="calibrated", choices=["calibrated", "literal"])
+    ap.add_argument("--extra", default=None,
+                    help="comma-separated names of EXTRA_WORKLOADS measured beside the headline "
+                         "(default: all of them at N = 1 on the default workload, none otherwise)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     ap.add_argument("--no-e2e", action="store_true")
     ap.add_argument("--no-profile", action="store_true",
@@ -282,172 +464,53 @@ def main():
     cai_build.build()
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
-    stream = torch.cuda.current_stream(dev)
 
-    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device=dev)
-    hs = synth.HiddenStates(wl, W, args.generator, seed=wl.seed_h + 1000 * rank)
-    norm = None
-    if args.final_norm:
-        norm = (synth.final_norm_weight(wl.H, device=dev), FINAL_NORM_EPS)
-        hs = synth.PreNormHidden(hs)
-    hidden = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
-    torch.cuda.synchronize()
-
-    cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
-    if args.diagnostics:
-        cfg.flags |= cai.CAI_DIAGNOSTICS
-    ctx = cai.cai_init_rmsnorm(cfg, W, *norm) if norm else cai.cai_init(cfg, W)
-
-    for _ in range(args.warmup):
-        cai.cai_reset(ctx)
-        run_trajectory(cai, ctx, hidden, wl)
-    torch.cuda.synchronize()
-    st0 = cai.cai_state_download(ctx)
-    positions = int(st0["m_hist"].sum())
-    nonzero_launch = int((st0["m_hist"] > 0).sum())   # steps that decoded rows
-    stats0 = cai.cai_get_stats(ctx)
-
-    # Timed region 1 (the value): K generations back to back, device time by
-    # CUDA events on the stream, no per-kernel events in between (an event
-    # between two kernels serialises them and would defeat the programmatic
-    # dependent launch the library uses).
-    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
-    with Clocks(local) as clk:
-        if dist:
-            dist.barrier()
-        torch.cuda.synchronize()
-        ev0.record(stream)
-        for _ in range(args.steps):
-            cai.cai_reset(ctx)
-            run_trajectory(cai, ctx, hidden, wl)
-        ev1.record(stream)
-        torch.cuda.synchronize()
-        if dist:
-            dist.barrier()
-    ms = ev0.elapsed_time(ev1)
-    stats1 = cai.cai_get_stats(ctx)
-    st1 = cai.cai_state_download(ctx)
-    assert np.array_equal(st1["m_hist"], st0["m_hist"]), "trajectory changed between runs"
-    gpu_launches = stats1["launches"] - stats0["launches"]
-    steps_issued = (stats1["steps"] - stats0["steps"]) // args.steps
-
-    # Timed region 2 (the roofline figure): the same K generations with CUDA
-    # events around every LM-head launch on its stream.
-    head_ms, head_launches, step_ms = 0.0, 0, 0.0
-    if not args.no_profile:
-        cai.cai_profile(ctx, True)
-        torch.cuda.synchronize()
-        for _ in range(args.steps):
-            cai.cai_reset(ctx)
-            run_trajectory(cai, ctx, hidden, wl)
-        torch.cuda.synchronize()
-        cai.cai_profile(ctx, False)
-        stats2 = cai.cai_get_stats(ctx)
-        head_launches = stats2["head_launches"] - stats1["head_launches"]
-        head_ms = stats2["head_ms"] - stats1["head_ms"]
-        step_ms = stats2["step_ms"] - stats1["step_ms"]
-
-    ms, total_positions = aggregate(ms, positions * args.steps, dist, dev)
-    value = total_positions / (ms / 1e3)
-
-    # Roofline of the dominant kernel (LM head), launch by launch: a launch
-    # that decodes M rows reads 2 V H + 2 M H bytes (W once, the rows once) and
-    # does 2 M V H flops; its roof is the slower of the two at the measured
-    # peaks.  Launches of empty steps (M = 0) have no algorithmic work.
-    hbm, tf_burst, tf_sus, peak_kind = _peaks()
-    tf = tf_sus or tf_burst
-    m_t = [int(x) for x in st0["m_hist"].reshape(-1) if x > 0]
-    bytes_t = [2.0 * wl.V * wl.H + 2.0 * m * wl.H for m in m_t]
-    flops_t = [2.0 * m * wl.V * wl.H for m in m_t]
-    t_hbm = sum(b / (hbm * 1e9) for b in bytes_t)
-    t_tc = sum(f / (tf * 1e12) for f in flops_t)
-    t_roof = sum(max(b / (hbm * 1e9), f / (tf * 1e12)) for b, f in zip(bytes_t, flops_t))
-    # LM-head time per generation.  Live: the timed region (no events between
-    # kernels, steps overlapping as they run) times the LM head's share of step
-    # time; the share comes from the event-profiled pass (LM-head launches over
-    # whole steps; 1 for single-kernel steps).  Isolated: the profiled pass's
-    # own LM-head time, each launch bracketed by events and run alone.
-    share = min(1.0, head_ms / step_ms) if step_ms > 0 else 1.0
-    head_s = ms / 1e3 / args.steps * share
-    head_iso_s = max(head_ms, 1e-9) / 1e3 / args.steps
-    tr = _traffic_record(wl.name)
-    per_launch = max(1, (head_launches if head_launches else int(steps_issued) * args.steps)
-                     // max(1, args.steps))
-    kps = int(stats1["kernels_per_step"])
-    if kps == 1:
-        kernel = "lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
-    elif stats1["pair_swap_max_n"] >= 32:
-        kernel = (f"lm_head_pair_kernel (every step; swapped orientation for tiles up to "
-                  f"{stats1['pair_swap_max_n']} rows wide)")
-    elif stats1["pair_grid"]:
-        kernel = "lm_head_pair_kernel (>= 32 rows) / lm_head_softmax_kernel (< 32 rows)"
+    head = measure(cai, wl, args.generator, args, dist, dev, args.steps, args.warmup,
+                   cpu_leg=(rank == 0 and world == 1 and not args.no_cpu_baseline))
+    if args.extra is None:
+        default = (world == 1 and args.workload == "llada" and args.generator == "calibrated"
+                   and not args.final_norm and not args.diagnostics)
+        extra = list(EXTRA_WORKLOADS) if default else []
     else:
-        kernel = "lm_head_softmax_kernel"
-    common = {"kernel": kernel, "head_launches": head_launches,
-              "head_share_of_step_time": round(share, 4),
-              "roofline_time_frac": round(t_roof / head_s, 4),
-              "isolated": None if args.no_profile else
-                          {"head_ms_total": round(head_ms, 3),
-                           "achieved_frac": round((sum(bytes_t) / head_iso_s / 1e9 / hbm)
-                                                  if t_hbm >= t_tc else
-                                                  (sum(flops_t) / head_iso_s / 1e12 / tf), 4),
-                           "roofline_time_frac": round(t_roof / head_iso_s, 4)},
-              "timing": "live: CUDA events around the timed region (K generations back to "
-                        "back) x the LM head's share of step time; the share and the isolated "
-                        "figures come from a second pass of the same K generations with events "
-                        "around every step and its LM-head launch(es) (multi-kernel steps: both "
-                        "LM-head kernels and the row merge)"}
-    traffic = tr["dram_bytes_per_launch"] if tr else None
-    traffic_basis = ("ncu dram read+write of one launch with M = %d (%s); algorithmic bytes of "
-                     "that launch %d" % (tr["captured_M"], tr["summary"],
-                                         tr["algorithmic_bytes_of_profiled_launch"])
-                     if tr else None)
-    if t_hbm >= t_tc:
-        achieved = sum(bytes_t) / head_s / 1e9
-        roof = {"bound": "hbm", "achieved": round(achieved, 1), "peak": hbm, "unit": "GB/s",
-                "frac": round(achieved / hbm, 4),
-                "traffic": traffic, "traffic_basis": traffic_basis,
-                "algorithmic_bytes_per_launch": round(sum(bytes_t) / per_launch),
-                "peak_source": f"{peak_kind} hbm_gbs", **common}
-    else:
-        achieved = sum(flops_t) / head_s / 1e12
-        roof = {"bound": "tensor", "achieved": round(achieved, 1), "peak": tf,
-                "unit": "TFLOP/s", "frac": round(achieved / tf, 4),
-                "traffic": traffic, "traffic_basis": traffic_basis,
-                "algorithmic_flops_per_launch": round(sum(flops_t) / per_launch),
-                "peak_source": f"{peak_kind} bf16 sustained", **common}
+        extra = [x for x in args.extra.split(",") if x]
+    workloads = {}
+    for name in extra:
+        wname, gen = EXTRA_WORKLOADS[name]
+        r = measure(cai, synth.WORKLOADS[wname], gen, args, dist, dev, args.steps, args.warmup)
+        r.pop("trajectory", None)
+        workloads[name] = r
 
+    cfg = head["config"]
     line = {
-        "metric": METRIC, "value": round(value, 1), "unit": UNIT, "n_gpus": world,
-        "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(ms / args.steps, 4),
+        "metric": METRIC, "value": head["value"], "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup,
+        "ms_per_step": head["ms_per_generation"],
+        "step_unit": (f"one bench step = one whole generation of the workload "
+                      f"({cfg['step_calls_per_generation']} step calls, "
+                      f"{cfg['positions_per_generation']} masked positions decoded)"),
+        "ms_per_generation": head["ms_per_generation"],
+        "ms_per_step_call": head["ms_per_step_call"],
         "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "bf16",
         "data": "synthetic (seeded LLaDA/Dream-shaped weight and hidden states; no model weights)",
-        "config": {**_workload_desc(wl, args.generator), "parallelism": f"replicas x{world}",
-                   "final_norm_in_head": bool(args.final_norm),
-                   "positions_per_step": positions,
-                   "denoising_steps_per_generation": nonzero_launch,
-                   "step_calls_per_generation": int(steps_issued)},
-        "roofline": roof,
-        "trajectory": _trajectory_summary(st0),
-        "gpu_launches": int(gpu_launches),
-        "clocks": clk.summary(),
+        "config": {**cfg, "parallelism": f"replicas x{world}",
+                   "positions_per_step": cfg["positions_per_generation"]},
+        "roofline": head["roofline"],
+        "trajectory": head["trajectory"],
+        "gpu_launches": head["gpu_launches"],
+        "clocks": head["clocks"],
     }
-
-    if args.diagnostics:
-        line["config"]["diagnostics"] = True
-        line["diagnostics"] = _diagnostics_summary(st0)
-    if not args.no_e2e:
-        line["e2e"] = e2e_run(cai, ctx, hs, wl, args, dist, dev)
-    if rank == 0 and world == 1 and not args.no_cpu_baseline:
-        line["cpu_baseline"] = cpu_baseline(wl, W, lambda b, t: hidden[b][t], norm=norm)
-    cai.cai_free(ctx)
+    for k in ("diagnostics", "e2e", "cpu_baseline"):
+        if k in head:
+            line[k] = head[k]
+    if workloads:
+        line["workloads"] = workloads
     if rank == 0:
         print(json.dumps(line), flush=True)
     if dist:
         dist.destroy_process_group()
 
 
-def e2e_run(cai, ctx, hs, wl, args, dist, dev):
+def e2e_run(cai, ctx, hs, wl, steps, dist, dev):
     """Same metric through the public C ABI with host buffers: every step's
     hidden states come from pinned host memory (copied inside the step call),
     every step's done flag is read from host-mapped memory, and each
@@ -455,7 +518,6 @@ def e2e_run(cai, ctx, hs, wl, args, dist, dev):
     import torch
     host = [[hs(blk, t).cpu().pin_memory() for t in range(wl.T)] for blk in range(wl.n_blocks)]
     out = torch.empty((wl.B, wl.n_blocks * wl.P), dtype=torch.int32).pin_memory()
-    steps = max(3, args.steps // 3)
     stream = torch.cuda.current_stream(dev)
     cai.cai_reset(ctx)
     run_trajectory(cai, ctx, host, wl)
@@ -533,7 +595,16 @@ def run_reference(args, wl):
     v = rows / dt
     line = {"impl": "reference", "metric": METRIC, "value": round(v, 3), "unit": UNIT,
             "n_gpus": args.gpus, "steps": args.steps, "warmup": args.warmup,
-            "ms_per_step": round(dt / k * 1e3, 3), "higher_is_better": True, "scaling": "weak",
+            "ms_per_step": round(dt / k * 1e3, 3),
+            "step_unit": "one bench step = one denoising step call of the trajectory (every "
+                         "masked row of that step), in trajectory order",
+            "ms_per_step_call": round(dt / k * 1e3, 3),
+            "same_config": {"workload": True, "metric": True, "unit": True,
+                            "differs": "the GPU arm's bench step is a whole generation; this "
+                                       "arm times K step calls of the same trajectory (a "
+                                       "bounded sample): both report masked positions "
+                                       "decoded per second"},
+            "higher_is_better": True, "scaling": "weak",
             "vs_baseline": None, "dtype": "f64", "data": "synthetic",
             "config": {**_workload_desc(wl, args.generator),
                        "final_norm_in_head": bool(args.final_norm)},

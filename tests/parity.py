@@ -191,3 +191,103 @@ def run_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_blocks: int | None = No
                 break
     assert cai.cai_test_check_guards(ctx) == 0, "a device buffer was written past its end"
     return rep, pre
+
+
+def check_controller_step(ocfg: oracle.Config, pre: dict, post: dict, blk: int, t: int) -> int:
+    """Controller-level check of one GPU step (pre -> post): the oracle runs
+    Algorithm 1 from the GPU's pre-step state on the GPU's own confidences and
+    argmaxes, taking each threshold decision in the kernel's fp32 precision;
+    every integer field must then match bit for bit.  Checks the commit rule,
+    budgets, the low-yield counter, exits and M_t at any size, independently
+    of the head (which check_rows_sampled samples).  Returns M_t."""
+    st = to_oracle_state(ocfg, pre)
+    B, P = ocfg.B, ocfg.P
+    sl = slice(blk * P, (blk + 1) * P)
+    mk = st.masked(blk)
+    M = int(mk.sum())
+    assert post["m_hist"][blk, t] == M, (post["m_hist"][blk, t], M)
+    g_conf = post["conf"][:, sl].astype(np.float64)
+    g_cand = post["cand"][:, sl]
+    conf_in = np.where(mk, g_conf, 0.0)
+    th = np.array([oracle.theta_token(ocfg, blk + 1, t, p) for p in range(P)])[None, :]
+    near = mk & ((np.abs(g_conf - th) <= DEC_TOL) | (np.abs(g_conf - ocfg.theta_fb) <= DEC_TOL))
+    for b, p in np.argwhere(near):
+        conf_in[b, p] = kernel_side_value(g_conf[b, p], th[0, p], ocfg.theta_fb)
+    idx_in = np.where(mk, g_cand, -1).astype(np.int32)
+    oracle.controller_step(st, blk, t, conf_in, idx_in)
+    for f in INT_FIELDS:
+        gv = post[f]
+        ov = getattr(st, f)
+        if gv.shape != ov.shape:
+            gv = gv.reshape(ov.shape)
+        if not np.array_equal(gv.astype(np.int64), ov.astype(np.int64)):
+            diff = np.argwhere(gv.astype(np.int64) != ov.astype(np.int64))
+            raise AssertionError(f"field {f} differs at {diff[:6].tolist()} (blk {blk} t {t}): "
+                                 f"gpu {gv[tuple(diff[0])]} oracle {ov[tuple(diff[0])]}")
+    return M
+
+
+def check_rows_sampled(W, hidden_bph, post: dict, blk: int, picks, P: int) -> int:
+    """The head on sampled (b, p) rows of one step, recomputed by the oracle
+    one by one: confidence within 2e-3, argmax where the top-2 gap > 1e-2."""
+    if not len(picks):
+        return 0
+    hb = oracle.bf16_bits(hidden_bph)
+    H = hb.shape[-1]
+    hb = hb.reshape(-1, P, H)
+    rows = np.ascontiguousarray(hb[[b for b, _ in picks], [p for _, p in picks]])
+    o = oracle.head_rows(W, rows)
+    for k, (b, p) in enumerate(picks):
+        g = blk * P + p
+        assert abs(post["conf"][b, g] - o["conf"][k]) <= CONF_TOL, (blk, b, p, post["conf"][b, g],
+                                                                     o["conf"][k])
+        if o["gap"][k] > GAP_TOL:
+            assert post["cand"][b, g] == o["idx"][k], (blk, b, p)
+    return len(picks)
+
+
+def run_controller_checked_trajectory(ctx: cai.Ctx, W, hidden_fn, n_sampled_steps: int,
+                                      rows_per_step: int, seed: int = 0, on_step=None) -> dict:
+    """A whole GPU trajectory, step by step: every step checked at the
+    controller level (check_controller_step); in every block, step zero and
+    n_sampled_steps seeded steps among the block's other steps that ran each
+    get a seeded sample of their masked rows (the first and the last
+    included) recomputed by the oracle (check_rows_sampled).
+    on_step(blk, t, M) sees each step's M_t.  Returns the final state."""
+    import torch
+    c = ctx.cfg
+    ocfg = oracle_config(c)
+    rng = np.random.default_rng(seed)
+    W_host = oracle.bf16_bits(W)
+    pre = cai.cai_state_download(ctx)
+    for blk in range(c.n_blocks):
+        if blk:
+            cai.cai_block_advance(ctx)
+        ran = []  # (t, hidden, post, masked (b, p) list) of every step that decoded rows
+        for t in range(c.T):
+            h = hidden_fn(blk, t)
+            (cai.cai_first_step if t == 0 else cai.cai_denoise_step)(ctx, h)
+            torch.cuda.synchronize()
+            post = cai.cai_state_download(ctx)
+            masked = np.argwhere(to_oracle_state(ocfg, pre).masked(blk))
+            M = check_controller_step(ocfg, pre, post, blk, t)
+            if on_step is not None:
+                on_step(blk, t, M)
+            if M:
+                ran.append((t, h, post, masked))
+            pre = post
+            if np.all(post["exit_reason"][:, blk] != 0):
+                assert cai.cai_poll(ctx, 0, 5000)
+                break
+        later = [k for k in range(len(ran)) if ran[k][0] > 0]
+        pick_steps = [k for k in range(len(ran)) if ran[k][0] == 0]
+        if later:
+            pick_steps += rng.choice(later, size=min(n_sampled_steps, len(later)),
+                                     replace=False).tolist()
+        for k in pick_steps:
+            t, h, post, masked = ran[k]
+            M = len(masked)
+            pick = set(rng.choice(M, size=min(rows_per_step, M), replace=False).tolist()) | {0, M - 1}
+            check_rows_sampled(W_host, h, post, blk, [tuple(masked[i]) for i in sorted(pick)], c.P)
+    assert cai.cai_test_check_guards(ctx) == 0, "a device buffer was written past its end"
+    return pre

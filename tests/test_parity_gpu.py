@@ -695,13 +695,12 @@ def test_full_size_first_step_sampled(name):
         cai.cai_free(ctx)
 
 
-@pytest.mark.parametrize("name,n_blocks", [("llada", None), ("dream", 2)])
+@pytest.mark.parametrize("name,n_blocks", [("llada", None), ("dream", None)])
 def test_full_size_trajectory_every_row(name, n_blocks):
-    # The benchmark's own configuration at full size (B = 1, P = 32, the LLaDA
-    # or Dream weight shape, single-kernel steps, the calibrated generator):
-    # every step of the generation (LLaDA: all eight blocks; Dream: the first
-    # two) is checked teacher-forced on every masked row, confidences,
-    # argmaxes and every integer field of the state.
+    # The B = 1 configurations at full size (P = 32, the LLaDA or Dream weight
+    # shape, single-kernel steps, the calibrated generator): every step of the
+    # whole generation (all eight blocks) is checked teacher-forced on every
+    # masked row, confidences, argmaxes and every integer field of the state.
     wl = synth.WORKLOADS[name]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks, preset=cai.CAI_PRESET_LLADA)
     hs = synth.HiddenStates(wl, W, "calibrated")
@@ -715,26 +714,65 @@ def test_full_size_trajectory_every_row(name, n_blocks):
         cai.cai_free(ctx)
 
 
-def test_batched_multi_chunk_step_sampled():
-    # B = 64 sequences, 2048 masked rows (8 MMA chunks of 256) at full LLaDA
-    # width; sampled rows across chunks against the oracle.
-    wl = synth.WORKLOADS["llada_batched"]
+@pytest.mark.parametrize("name,B,P,T,nb,a0", [
+    ("b64", 64, 32, 32, 8, "u04"),      # batched LLaDA layout: 2048 rows at step zero
+    ("long", 8, 64, 64, 16, "long"),    # long-Dream layout: 16 blocks of 64, T = 64
+])
+def test_batch_layouts_full_trajectory_small_vocab(name, B, P, T, nb, a0):
+    # The batched-LLaDA (B = 64, P = 32, 8 blocks) and long-Dream (B = 8,
+    # P = 64, T = 64, 16 blocks, later blocks easier) layouts with a small
+    # vocabulary and hidden size, so that the oracle recomputes every row:
+    # every step of the whole generation teacher-forced, every field.  At
+    # B = 64 the commit kernel runs 64 CTAs and builds the 2048-token row list
+    # in four rounds; the long layout runs theta_e^(b) down to its floor
+    # (b > 4) and exits blocks early.
+    V, H = 4096, 256
+    wl = synth.Workload(name, B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0=a0)
+    ctx, W = _ctx(B, P, H, V, T, nb)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=B + P)
+    try:
+        assert cai.cai_get_stats(ctx)["kernels_per_step"] > 1
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P * nb
+        assert final["m_hist"][0, 0] == B * P
+        assert np.all(final["exit_reason"] != 0)
+        ex = final["exit_step"]
+        assert (ex < T - 1).all(axis=0).any()          # some block ended early for everyone
+        if nb > 4:
+            ocfg = parity.oracle_config(ctx.cfg)
+            assert oracle.theta_e(ocfg, nb) == pytest.approx(0.40)
+            assert (final["exit_reason"][:, 4:] != 0).all()
+        print(name, rep, "steps per block", (ex.max(axis=0) + 1).tolist())
+    finally:
+        cai.cai_free(ctx)
+
+
+@pytest.mark.parametrize("name", ["llada_batched", "dream_long"])
+def test_full_size_batch_trajectory_controller_and_sampled_rows(name):
+    # The batched LLaDA (B = 64, H = 4096, V = 126464) and long Dream (B = 8,
+    # P = 64, T = 64, H = 3584, V = 152064, 16 blocks) configurations at full
+    # size, the whole generation: every step checked at the controller level
+    # (the oracle runs Algorithm 1 from the GPU's pre-step state on the GPU's
+    # confidences and argmaxes; tokens, commit steps, budgets, low-yield
+    # counters, exits and M_t bit-exact), and at step zero of every block
+    # plus four seeded steps among each block's others, 14 sampled masked rows
+    # (the first and last included) recomputed by the fp64 oracle.
+    wl = synth.WORKLOADS[name]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
     hs = synth.HiddenStates(wl, W, "calibrated")
+    seen = set()
+
+    def on_step(blk, t, M):
+        seen.add("pair2" if M > 256 else "pair1" if M >= 32 else "narrow" if M else "empty")
+
     try:
-        h = hs(0, 0)
-        cai.cai_first_step(ctx, h)
-        torch.cuda.synchronize()
-        st = cai.cai_state_download(ctx)
-        flat = [0, 255, 256, 1023, 1500, 2047]
-        rows = oracle.bf16_bits(h.reshape(-1, wl.H))[flat]
-        o = oracle.head_rows(W, rows)
-        for k, i in enumerate(flat):
-            b, p = divmod(i, wl.P)
-            assert abs(st["s0"][b, p] - o["conf"][k]) <= parity.CONF_TOL
-            if o["gap"][k] > parity.GAP_TOL:
-                assert st["cand"][b, p] == o["idx"][k]
-        assert st["m_hist"][0, 0] == wl.B * wl.P
+        final = parity.run_controller_checked_trajectory(ctx, W, hs, 4, 12, seed=7,
+                                                         on_step=on_step)
+        assert np.all(final["exit_reason"] != 0)
+        assert final["m_hist"][0, 0] == wl.B * wl.P
+        assert {"pair2", "pair1", "narrow"} <= seen, seen
+        print(name, "steps per block", (final["exit_step"].max(axis=0) + 1).tolist(),
+              "exits", np.bincount(final["exit_reason"].reshape(-1), minlength=4).tolist())
     finally:
         cai.cai_free(ctx)
 
@@ -766,45 +804,6 @@ def test_debug_build_range_checks_stay_quiet():
                          capture_output=True, text=True, timeout=900)
     assert out.returncode == 0, out.stdout[-2000:] + out.stderr[-2000:]
     assert "debug build clean" in out.stdout
-
-
-def test_long_dream_full_size_steps_sampled():
-    # Long-generation Dream shape (B = 8, P = 64, H = 3584, V = 152064): the
-    # first steps of block 0 run on the pair kernel with two row tiles and
-    # then one (per-pair partials), down to narrow steps with M < 32; at every
-    # step a sample of the rows it decoded is recomputed by the oracle.
-    wl = synth.WORKLOADS["dream_long"]
-    ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
-    hs = synth.HiddenStates(wl, W, "calibrated")
-    rng = np.random.default_rng(5)
-    try:
-        pre = cai.cai_state_download(ctx)
-        seen = set()
-        for t in range(wl.T):
-            h = hs(0, t)
-            (cai.cai_first_step if t == 0 else cai.cai_denoise_step)(ctx, h)
-            torch.cuda.synchronize()
-            post = cai.cai_state_download(ctx)
-            M = int(post["m_hist"][0, t])
-            masked = np.argwhere(pre["tok"][:, :wl.P] == cai.CAI_MASK_TOKEN)
-            masked = [tuple(x) for x in masked if pre["exit_reason"][x[0], 0] == 0]
-            assert len(masked) == M
-            pick = [masked[i] for i in rng.choice(len(masked), size=min(3, len(masked)),
-                                                  replace=False)]
-            rows = oracle.bf16_bits(h)[[b for b, _ in pick], [p for _, p in pick]]
-            o = oracle.head_rows(W, rows)
-            for k, (b, p) in enumerate(pick):
-                assert abs(post["conf"][b, p] - o["conf"][k]) <= parity.CONF_TOL, (t, b, p)
-                if o["gap"][k] > parity.GAP_TOL:
-                    assert post["cand"][b, p] == o["idx"][k], (t, b, p)
-            seen.add("pair2" if M > 256 else "pair1" if M >= 32 else "swap")
-            pre = post
-            if cai.cai_poll(ctx, 0, 5000) or len(seen) == 3:
-                break
-        assert seen == {"pair2", "pair1", "swap"}
-        assert cai.cai_test_check_guards(ctx) == 0
-    finally:
-        cai.cai_free(ctx)
 
 
 def test_bench_json_line_contract():

@@ -61,3 +61,59 @@ def test_random_values_near_thresholds():
         c = np.float32(theta + rng.integers(-3, 4) * 6e-8)
         v = kernel_side_value(c, theta, fb)
         assert _double(v, theta, fb) == _kernel(c, theta, fb), (c, theta)
+
+
+def _simulated_gpu_steps(B=6, P=16, T=8, seed=3):
+    """States before and after each step of a synthetic trajectory, taken by
+    the oracle's own controller on fp32-rounded confidences (standing in for
+    the states a GPU step downloads), block 0 then block 1."""
+    import oracle
+    rng = np.random.default_rng(seed)
+    cfg = oracle.Config(B=B, P=P, T=T, n_blocks=2)
+    st = oracle.State(cfg)
+
+    def dump(s):
+        d = {f: getattr(s, f).copy() for f in oracle.State.FIELDS}
+        d["conf"] = d["conf"].astype(np.float32)
+        d["s0"] = d["s0"].astype(np.float32)
+        d["m_hist"] = np.zeros((cfg.n_blocks, T), np.int32)
+        return d
+
+    pre = dump(st)
+    steps = []
+    for blk in range(2):
+        for t in range(T):
+            mk = st.masked(blk)
+            conf = np.float32(rng.uniform(0.0, 1.0, (B, P))).astype(np.float64)
+            idx = rng.integers(0, 1000, (B, P)).astype(np.int32)
+            oracle.controller_step(st, blk, t, np.where(mk, conf, 0.0), np.where(mk, idx, -1))
+            post = dump(st)
+            post["m_hist"] = pre["m_hist"].copy()
+            post["m_hist"][blk, t] = int(mk.sum())
+            steps.append((blk, t, pre, post))
+            pre = post
+            if np.all(st.exit_reason[:, blk] != 0):
+                break
+    return cfg, steps
+
+
+def test_controller_check_passes_on_a_consistent_step_and_catches_mistakes():
+    from tests.parity import check_controller_step
+    cfg, steps = _simulated_gpu_steps()
+    assert len(steps) >= 4
+    for blk, t, pre, post in steps:
+        assert check_controller_step(cfg, pre, post, blk, t) == post["m_hist"][blk, t]
+    # A committed token, a low-yield counter and M_t each changed in one
+    # step's post state: the check must fail on each.
+    blk, t, pre, post = next(s for s in steps if (s[3]["tok"] != s[2]["tok"]).any())
+    for field, change in (("tok", lambda a: a.__setitem__(tuple(np.argwhere(
+                              (post["tok"] != pre["tok"]))[0]), 999999)),
+                          ("ell", lambda a: a.__setitem__(0, a[0] + 1)),
+                          ("m_hist", lambda a: a.__setitem__((blk, t), a[blk, t] + 1))):
+        bad = {k: (v.copy() if isinstance(v, np.ndarray) else v) for k, v in post.items()}
+        change(bad[field])
+        try:
+            check_controller_step(cfg, pre, bad, blk, t)
+        except AssertionError:
+            continue
+        raise AssertionError(f"a changed {field} was not caught")

@@ -18,6 +18,7 @@
 // head_kernel.cuh, whose kernels must be defined in a single unit).
 #pragma once
 
+#include <atomic>
 #include <mutex>
 
 namespace cai {
@@ -333,6 +334,21 @@ bool encode(CUtensorMap* m, const void* base, uint64_t rows, uint64_t cols, uint
                   CU_TENSOR_MAP_FLOAT_OOB_FILL_NONE) == CUDA_SUCCESS;
 }
 
+// Whether p is device (or managed) memory of device dev: the TMA maps and the
+// kernels' stores must never be pointed at host memory.
+bool on_device(const void* p, int dev) {
+  cudaPointerAttributes a;
+  if (cudaPointerGetAttributes(&a, p) != cudaSuccess) {
+    cudaGetLastError();
+    return false;
+  }
+  return (a.type == cudaMemoryTypeDevice || a.type == cudaMemoryTypeManaged) && a.device == dev;
+}
+
+// Test hook: the next call makes its error word record a failed bounded wait
+// before the merge (see cai_test_static_wait_timeout).
+std::atomic<int> g_static_fail_next{0};
+
 }  // namespace
 }  // namespace cai
 
@@ -352,6 +368,9 @@ extern "C" int cai_head_rows_static(const void* W, int32_t V, int32_t H, const v
     return CAI_ERR_CUDA;
   }
   if (major != 10 || minor != 3) return CAI_ERR_UNSUPPORTED;
+  if (!on_device(W, dev) || !on_device(rows, dev) || !on_device(conf, dev) ||
+      !on_device(argmax, dev))
+    return CAI_ERR_ARG;
   DeviceSetup* d = nullptr;
   int r = setup_device(dev, &d);
   if (r != CAI_OK) return r;
@@ -363,10 +382,21 @@ extern "C" int cai_head_rows_static(const void* W, int32_t V, int32_t H, const v
       !encode(&tm_r, rows, static_cast<uint64_t>(M), static_cast<uint64_t>(H), kBoxRowsB))
     return CAI_ERR_ARG;
   cudaStream_t s = static_cast<cudaStream_t>(stream);
+  // An error left pending by earlier, unrelated work is not this call's.
+  cudaGetLastError();
   lm_head_rows_static_kernel<<<G, kHeadThreads, kStaticSmemBytes, s>>>(tm_w, tm_r, d->part, d->err,
                                                                        V, H, M, n_tiles);
+  // If the LM head did not launch, the merge would read a previous call's partials.
+  if (cudaGetLastError() != cudaSuccess) return CAI_ERR_CUDA;
+  if (g_static_fail_next.exchange(0) != 0)
+    wait_timeout_probe_kernel<<<1, 32, 0, s>>>(d->err, kErrWaitFull);
   merge_rows_static_kernel<<<(M + 7) / 8, 256, 0, s>>>(d->part, d->err, M, G, conf, argmax);
   clear_static_err_kernel<<<1, 1, 0, s>>>(d->err);
   if (cudaGetLastError() != cudaSuccess) return CAI_ERR_CUDA;
+  return CAI_OK;
+}
+
+extern "C" int cai_test_static_wait_timeout(void) {
+  cai::g_static_fail_next.store(1);
   return CAI_OK;
 }

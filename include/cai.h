@@ -236,6 +236,53 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
                      void* stream, cai_ctx** out);
 
 /*
+ * Vocabulary-parallel decoding head.  Box 1's confidence and argmax are a
+ * maximum, a sum of exponentials and a lowest-index argmax over the
+ * vocabulary, and each of them is an exact merge of the same reductions over
+ * the parts of any split of the vocabulary.  So g shards (one per GPU, or
+ * several on one GPU) can each hold a slice of W and decode it: every shard
+ * context keeps a full copy of the controller state, computes for every
+ * masked row one triple over its slice, the triples of all shards are
+ * exchanged (an all-gather of rows x 16 bytes per shard, by the caller:
+ * torch.distributed, NCCL or anything else), and every shard merges them and
+ * applies the same commit rule, so the states stay identical.
+ *
+ * cai_init_vocab_shard creates a shard context.  cfg->V is the size V of the
+ * whole vocabulary; W_shard [V_shard, H] bf16 (row-major, host or device,
+ * read during the call as for cai_init) holds its rows [v0, v0 + V_shard).
+ * Requires 0 <= v0, V_shard >= 64 and v0 + V_shard <= V (else
+ * CAI_ERR_SHAPE).  A shard context always runs multi-kernel steps; the plain
+ * step calls refuse it (CAI_ERR_ARG).  A step is, in this order:
+ *
+ *   cai_shard_head(ctx, hidden, triples, stream): the gather, the shard's LM
+ *   head and, into `triples` (device, 16-byte aligned, cai_shard_rows()
+ *   entries of 16 bytes), one triple per row of the step's masked-row list:
+ *   {float m = max z * log2(e), float S = sum 2^(z log2(e) - m), int32 idx
+ *   = the lowest global vocabulary index reaching the maximum, 0}, the empty
+ *   triple {-3e38, 0, INT32_MAX, 0} past the step's M rows.  Step zero of a
+ *   block when the context's next local step is 0, else a denoising step,
+ *   with the order rules of cai_first_step / cai_denoise_step; hidden as
+ *   there (device, or page-locked host rows read in place).
+ *
+ *   cai_shard_commit(ctx, gathered, n_shards, stream): `gathered` (device,
+ *   16-byte aligned) holds every shard's triples one after the other,
+ *   [n_shards][cai_shard_rows()] (any order of shards: ties keep the lower
+ *   index); merges each row's n_shards triples into c = 1 / S and the argmax
+ *   and applies the commit rule, ending the step.  Errors: CAI_ERR_ORDER
+ *   without a preceding cai_shard_head; CAI_ERR_ARG for n_shards outside
+ *   [1, 4096] or a pointer that is not device memory.
+ *
+ * Between the two calls, cai_block_advance returns CAI_ERR_ORDER.  The
+ * library performs no communication itself.
+ */
+int cai_init_vocab_shard(const cai_config* cfg, const void* W_shard, int32_t v0, int32_t V_shard,
+                         void* stream, cai_ctx** out);
+/* Rows of a shard context's exchange buffers (B P rounded up to 16). */
+int cai_shard_rows(const cai_ctx* ctx, int32_t* rows);
+int cai_shard_head(cai_ctx* ctx, const void* hidden, void* triples, void* stream);
+int cai_shard_commit(cai_ctx* ctx, const void* gathered, int32_t n_shards, void* stream);
+
+/*
  * Local step t = 0 of the current block (Algorithm 1, step-zero init): every
  * position of every sequence is masked, so M = B P rows are decoded.  Stores
  * s_i and B_i, then applies the commit rule with theta^(b)(0).
@@ -325,7 +372,11 @@ void cai_free(cai_ctx* ctx);
  * that maximum, against the caller's W ([V, H] bf16 row-major, device, read in
  * place).  conf (float) and argmax (int32) are device arrays of M entries.
  * Asynchronous on `stream`.  Limits: 1 <= M <= 256, V >= 128, H % 64 == 0 and
- * 64 <= H <= 16384; pointers 16-byte aligned (else CAI_ERR_SHAPE / CAI_ERR_ARG).
+ * 64 <= H <= 16384 (else CAI_ERR_SHAPE); W and rows 16-byte aligned, and all
+ * four pointers device (or managed) memory of the current device (else
+ * CAI_ERR_ARG, with nothing launched).  Any CUDA error already pending from
+ * earlier work is cleared first; if the LM-head kernel fails to launch, the
+ * call returns CAI_ERR_CUDA without launching the merge.
  *
  * Scratch: a fixed file-scope device array of 256 x 160 partial triples
  * (640 KiB) plus an error word, held by every GPU that loads this library until
@@ -338,6 +389,16 @@ void cai_free(cai_ctx* ctx);
  */
 int cai_head_rows_static(const void* W, int32_t V, int32_t H, const void* rows, int32_t M,
                          float* conf, int32_t* argmax, void* stream);
+
+/*
+ * Testing hook for cai_head_rows_static: the next call (process-wide, once)
+ * runs, between its LM-head and merge kernels, a kernel that waits through
+ * the step kernels' bounded barrier wait on a barrier nothing arrives at and,
+ * after the 2 s limit, records a failed wait in the static error word, as a
+ * kernel whose wait gave up would.  That call's outputs are then NaN / -1 and
+ * the word is cleared for the next call.  No trap and no fault.
+ */
+int cai_test_static_wait_timeout(void);
 
 /* Static string for a status code. */
 const char* cai_strerror(int status);

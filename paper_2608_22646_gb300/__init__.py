@@ -54,7 +54,8 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_strerror", "cai_test_fail_alloc_after", "cai_test_head_grid_limit",
            "cai_test_pair_plan", "cai_test_theta_table", "cai_test_wait_timeout",
            "cai_test_check_guards",
-           "cai_head_rows_static")
+           "cai_head_rows_static", "cai_test_static_wait_timeout",
+           "cai_init_vocab_shard", "cai_shard_rows", "cai_shard_head", "cai_shard_commit")
 
 
 class CaiError(RuntimeError):
@@ -129,6 +130,12 @@ def _load():
         "cai_test_wait_timeout": (ctypes.c_int, [vp, vp]),
         "cai_test_check_guards": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
         "cai_head_rows_static": (ctypes.c_int, [vp, i32, i32, vp, i32, vp, vp, vp]),
+        "cai_test_static_wait_timeout": (ctypes.c_int, []),
+        "cai_init_vocab_shard": (ctypes.c_int, [ctypes.POINTER(cai_config), vp, i32, i32, vp,
+                                                ctypes.POINTER(vp)]),
+        "cai_shard_rows": (ctypes.c_int, [vp, ctypes.POINTER(i32)]),
+        "cai_shard_head": (ctypes.c_int, [vp, vp, vp, vp]),
+        "cai_shard_commit": (ctypes.c_int, [vp, vp, i32, vp]),
     }
     for name, (res, args) in sig.items():
         f = getattr(lib, name)
@@ -240,6 +247,44 @@ def cai_init_rmsnorm(cfg: cai_config, W, norm_weight, eps: float, stream=None) -
                                   _buf(norm_weight, "norm_weight", "bfloat16"), float(eps),
                                   _stream(stream), ctypes.byref(h)), "cai_init_rmsnorm")
     return Ctx(h.value, cfg, W, norm_weight, float(eps))
+
+
+def cai_init_vocab_shard(cfg: cai_config, W_shard, v0: int, stream=None) -> Ctx:
+    """A shard context of the vocabulary-parallel head: ``W_shard`` [V_shard, H]
+    holds the rows [v0, v0 + V_shard) of W; ``cfg.V`` is the whole vocabulary."""
+    h = ctypes.c_void_p()
+    _check(lib().cai_init_vocab_shard(ctypes.byref(cfg), _buf(W_shard, "W_shard", "bfloat16"),
+                                      int(v0), int(W_shard.shape[0]), _stream(stream),
+                                      ctypes.byref(h)), "cai_init_vocab_shard")
+    return Ctx(h.value, cfg, W_shard)
+
+
+def cai_shard_rows(ctx: Ctx) -> int:
+    n = ctypes.c_int32(0)
+    _check(lib().cai_shard_rows(ctx.handle, ctypes.byref(n)), "cai_shard_rows")
+    return n.value
+
+
+def cai_shard_head(ctx: Ctx, hidden, triples, stream=None) -> None:
+    """This shard's triple of every masked row into ``triples``, a float32
+    tensor [cai_shard_rows(ctx), 4] (the argmax travels as int32 bits)."""
+    rows = cai_shard_rows(ctx)
+    if not isinstance(triples, int) and tuple(triples.shape) != (rows, 4):
+        raise ValueError(f"triples: expected shape ({rows}, 4), got {tuple(triples.shape)}")
+    _check(lib().cai_shard_head(ctx.handle, _buf(hidden, "hidden", "bfloat16"),
+                                _buf(triples, "triples", "float32"), _stream(stream)),
+           "cai_shard_head")
+
+
+def cai_shard_commit(ctx: Ctx, gathered, stream=None) -> None:
+    """Merge every shard's triples, ``gathered`` float32 [n_shards, rows, 4],
+    and apply the commit rule (ends the step)."""
+    rows = cai_shard_rows(ctx)
+    if gathered.ndim != 3 or tuple(gathered.shape[1:]) != (rows, 4):
+        raise ValueError(f"gathered: expected shape (n_shards, {rows}, 4), "
+                         f"got {tuple(gathered.shape)}")
+    _check(lib().cai_shard_commit(ctx.handle, _buf(gathered, "gathered", "float32"),
+                                  int(gathered.shape[0]), _stream(stream)), "cai_shard_commit")
 
 
 def cai_first_step(ctx: Ctx, hidden, stream=None) -> None:
@@ -376,6 +421,11 @@ def cai_head_rows_static(W, rows, conf, argmax, stream=None) -> None:
                                       M, _buf(conf, "conf", "float32"),
                                       _buf(argmax, "argmax", "int32"), _stream(stream)),
            "cai_head_rows_static")
+
+
+def cai_test_static_wait_timeout() -> None:
+    """Make the next cai_head_rows_static call record a failed bounded wait."""
+    _check(lib().cai_test_static_wait_timeout(), "cai_test_static_wait_timeout")
 
 
 def config_from_dict(d: dict) -> cai_config:

@@ -251,6 +251,13 @@ struct cai_ctx {
   unsigned long long* stage_seq_dev = nullptr;
   bool stage_by_word = false;
   bool fused = false;    // single-kernel step (B P <= 32)
+  // Vocabulary shard (cai_init_vocab_shard): the context's LM head covers the
+  // rows [v_off, v_off + cfg.V) of a vocabulary of V_total rows; a step is
+  // cai_shard_head, an exchange of every shard's triples, cai_shard_commit.
+  bool shard = false;
+  int v_off = 0, V_total = 0;
+  bool shard_pending = false;  // a shard head ran; its commit has not
+  bool shard_first = false;    // ... and it was the block's step zero
   int G = 0, n_stages = 0, n_bslots = 0, n_max = 0, slot_cols = 0, gmax = 1, tmem_cols = 0;
   int b_slot_bytes = 0;
   size_t head_smem = 0;
@@ -407,6 +414,85 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   return cp;
 }
 
+// Multi-kernel step, kernel 1: the gather of this step's masked rows into
+// the compact operand (all rows at step zero).
+int launch_gather(cai_ctx* c, const void* hid, bool first, cudaStream_t stream) {
+  GatherParams gp{};
+  gp.hidden = static_cast<const __nv_bfloat16*>(hid);
+  gp.hc = c->hc;
+  gp.list = c->list;
+  gp.row_of = c->row_of;
+  gp.d_M = c->d_M;
+  gp.B = c->cfg.B;
+  gp.BP = c->BP;
+  gp.H = c->cfg.H;
+  gp.first = first ? 1 : 0;
+  gp.inv_r = c->norm ? c->inv_r : nullptr;
+  gp.err = c->err;
+  gp.eps = c->norm_eps;
+  const int g_grid = c->rows_cap / kGatherRowsPerCta;
+  if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) !=
+      cudaSuccess)
+    return check_launch(c);
+  c->stats.launches++;
+  return CAI_OK;
+}
+
+// Multi-kernel step: the CTA-pair LM head at local step t, and the row merge
+// of its per-tile partials in contexts where some step size leaves them.
+int launch_pair_head(cai_ctx* c, int t, cudaStream_t stream) {
+  const cai_config& cfg = c->cfg;
+  PairParams pp{};
+  pp.d_M = c->d_M;
+  pp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
+  pp.part = c->part;
+  pp.err = c->err;
+  pp.V = cfg.V;
+  pp.H = cfg.H;
+  pp.n_vt = c->n_vt;
+  pp.min_M = c->pair_min_M;
+  pp.swap_max_n = c->swap_max_n;
+  pp.n_stages = c->pair_stages;
+  pp.inv_r = c->inv_r;
+  if (launch_pdl(c->pdl, c->pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
+                 c->tm_a, c->tm_w, c->tm_rows, pp) != cudaSuccess)
+    return check_launch(c);
+  c->stats.launches++;
+  if (c->need_reduce) {
+    ReduceParams rp{};
+    rp.part = c->part;
+    rp.rowres = c->rowres;
+    rp.d_M = c->d_M;
+    rp.n_vt = c->n_vt;
+    rp.min_M = c->pair_min_M;
+    rp.n_pairs = c->pair_grid / 2;
+    rp.swap_max_n = c->swap_max_n;
+    if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream,
+                   rp) != cudaSuccess)
+      return check_launch(c);
+    c->stats.launches++;
+  }
+  return CAI_OK;
+}
+
+// The rows a multi-kernel step reads: device rows as they are, page-locked
+// host rows in place over the host link (the gather reads only the masked
+// ones), other host rows copied to the device on the stream first.
+int multi_kernel_rows(cai_ctx* c, const void* hidden, cudaStream_t stream, const void** hid) {
+  *hid = hidden;
+  if (is_device_ptr(hidden)) return CAI_OK;
+  if (const void* mapped = host_mapped_ptr(hidden)) {
+    *hid = mapped;
+    return CAI_OK;
+  }
+  const size_t bytes = static_cast<size_t>(c->BP) * c->cfg.H * 2;
+  if (cudaMemcpyAsync(c->hidden_stage, hidden, bytes, cudaMemcpyHostToDevice, stream) !=
+      cudaSuccess)
+    return fail(c, CAI_ERR_CUDA);
+  *hid = c->hidden_stage;
+  return CAI_OK;
+}
+
 // One denoising step.  Single-kernel step (B P <= 32): the LM-head kernel
 // reads the hidden states in place and its last CTA commits.  Otherwise:
 // gather -> LM head -> merge + commit.
@@ -493,24 +579,8 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   }
 
   if (!c->fused) {
-    GatherParams gp{};
-    gp.hidden = static_cast<const __nv_bfloat16*>(hid);
-    gp.hc = c->hc;
-    gp.list = c->list;
-    gp.row_of = c->row_of;
-    gp.d_M = c->d_M;
-    gp.B = cfg.B;
-    gp.BP = c->BP;
-    gp.H = cfg.H;
-    gp.first = first ? 1 : 0;
-    gp.inv_r = c->norm ? c->inv_r : nullptr;
-    gp.err = c->err;
-    gp.eps = c->norm_eps;
-    const int g_grid = c->rows_cap / kGatherRowsPerCta;
-    if (launch_pdl(c->pdl, gather_rows_kernel, g_grid, kGatherThreads, 0, stream, gp) !=
-        cudaSuccess)
-      return check_launch(c);
-    c->stats.launches++;
+    const int r = launch_gather(c, hid, first, stream);
+    if (r != CAI_OK) return r;
   } else {
     if (stage_slot < 0 && hid != c->hid_mapped) {
       // The single-kernel step reads the caller's [B P, H] rows through TMA.
@@ -578,36 +648,8 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
     // Only one of the two LM-head kernels decodes a step: the other reads
     // this step's M and returns at once (with pair_min_M = 1 the pair kernel
     // decodes every step and the other one is not launched).
-    PairParams pp{};
-    pp.d_M = c->d_M;
-    pp.m_hist_slot = c->st.m_hist + c->blk * cfg.T + t;
-    pp.part = c->part;
-    pp.err = c->err;
-    pp.V = cfg.V;
-    pp.H = cfg.H;
-    pp.n_vt = c->n_vt;
-    pp.min_M = c->pair_min_M;
-    pp.swap_max_n = c->swap_max_n;
-    pp.n_stages = c->pair_stages;
-    pp.inv_r = c->inv_r;
-    if (launch_pdl(c->pdl, c->pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
-                   c->tm_a, c->tm_w, c->tm_rows, pp) != cudaSuccess)
-      return check_launch(c);
-    c->stats.launches++;
-    if (c->need_reduce) {
-      ReduceParams rp{};
-      rp.part = c->part;
-      rp.rowres = c->rowres;
-      rp.d_M = c->d_M;
-      rp.n_vt = c->n_vt;
-      rp.min_M = c->pair_min_M;
-      rp.n_pairs = c->pair_grid / 2;
-      rp.swap_max_n = c->swap_max_n;
-      if (launch_pdl(c->pdl, reduce_partials_kernel, c->reduce_grid, kReduceThreads, 0, stream,
-                     rp) != cudaSuccess)
-        return check_launch(c);
-      c->stats.launches++;
-    }
+    const int r = launch_pair_head(c, t, stream);
+    if (r != CAI_OK) return r;
   }
   if (c->profiling) cudaEventRecord(ev[2], stream);
   c->stats.head_launches++;
@@ -660,14 +702,24 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
 
 namespace {
 
-// cai_init and cai_init_rmsnorm; g (bf16 [H], host or device) is null for cai_init.
-int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, void* stream,
-              cai_ctx** out) {
-  if (!cfg || !W || !out) return CAI_ERR_ARG;
+// cai_init, cai_init_rmsnorm and cai_init_vocab_shard; g (bf16 [H], host or
+// device) is null except for cai_init_rmsnorm; V_shard > 0 makes a shard
+// context whose W holds the vocabulary rows [v0, v0 + V_shard).
+int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps, int v0,
+              int V_shard, void* stream, cai_ctx** out) {
+  if (!cfg_in || !W || !out) return CAI_ERR_ARG;
   *out = nullptr;
-  int r = validate(cfg);
+  int r = validate(cfg_in);
   if (r != CAI_OK) return r;
   if (reinterpret_cast<uintptr_t>(W) % 16 != 0) return CAI_ERR_ARG;
+  const bool shard = V_shard > 0;
+  if (shard && (v0 < 0 || V_shard < 64 ||
+                static_cast<int64_t>(v0) + V_shard > static_cast<int64_t>(cfg_in->V)))
+    return CAI_ERR_SHAPE;
+  // A shard context runs its LM head over its own V_shard rows.
+  cai_config local_cfg = *cfg_in;
+  if (shard) local_cfg.V = V_shard;
+  const cai_config* cfg = &local_cfg;
 
   int dev = 0, major = 0, minor = 0, sms = 0, smem_optin = 0;
   if (cudaGetDevice(&dev) != cudaSuccess ||
@@ -697,12 +749,18 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   // 168.0k; B P = 128, 256 ran at 0.60, 0.29 of the roofline single-kernel).
   // CAI_FUSED_MAX_BP overrides the limit (up to 256).
   const int fmax = env_int("CAI_FUSED_MAX_BP");
-  c->fused = c->BP <= (fmax > 0 && fmax <= kChunkN ? fmax : kFusedMaxRows);
+  c->fused = !shard && c->BP <= (fmax > 0 && fmax <= kChunkN ? fmax : kFusedMaxRows);
   c->norm = g != nullptr;
   c->norm_eps = static_cast<float>(eps);
   c->head_kernel = c->norm ? lm_head_softmax_kernel<true> : lm_head_softmax_kernel<false>;
-  c->use_pair = !c->fused && pair_enabled();
+  // Shard contexts always run multi-kernel steps on the pair kernel with
+  // swapped narrow steps, so that the pair kernel decodes every step.
+  c->shard = shard;
+  c->v_off = shard ? v0 : 0;
+  c->V_total = cfg_in->V;
+  c->use_pair = shard || (!c->fused && pair_enabled());
   c->swap_max_n = c->use_pair ? pair_swap_max_n() : 0;
+  if (shard && c->swap_max_n < kSwapColStep) c->swap_max_n = 192;
   c->pair_kernel = c->norm ? lm_head_pair_kernel<true> : lm_head_pair_kernel<false>;
 
   // LM-head launch shape.  N chunk (positions per MMA), grid (one CTA per SM,
@@ -1011,7 +1069,8 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
   c->stats.pair_stages = c->use_pair ? c->pair_stages : 0;
   c->stats.kernels_per_step =
       c->fused ? 1
-               : 2 + (c->head_in_step ? 1 : 0) + (c->use_pair ? 1 : 0) + (c->need_reduce ? 1 : 0);
+               : 2 + (c->head_in_step ? 1 : 0) + (c->use_pair ? 1 : 0) + (c->need_reduce ? 1 : 0) +
+                     (c->shard ? 2 : 0);
   r = cai_reset(c, stream);
   if (r != CAI_OK) {
     release(c);
@@ -1025,7 +1084,7 @@ int init_impl(const cai_config* cfg, const void* W, const void* g, double eps, v
 }  // namespace
 
 int cai_init(const cai_config* cfg, const void* W, void* stream, cai_ctx** out) {
-  return init_impl(cfg, W, nullptr, 0.0, stream, out);
+  return init_impl(cfg, W, nullptr, 0.0, 0, 0, stream, out);
 }
 
 int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weight, double eps,
@@ -1033,7 +1092,13 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
   if (!norm_weight || reinterpret_cast<uintptr_t>(norm_weight) % 2 != 0 || !(eps >= 0.0) ||
       !std::isfinite(eps))
     return CAI_ERR_ARG;
-  return init_impl(cfg, W, norm_weight, eps, stream, out);
+  return init_impl(cfg, W, norm_weight, eps, 0, 0, stream, out);
+}
+
+int cai_init_vocab_shard(const cai_config* cfg, const void* W_shard, int32_t v0, int32_t V_shard,
+                         void* stream, cai_ctx** out) {
+  if (V_shard < 1) return CAI_ERR_SHAPE;
+  return init_impl(cfg, W_shard, nullptr, 0.0, v0, V_shard, stream, out);
 }
 
 int cai_reset(cai_ctx* c, void* stream_v) {
@@ -1069,11 +1134,12 @@ int cai_reset(cai_ctx* c, void* stream_v) {
   c->blk = 0;
   c->t_next = 0;
   c->block_done_seen = false;
+  c->shard_pending = false;
   return CAI_OK;
 }
 
 int cai_first_step(cai_ctx* c, const void* hidden, void* stream) {
-  if (!c || !hidden) return CAI_ERR_ARG;
+  if (!c || !hidden || c->shard) return CAI_ERR_ARG;
   if (c->sticky) return c->sticky;
   if (reinterpret_cast<uintptr_t>(hidden) % 16 != 0) return CAI_ERR_ARG;
   if (c->t_next != 0) return CAI_ERR_ORDER;
@@ -1082,7 +1148,7 @@ int cai_first_step(cai_ctx* c, const void* hidden, void* stream) {
 }
 
 int cai_denoise_step(cai_ctx* c, const void* hidden, void* stream) {
-  if (!c || !hidden) return CAI_ERR_ARG;
+  if (!c || !hidden || c->shard) return CAI_ERR_ARG;
   if (c->sticky) return c->sticky;
   if (reinterpret_cast<uintptr_t>(hidden) % 16 != 0) return CAI_ERR_ARG;
   if (c->t_next < 1 || c->t_next >= c->cfg.T || c->block_done_seen) return CAI_ERR_ORDER;
@@ -1093,10 +1159,92 @@ int cai_block_advance(cai_ctx* c, void* stream) {
   (void)stream;
   if (!c) return CAI_ERR_ARG;
   if (c->sticky) return c->sticky;
-  if (c->t_next < 1 || c->blk + 1 >= c->cfg.n_blocks) return CAI_ERR_ORDER;
+  if (c->t_next < 1 || c->blk + 1 >= c->cfg.n_blocks || c->shard_pending) return CAI_ERR_ORDER;
   c->blk += 1;
   c->t_next = 0;
   c->block_done_seen = false;
+  return CAI_OK;
+}
+
+int cai_shard_rows(const cai_ctx* c, int32_t* rows) {
+  if (!c || !rows || !c->shard) return CAI_ERR_ARG;
+  *rows = c->rows_cap;
+  return CAI_OK;
+}
+
+int cai_shard_head(cai_ctx* c, const void* hidden, void* triples, void* stream_v) {
+  if (!c || !hidden || !triples || !c->shard) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (reinterpret_cast<uintptr_t>(hidden) % 16 != 0 ||
+      reinterpret_cast<uintptr_t>(triples) % 16 != 0 || !is_device_ptr(triples))
+    return CAI_ERR_ARG;
+  const bool first = c->t_next == 0;
+  if (c->shard_pending || (!first && (c->t_next >= c->cfg.T || c->block_done_seen)))
+    return CAI_ERR_ORDER;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  const void* hid = nullptr;
+  int r = multi_kernel_rows(c, hidden, stream, &hid);
+  if (r != CAI_OK) return r;
+  if (first) c->block_done_seen = false;
+  if ((r = launch_gather(c, hid, first, stream)) != CAI_OK) return r;
+  if ((r = launch_pair_head(c, c->t_next, stream)) != CAI_OK) return r;
+  ShardRowsParams sp{};
+  sp.part = c->part;
+  sp.rowres = c->rowres;
+  sp.d_M = c->d_M;
+  sp.out = static_cast<float4*>(triples);
+  sp.rows_cap = c->rows_cap;
+  sp.n_pairs = c->pair_grid / 2;
+  sp.swap_max_n = c->swap_max_n;
+  sp.v_off = c->v_off;
+  const int warps = kShardThreads / 32;
+  if (launch_pdl(c->pdl, shard_rows_kernel, (c->rows_cap + warps - 1) / warps, kShardThreads, 0,
+                 stream, sp) != cudaSuccess)
+    return check_launch(c);
+  c->stats.launches++;
+  c->stats.head_launches++;
+  if ((r = check_launch(c)) != CAI_OK) return r;
+  c->shard_pending = true;
+  c->shard_first = first;
+  return CAI_OK;
+}
+
+int cai_shard_commit(cai_ctx* c, const void* gathered, int32_t n_shards, void* stream_v) {
+  if (!c || !gathered || !c->shard || n_shards < 1 || n_shards > 4096) return CAI_ERR_ARG;
+  if (c->sticky) return c->sticky;
+  if (reinterpret_cast<uintptr_t>(gathered) % 16 != 0 || !is_device_ptr(gathered))
+    return CAI_ERR_ARG;
+  if (!c->shard_pending) return CAI_ERR_ORDER;
+  cudaStream_t stream = static_cast<cudaStream_t>(stream_v);
+  const int t = c->t_next;
+  const int64_t step_id = c->last_step_id + 1;
+  ShardMergeParams mp{};
+  mp.gathered = static_cast<const float4*>(gathered);
+  mp.rowres = c->rowres;
+  mp.d_M = c->d_M;
+  mp.rows_cap = c->rows_cap;
+  mp.n_shards = n_shards;
+  const int warps = kShardThreads / 32;
+  if (launch_pdl(c->pdl, shard_merge_kernel, (c->rows_cap + warps - 1) / warps, kShardThreads, 0,
+                 stream, mp) != cudaSuccess)
+    return check_launch(c);
+  c->stats.launches++;
+  // The commit reads the one merged triple per row.
+  CommitParams cp = commit_params(c, t, step_id);
+  cp.part = c->rowres;
+  cp.n_part = 1;
+  cp.pair_min_M = INT_MAX;
+  const int commit_threads = c->cfg.P < kCommitThreads / 32 ? 32 * c->cfg.P : kCommitThreads;
+  if (launch_pdl(c->pdl, merge_commit_kernel, c->cfg.B, commit_threads, 0, stream, cp) !=
+      cudaSuccess)
+    return check_launch(c);
+  c->stats.launches++;
+  c->stats.steps++;
+  const int r = check_launch(c);
+  if (r != CAI_OK) return r;
+  c->shard_pending = false;
+  c->last_step_id = step_id;
+  c->t_next = t + 1;
   return CAI_OK;
 }
 

@@ -215,6 +215,93 @@ __global__ void __launch_bounds__(kListThreads) rebuild_list_kernel(const ListPa
   if (threadIdx.x == 0) *p.d_M = n;
 }
 
+// ------------------------------------------ vocabulary-parallel head (shards) --
+
+// A shard context holds the rows [v_off, v_off + V_shard) of W.  After its
+// LM head, shard_rows_kernel reduces each masked row's partials into one
+// triple (max * log2 e, sum of 2^(z log2 e - max), argmax as a global
+// vocabulary index) in the exchange buffer; rows past M get the empty triple.
+// Box 1's max, sum of exponentials and lowest-index argmax over the whole
+// vocabulary are exact merges of these triples over the shards, which
+// shard_merge_kernel does for every row before the commit.
+constexpr int kShardThreads = 256;
+
+struct ShardRowsParams {
+  const float4* part;    // [rows, per_row] pair partials of this step (local indices)
+  const float4* rowres;  // [rows] merged triple when the step wrote per-tile partials
+  const int* d_M;
+  float4* out;           // [rows_cap] exchange buffer
+  int rows_cap;
+  int n_pairs;           // the pair kernel's pairs
+  int swap_max_n;        // its orientation rule
+  int v_off;             // first vocabulary row of this shard
+};
+
+__global__ void __launch_bounds__(kShardThreads) shard_rows_kernel(const ShardRowsParams p) {
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // the pair kernel's partials (and the row merge's)
+  const int M = *p.d_M;
+  const int per_row = M > 0 ? pair_partials_per_row(M, p.n_pairs, pair_swapped(M, p.swap_max_n)) : 0;
+  const int lane = threadIdx.x & 31;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < p.rows_cap; row += nw) {
+    float m = kNegBig, s = 0.0f;
+    int ix = INT_MAX;
+    if (row < M) {
+      if (per_row > 0) {
+        for (int k = lane; k < per_row; k += 32) {
+          const float4 a = __ldcg(p.part + static_cast<size_t>(row) * per_row + k);
+          merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+        }
+      } else if (lane == 0) {
+        const float4 a = __ldcg(p.rowres + row);
+        merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+      }
+#pragma unroll
+      for (int off = 16; off >= 1; off >>= 1) {
+        const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+        const float so = __shfl_xor_sync(0xffffffffu, s, off);
+        const int io = __shfl_xor_sync(0xffffffffu, ix, off);
+        merge_tri(m, s, ix, mo, so, io);
+      }
+    }
+    if (lane == 0)
+      p.out[row] = make_float4(m, s, __int_as_float(ix == INT_MAX ? INT_MAX : ix + p.v_off), 0.0f);
+  }
+}
+
+struct ShardMergeParams {
+  const float4* gathered;  // [n_shards, rows_cap] every shard's exchange buffer, any order
+  float4* rowres;          // [rows_cap] merged triple per row, read by the commit
+  const int* d_M;
+  int rows_cap, n_shards;
+};
+
+// One warp per masked row: the merge of the row's triples from every shard.
+__global__ void __launch_bounds__(kShardThreads) shard_merge_kernel(const ShardMergeParams p) {
+  grid_launch_dependents();  // every thread: the CTA counts once all of them have
+  grid_dependency_wait();    // the previous commit's M and rowres readers
+  const int M = *p.d_M;
+  const int lane = threadIdx.x & 31;
+  const int nw = (gridDim.x * blockDim.x) >> 5;
+  for (int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5; row < M; row += nw) {
+    float m = kNegBig, s = 0.0f;
+    int ix = INT_MAX;
+    for (int k = lane; k < p.n_shards; k += 32) {
+      const float4 a = __ldcg(p.gathered + static_cast<size_t>(k) * p.rows_cap + row);
+      merge_tri(m, s, ix, a.x, a.y, __float_as_int(a.z));
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) {
+      const float mo = __shfl_xor_sync(0xffffffffu, m, off);
+      const float so = __shfl_xor_sync(0xffffffffu, s, off);
+      const int io = __shfl_xor_sync(0xffffffffu, ix, off);
+      merge_tri(m, s, ix, mo, so, io);
+    }
+    if (lane == 0) p.rowres[row] = make_float4(m, s, __int_as_float(ix), 0.0f);
+  }
+}
+
 // ------------------------------------------------------ merge + commit (K3) --
 
 // One CTA per sequence: merge_commit_sequence for sequence blockIdx.x, then the

@@ -13,7 +13,7 @@ LIB = os.path.join(PKG, "libcai.so")
 LIB_DEBUG = os.path.join(PKG, "libcai_debug.so")  # CAI_DEBUG: range checks on index lists
 SOURCES = ["cai.cu"]
 DEPS = ["cai.cu", "ptx.cuh", "softmax.cuh", "commit.cuh", "head_kernel.cuh", "step_kernels.cuh", "pair_kernel.cuh",
-        "static_head.cuh"]
+        "rows_kernel.cuh", "static_head.cuh"]
 
 
 def _stale(lib: str = LIB) -> bool:

@@ -20,6 +20,7 @@
 
 #include "cai.h"
 #include "pair_kernel.cuh"
+#include "rows_kernel.cuh"
 #include "step_kernels.cuh"
 
 using namespace cai;
@@ -251,6 +252,7 @@ struct cai_ctx {
   unsigned long long* stage_seq_dev = nullptr;
   bool stage_by_word = false;
   bool fused = false;    // single-kernel step (B P <= 32)
+  bool rows_head = false;  // the single-kernel step runs lm_head_rows_kernel
   // Vocabulary shard (cai_init_vocab_shard): the context's LM head covers the
   // rows [v_off, v_off + cfg.V) of a vocabulary of V_total rows; a step is
   // cai_shard_head, an exchange of every shard's triples, cai_shard_commit.
@@ -810,10 +812,13 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
   if (c->gmax < 1) c->gmax = 1;
   c->tmem_cols = next_pow2(2 * c->gmax * c->slot_cols < 32 ? 32 : 2 * c->gmax * c->slot_cols);
   c->b_slot_bytes = c->n_max * 128;
+  // CAI_HEAD_BSLOTS_TIGHT=1: size the hidden ring for full groups only (a
+  // shorter last group then throttles the producer a little; tuning knob).
+  const bool tight = env_int("CAI_HEAD_BSLOTS_TIGHT") == 1;
   auto bslots_for = [&](int stages) {
     // One hidden stage serves a group of tiles; keep enough of them in flight
     // to cover the W ring (groups may be one tile smaller than gmax).
-    const int per = c->gmax > 1 ? c->gmax - 1 : 1;
+    const int per = c->gmax > 1 ? (tight ? c->gmax : c->gmax - 1) : 1;
     return c->gmax == 1 ? stages : (stages + per - 1) / per + 1;
   };
   // Dynamic shared memory may use what the kernel's static shared memory leaves.
@@ -825,13 +830,44 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
   }
   const size_t dyn_limit = static_cast<size_t>(smem_optin) - head_attr.sharedSizeBytes;
   const int scap = env_int("CAI_HEAD_STAGES");
-  int stages = scap >= 2 && scap < 12 ? scap : 12;
+  int stages = scap >= 2 && scap <= 16 ? scap : 12;
   while (stages > 2 && head_smem_bytes(stages, bslots_for(stages), c->b_slot_bytes,
                                        c->slot_cols) > dyn_limit)
     --stages;
   c->n_stages = stages;
   c->n_bslots = bslots_for(stages);
   c->head_smem = head_smem_bytes(stages, c->n_bslots, c->b_slot_bytes, c->slot_cols);
+  // Single-kernel steps of up to 128 rows run lm_head_rows_kernel, the rows
+  // as the MMA's A operand and up to 256 vocabulary rows as N, which consumes
+  // W twice as fast per MMA as the swapped kernel (CAI_ROWS_HEAD=0: the
+  // swapped kernel instead).  W is packed by pack_weight_rows_kernel.
+  const char* rh_env = std::getenv("CAI_ROWS_HEAD");
+  if (c->fused && c->BP <= kRowsM && !(rh_env && rh_env[0] == '0')) {
+    c->rows_head = true;
+    c->head_kernel = c->norm ? lm_head_rows_kernel<true> : lm_head_rows_kernel<false>;
+    cudaFuncAttributes ra{};
+    if (cudaFuncGetAttributes(&ra, c->head_kernel) != cudaSuccess) {
+      cudaGetLastError();
+      delete c;
+      return CAI_ERR_CUDA;
+    }
+    const size_t rlimit = static_cast<size_t>(smem_optin) - ra.sharedSizeBytes;
+    // As many W stages as fit next to a rows ring of the same depth (the
+    // rows stages are small); CAI_ROWS_STAGES caps the W ring (tuning knob).
+    // Four 32 KiB W stages in flight per SM: deeper rings stream faster on
+    // most SMs but starve some (measured, LLaDA shape: finish spread 4 us at
+    // 4 stages, 20 us at 6), and a step waits for its slowest CTA.
+    const int hs = rows_h_stride(c->BP);
+    const int scap2 = env_int("CAI_ROWS_STAGES");
+    int st = scap2 >= 2 && scap2 <= 8 ? scap2 : 4;
+    while (st > 2 && rows_smem_bytes(st, 2 * st, hs) > rlimit) --st;
+    int bs = 2 * st;
+    while (bs > 2 && rows_smem_bytes(st, bs, hs) > rlimit) --bs;
+    c->n_stages = st;
+    c->n_bslots = bs;
+    c->tmem_cols = kRowsTmemCols;
+    c->head_smem = rows_smem_bytes(st, bs, hs);
+  }
 
   // Pair kernel launch shape: a persistent grid of as many 2-CTA clusters as
   // can be resident at once.
@@ -990,7 +1026,11 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
   }
   {
     const long long n_chunks = static_cast<long long>(units) * kUnitRows * cfg->H / 8;
-    if (c->head_in_step)
+    if (c->rows_head)
+      pack_weight_rows_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
+          static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units,
+          c->G, n_chunks, g_dev);
+    else if (c->head_in_step)
       pack_weight_kernel<<<4 * sms, 256, 0, static_cast<cudaStream_t>(stream)>>>(
           static_cast<const uint4*>(w_src), static_cast<uint4*>(c->wpk), cfg->V, cfg->H, units,
           c->G, c->gmax, n_chunks, g_dev);

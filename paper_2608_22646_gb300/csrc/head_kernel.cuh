@@ -285,6 +285,32 @@ struct Ring {
   }
 };
 
+// Single-kernel step, end of every CTA: the last CTA to finish (atomic
+// ticket, no waiting) merges the partials and commits the step for every
+// sequence, after the previous step's commit (state, ticket) is complete.
+// `free_smem` is at least sizeof(CommitSmem) bytes of shared memory that no
+// copy or MMA touches any more (the drained W ring).
+__device__ __forceinline__ void fused_step_commit(const CommitParams& cp, uint8_t* free_smem) {
+  grid_dependency_wait();
+  __shared__ int s_last;
+  if (threadIdx.x == 0) {
+    __threadfence();
+    s_last = atomicAdd(cp.ticket, 1u) == gridDim.x - 1;
+  }
+  __syncthreads();
+  if (!s_last) return;
+  __threadfence();
+  int decoded = 0, remaining = 0;
+  for (int b = 0; b < cp.B; ++b) {
+    int left = 0;
+    decoded += merge_commit_sequence(cp, b, *reinterpret_cast<CommitSmem*>(free_smem), cp.part,
+                                     cp.n_part, &left);
+    remaining += left;
+  }
+  if (threadIdx.x == 0) *cp.m_hist_slot = decoded;
+  finish_step(cp, remaining);
+}
+
 // ---------------------------------------------------------------- kernel --
 
 // kNorm: the model's final RMSNorm is part of the head.  Its weight is
@@ -686,29 +712,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     tmem_dealloc(tmem_base, static_cast<uint32_t>(p.tmem_cols));
   }
 
-  if (p.fused) {
-    // Single-kernel step: the last CTA to finish commits the step, after the
-    // previous step's commit (state, ticket) is complete.
-    grid_dependency_wait();
-    __shared__ int s_last;
-    if (threadIdx.x == 0) {
-      __threadfence();
-      s_last = atomicAdd(p.cp.ticket, 1u) == static_cast<unsigned>(G - 1);
-    }
-    __syncthreads();
-    if (!s_last) return;
-    __threadfence();
-    int decoded = 0, remaining = 0;
-    for (int b = 0; b < p.cp.B; ++b) {
-      int left = 0;
-      // Every copy and MMA has completed: the W ring is free shared memory.
-      decoded += merge_commit_sequence(p.cp, b, *reinterpret_cast<CommitSmem*>(sm.a), p.cp.part,
-                                       p.cp.n_part, &left);
-      remaining += left;
-    }
-    if (threadIdx.x == 0) *p.cp.m_hist_slot = decoded;
-    finish_step(p.cp, remaining);
-  }
+  if (p.fused) fused_step_commit(p.cp, sm.a);
 }
 
 }  // namespace cai

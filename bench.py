@@ -259,7 +259,10 @@ def _roofline(wl, st0, stats1, head_ms, head_launches, step_ms, ms, steps, steps
     head_iso_s = (head_ms / 1e3 / steps) if profiled and head_ms > 0 else head_live_s
     per_launch = max(1, (head_launches if head_launches else int(steps_issued) * steps) // steps)
     kps = int(stats1["kernels_per_step"])
-    if kps == 1:
+    if kps == 1 and stats1.get("head_rows"):
+        kernel = ("lm_head_rows_kernel (single-kernel step: LM head with the rows as the MMA's A "
+                  "operand, softmax and commit)")
+    elif kps == 1:
         kernel = "lm_head_softmax_kernel (single-kernel step: LM head, softmax and commit)"
     elif stats1["pair_swap_max_n"] >= 32:
         kernel = (f"lm_head_pair_kernel (every step; swapped orientation for tiles up to "

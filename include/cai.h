@@ -27,7 +27,9 @@
  * one kernel: the LM head over every row of the block, whose last CTA applies
  * the commit rule; it streams W before the previous step has committed and
  * waits for it only to write its partials and to commit (CAI_FUSED_MAX_BP=n
- * moves the limit, up to 256).  With B P > 32 a step is gather, LM head,
+ * moves the limit, up to 256).  That LM head puts the rows in the MMA's A
+ * operand and 256 vocabulary rows in N (up to 128 rows; CAI_ROWS_HEAD=0 uses
+ * the swapped-operand kernel instead, W in A and the rows in N).  With B P > 32 a step is gather, LM head,
  * merge + commit.  The LM head is the CTA-pair
  * kernel (tcgen05 cta_group::2), which picks its orientation per step from
  * the masked-row count M: the rows as MMA N in row tiles of equal width (a
@@ -197,6 +199,8 @@ typedef struct cai_stats {
                                (masked rows in the MMA N dimension) is at most
                                this run swapped on the pair LM head (0: never)     */
   int32_t pair_stages;      /* pipeline stages of the pair LM head                 */
+  int32_t head_rows;        /* 1: single-kernel steps run the LM head with the rows
+                               as the MMA's A operand (B P <= 128), 0: otherwise   */
 } cai_stats;
 
 /* Fill *cfg with the paper's hyperparameters (Section 5, Appendix "Setup")

@@ -96,7 +96,7 @@ class cai_stats(ctypes.Structure):
                 ("stages", ctypes.c_int32), ("n_max", ctypes.c_int32),
                 ("kernels_per_step", ctypes.c_int32), ("step_ms", ctypes.c_double),
                 ("pair_grid", ctypes.c_int32), ("pair_swap_max_n", ctypes.c_int32),
-                ("pair_stages", ctypes.c_int32)]
+                ("pair_stages", ctypes.c_int32), ("head_rows", ctypes.c_int32)]
 
 
 def _load():

@@ -1107,6 +1107,7 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
   c->stats.pair_grid = c->use_pair ? c->pair_grid : 0;
   c->stats.pair_swap_max_n = c->swap_max_n;
   c->stats.pair_stages = c->use_pair ? c->pair_stages : 0;
+  c->stats.head_rows = c->rows_head ? 1 : 0;
   c->stats.kernels_per_step =
       c->fused ? 1
                : 2 + (c->head_in_step ? 1 : 0) + (c->use_pair ? 1 : 0) + (c->need_reduce ? 1 : 0) +

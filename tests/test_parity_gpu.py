@@ -835,3 +835,33 @@ def test_bench_json_line_contract():
     assert e2e["d2h_bytes_per_step"] > 0
     assert line["gpu_launches"] > 0
     assert line["clocks"]["sm_max_mhz"] > 0
+
+
+@pytest.mark.parametrize("rows_head,max_bp,shape", [
+    # (CAI_ROWS_HEAD, CAI_FUSED_MAX_BP, (B, P, H, V, T, n_blocks)): single-kernel
+    # steps of up to 128 rows on the rows-operand LM head (2 to 4 epilogue
+    # warps with rows; rows stages of 8 and 16 KiB), ragged V (V % 8, V % 256),
+    # one K block (H = 64); and the swapped-operand kernel that CAI_ROWS_HEAD=0
+    # selects, at the default limit.
+    ("1", "64", (2, 32, 256, 4096, 8, 2)),
+    ("1", "128", (4, 32, 192, 5003, 8, 2)),
+    ("1", "128", (1, 100, 64, 2085, 6, 1)),
+    ("1", "32", (1, 20, 128, 300, 6, 2)),
+    ("0", "32", (1, 16, 256, 4096, 8, 4)),
+    ("0", "32", (2, 16, 128, 1003, 6, 2)),
+])
+def test_single_kernel_heads(rows_head, max_bp, shape, monkeypatch):
+    monkeypatch.setenv("CAI_ROWS_HEAD", rows_head)
+    monkeypatch.setenv("CAI_FUSED_MAX_BP", max_bp)
+    B, P, H, V, T, nb = shape
+    wl = synth.Workload("fused", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=B * 31 + P)
+    try:
+        st = cai.cai_get_stats(ctx)
+        assert st["kernels_per_step"] == 1
+        assert st["head_rows"] == (1 if rows_head == "1" else 0)
+        rep, _ = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P
+    finally:
+        cai.cai_free(ctx)

@@ -122,9 +122,21 @@ class Clocks:
                 "samples": len(sm)}
 
 
+def source_code_sha(path: str) -> str:
+    """sha256 prefix of a source file's code: comments and blank lines removed,
+    so that a comment edit does not count as a change of the kernel."""
+    import re
+    with open(path) as f:
+        s = f.read()
+    s = re.sub(r"/\*.*?\*/", "", s, flags=re.S)
+    s = re.sub(r"//[^\n]*", "", s)
+    s = "\n".join(line.rstrip() for line in s.splitlines() if line.strip())
+    return hashlib.sha256(s.encode()).hexdigest()[:16]
+
+
 def _traffic_record(workload: str):
     """DRAM bytes per launch of the workload's dominant LM-head kernel from the
-    committed ncu summaries, if they were taken on the current kernel source."""
+    committed ncu summaries, if they were taken on the current kernel code."""
     p = os.path.join(PROFILES, "lm_head_traffic.json")
     if not os.path.exists(p):
         return None
@@ -136,9 +148,7 @@ def _traffic_record(workload: str):
         src = os.path.join(ROOT, "paper_2608_22646_gb300", "csrc", rec["source"])
         if not os.path.exists(src):
             return None
-        with open(src, "rb") as f:
-            h = hashlib.sha256(f.read()).hexdigest()[:16]
-        return rec if rec.get("source_sha") == h else None
+        return rec if rec.get("source_code_sha") == source_code_sha(src) else None
     return None
 
 

@@ -4,15 +4,16 @@
 // logits never leaving tensor memory), for the M <= 128 rows of a step whose
 // block holds at most 128 positions.
 //
-// Why this orientation.  A tcgen05.mma of M = 128 rows and K = 16 costs about
-// the same time whatever its N (measured: 128 x 32 x 16 steps of the swapped
-// kernel run at one MMA per ~86 ns, the pair kernel's 256 x 256 x 16 at one
-// per ~156 cycles).  With W as the A operand (lm_head_softmax_kernel) each
-// MMA consumes 4 KiB of W, which caps an SM at ~48 GB/s of W, just the HBM
-// share of 151 SMs: the stream is paced by MMAs, and a CTA's short last tile
-// costs as much as a full one.  With W as the B operand, N = 256 vocabulary
-// rows, each MMA consumes 8 KiB of W, and the stream is HBM-bound again.  The
-// rows pad to M = 128, which the tensor cores absorb.
+// Why this orientation.  In the swapped kernel (lm_head_softmax_kernel, W as
+// the A operand, the rows as N = 32) every 16 KiB W stage took ~0.345 us of
+// the MMA thread (four K = 16 MMAs, their waits and commits), whatever the
+// stage held: ~48 GB/s of W per SM, the HBM share of 151 SMs, so the stream
+// was paced by the MMA side and a CTA's short last tile cost as much as a
+// full one (the same stream without MMAs, or with one MMA per stage, ran at
+// 7.7-7.8 TB/s).  With the rows as A and up to 256 vocabulary rows as B, a
+// 32 KiB stage of W takes four MMAs, half as many per byte, and the stream is
+// HBM-bound.  The rows pad to M = 128, which the tensor cores absorb (an
+// M = 128, N = 256, K = 16 MMA takes ~65 ns on resident operands).
 //
 // Rows stages.  The MMA reads 128 rows of A, but only the first mq =
 // round16(M) are the step's; the accumulator rows past M are never read.  So

@@ -14,6 +14,7 @@
 namespace cai {
 
 constexpr int kGatherRowsPerCta = 4;
+constexpr int kGatherVecs = 8;       // 16-byte loads in flight per gather thread (H <= 4096 in one round)
 constexpr int kGatherThreads = 256;
 constexpr int kListThreads = 256;    // rebuild_list_kernel
 // Merge kernel: one CTA per sequence, 16 warps of 4 positions each, so that
@@ -74,10 +75,24 @@ __global__ void __launch_bounds__(kGatherThreads)
       if (!CAI_IN_RANGE(src_row >= 0 && src_row < p.BP, p.err)) src_row = 0;
       const uint4* src =
           reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(src_row) * p.H);
-      for (int v = t; v < nvec; v += 64) {
-        const uint4 x = __ldg(src + v);
-        dst[v] = x;
-        if (p.inv_r) ss += sumsq8(x);
+      // All of a thread's loads are issued before its first store (the
+      // compiler cannot reorder them: dst and src could alias as far as it
+      // knows), so a row costs one memory round trip, not one per vector.
+      for (int v0 = t; v0 < nvec; v0 += 64 * kGatherVecs) {
+        uint4 x[kGatherVecs];
+#pragma unroll
+        for (int j = 0; j < kGatherVecs; ++j) {
+          const int v = v0 + 64 * j;
+          x[j] = v < nvec ? __ldg(src + v) : make_uint4(0u, 0u, 0u, 0u);
+        }
+#pragma unroll
+        for (int j = 0; j < kGatherVecs; ++j) {
+          const int v = v0 + 64 * j;
+          if (v < nvec) {
+            dst[v] = x[j];
+            if (p.inv_r) ss += sumsq8(x[j]);
+          }
+        }
       }
     } else {
       for (int v = t; v < nvec; v += 64) dst[v] = make_uint4(0u, 0u, 0u, 0u);

@@ -162,3 +162,52 @@ def test_vocab_shard_arguments_and_order():
     finally:
         cai.cai_free(ctx)
         cai.cai_free(plain)
+
+
+@pytest.mark.parametrize("g", [2, 3])
+def test_vocab_shards_full_size_llada(g):
+    # The LLaDA-8B shape (V = 126464, H = 4096, B = 1, P = 32) split over g
+    # shard contexts on one GPU, the first two blocks: every step checked at
+    # the controller level (the oracle's Algorithm 1 on the merged triples the
+    # shards produced, every integer field bit-exact), the shards' states
+    # identical, and at step zero of each block 8 sampled rows recomputed by
+    # the fp64 oracle over the whole vocabulary.
+    wl = synth.WORKLOADS["llada"]
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device="cuda")
+    hs = synth.HiddenStates(wl, W, "calibrated")
+    cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    ctxs = _shard_ctxs(cfg, W, g)
+    ocfg = parity.oracle_config(cfg)
+    W_host = oracle.bf16_bits(W)
+    rng = np.random.default_rng(g)
+    try:
+        rows = cai.cai_shard_rows(ctxs[0])
+        bufs = [torch.empty((rows, 4), dtype=torch.float32, device="cuda") for _ in ctxs]
+        pre = cai.cai_state_download(ctxs[0])
+        decoded = 0
+        for blk in range(2):
+            if blk:
+                for c in ctxs:
+                    cai.cai_block_advance(c)
+            for t in range(wl.T):
+                h = hs(blk, t)
+                _step(ctxs, bufs, h)
+                torch.cuda.synchronize()
+                posts = [cai.cai_state_download(c) for c in ctxs]
+                for p in posts[1:]:
+                    for f in FIELDS:
+                        assert np.array_equal(p[f], posts[0][f]), (f, blk, t)
+                masked = np.argwhere(parity.to_oracle_state(ocfg, pre).masked(blk))
+                decoded += parity.check_controller_step(ocfg, pre, posts[0], blk, t)
+                if t == 0:
+                    pick = rng.choice(len(masked), size=8, replace=False)
+                    parity.check_rows_sampled(W_host, h, posts[0], blk,
+                                              [tuple(masked[i]) for i in pick], wl.P)
+                pre = posts[0]
+                if np.all(pre["exit_reason"][:, blk] != 0):
+                    break
+        assert decoded >= 2 * wl.P
+        assert np.all(pre["exit_reason"][:, :2] != 0)
+    finally:
+        for c in ctxs:
+            cai.cai_free(c)

@@ -23,13 +23,13 @@
  * use programmatic dependent launch: each may be scheduled while the kernel
  * before it in the stream still runs, and waits for that kernel to complete
  * before touching anything it produces (setting CAI_PDL=0 in the environment
- * before cai_init launches them plainly instead).  With B P <= 32 a step is
+ * before cai_init launches them plainly instead).  With B P <= 64 a step is
  * one kernel: the LM head over every row of the block, whose last CTA applies
  * the commit rule; it streams W before the previous step has committed and
  * waits for it only to write its partials and to commit (CAI_FUSED_MAX_BP=n
  * moves the limit, up to 256).  That LM head puts the rows in the MMA's A
  * operand and 256 vocabulary rows in N (up to 128 rows; CAI_ROWS_HEAD=0 uses
- * the swapped-operand kernel instead, W in A and the rows in N).  With B P > 32 a step is gather, LM head,
+ * the swapped-operand kernel instead, W in A and the rows in N).  With B P > 64 a step is gather, LM head,
  * merge + commit.  The LM head is the CTA-pair
  * kernel (tcgen05 cta_group::2), which picks its orientation per step from
  * the masked-row count M: the rows as MMA N in row tiles of equal width (a
@@ -191,7 +191,7 @@ typedef struct cai_stats {
   int32_t grid;             /* CTAs of the LM-head kernel                          */
   int32_t stages;           /* pipeline stages of the LM-head kernel               */
   int32_t n_max;            /* positions per MMA chunk (N of the swapped MMA)      */
-  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 32); else gather,
+  int32_t kernels_per_step; /* 1: single-kernel step (B P <= 64); else gather,
                                LM head(s), row merge if needed, commit (2 to 5)    */
   double step_ms;           /* summed device time of profiled steps, every kernel  */
   int32_t pair_grid;        /* CTAs of the CTA-pair LM head (0: not used)          */
@@ -211,7 +211,7 @@ int cai_config_default(cai_config* cfg, int32_t preset, int32_t B, int32_t P, in
 /*
  * Create a context.  W is the LM-head weight [V, H] bf16, row-major, host or
  * device memory.  It is read once, during this call, into the library's
- * packed copies (2 V H bytes each: one copy when B P <= 32, two otherwise);
+ * packed copies (2 V H bytes each: one copy when B P <= 64, two otherwise);
  * the caller may free or change it afterwards.  All state starts at block 0,
  * t = 0, every token masked.  Allocates device memory and one page of mapped
  * pinned host memory.  Synchronous.
@@ -293,14 +293,14 @@ int cai_shard_commit(cai_ctx* ctx, const void* gathered, int32_t n_shards, void*
  * hidden: the block's final hidden states [B, P, H] bf16, row-major; row
  * (b, p) is the one that predicts position p of the block.  Device pointer:
  * read on the stream, must stay valid until the stream passes this call.
- * Host pointer: with B P > 32 and page-locked, device-mapped memory (e.g.
+ * Host pointer: with B P > 64 and page-locked, device-mapped memory (e.g.
  * cudaHostAlloc), the gather reads the masked rows in place over the host
  * link, on the stream (valid until the stream passes this call).  Otherwise
- * the rows are copied to the device: with B P <= 32 on a stream of the
+ * the rows are copied to the device: with B P <= 64 on a stream of the
  * context's own into one of two alternating device buffers, which the step's
  * kernel waits for on the device (so the copy for the next step runs during
  * this one and the step's stream itself waits for nothing), with
- * B P > 32 on the step's stream; page-locked memory must stay valid until
+ * B P > 64 on the step's stream; page-locked memory must stay valid until
  * the stream passes this call, pageable memory is staged by the CUDA runtime
  * before the call returns.
  * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call

@@ -33,7 +33,7 @@ std::atomic<int> g_head_grid_limit{0};
 // Programmatic dependent launch between the step's kernels; CAI_PDL=0 in the
 // environment turns it off (read once per context at cai_init).
 // Largest B P that runs single-kernel steps by default.
-constexpr int kFusedMaxRows = 32;
+constexpr int kFusedMaxRows = 64;
 
 bool pdl_enabled() {
   const char* e = std::getenv("CAI_PDL");
@@ -251,7 +251,7 @@ struct cai_ctx {
   // ev_copied.
   unsigned long long* stage_seq_dev = nullptr;
   bool stage_by_word = false;
-  bool fused = false;    // single-kernel step (B P <= 32)
+  bool fused = false;    // single-kernel step (B P <= 64)
   bool rows_head = false;  // the single-kernel step runs lm_head_rows_kernel
   // Vocabulary shard (cai_init_vocab_shard): the context's LM head covers the
   // rows [v_off, v_off + cfg.V) of a vocabulary of V_total rows; a step is
@@ -495,7 +495,7 @@ int multi_kernel_rows(cai_ctx* c, const void* hidden, cudaStream_t stream, const
   return CAI_OK;
 }
 
-// One denoising step.  Single-kernel step (B P <= 32): the LM-head kernel
+// One denoising step.  Single-kernel step (B P <= 64): the LM-head kernel
 // reads the hidden states in place and its last CTA commits.  Otherwise:
 // gather -> LM head -> merge + commit.
 int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first);
@@ -743,13 +743,13 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
   c->rows_cap = round_up(c->BP, 16);
   c->pdl = pdl_enabled();
   c->nvtx = nvtx_enabled();
-  // Single-kernel steps decode every row of the block each step, through one
-  // N = B P chunk of the swapped-operand kernel, and save the gather and
-  // commit launches.  Larger batches run multi-kernel steps, whose pair kernel
-  // decodes only the masked rows (measured, LLaDA shape, positions/s: B P = 32
-  // 92.3k single-kernel against 85.3k multi-kernel; B P = 64 161.9k against
-  // 168.0k; B P = 128, 256 ran at 0.60, 0.29 of the roofline single-kernel).
-  // CAI_FUSED_MAX_BP overrides the limit (up to 256).
+  // Single-kernel steps decode every row of the block each step (the
+  // rows-operand LM head pads the rows to 128 anyway) and save the gather and
+  // commit launches; larger batches run multi-kernel steps, whose pair kernel
+  // decodes only the masked rows.  Measured, LLaDA shape, positions/s,
+  // single- against multi-kernel: B P = 64 197.8k against 169.5k, B P = 128
+  // 329.3k against 331.5k.  CAI_FUSED_MAX_BP overrides the limit (up to 256;
+  // above 128 rows the swapped-operand kernel runs).
   const int fmax = env_int("CAI_FUSED_MAX_BP");
   c->fused = !shard && c->BP <= (fmax > 0 && fmax <= kChunkN ? fmax : kFusedMaxRows);
   c->norm = g != nullptr;

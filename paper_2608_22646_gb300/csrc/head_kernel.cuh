@@ -30,7 +30,8 @@
 // contiguous copies keep DRAM pages open, the strided 128-byte rows of a 2-D
 // tensor box do not.
 //
-// Single-kernel step (fused = 1, used when B P <= 32): the kernel decodes all
+// Single-kernel step (fused = 1, B P <= 64 and CAI_ROWS_HEAD=0, or more than
+// 128 rows): the kernel decodes all
 // B P rows straight from the caller's hidden states (no gather; at N <= 256 a
 // step reads W once whatever N is), and the last CTA to finish (atomic
 // ticket, no waiting) merges the partials and applies the commit rule for

@@ -234,16 +234,16 @@ def test_fraction_eta_mode():
         cai.cai_free(ctx)
 
 
-@pytest.mark.parametrize("B", [2, 3])
+@pytest.mark.parametrize("B", [2, 5])
 def test_all_commit_at_step_zero_and_noop_steps(B):
     # Hidden rows equal to a scaled W row make every confidence ~1: every
     # token commits at t = 0, the block exits DONE, and later steps decode
-    # nothing.  B P = 32: single-kernel steps; 48: multi-kernel steps, whose
+    # nothing.  B P = 32: single-kernel steps; 80: multi-kernel steps, whose
     # pair LM head records the empty step's M = 0 itself.
     P, H, V, T = 16, 256, 4096, 8
     ctx, W = _ctx(B, P, H, V, T, 2)
     try:
-        assert (cai.cai_get_stats(ctx)["kernels_per_step"] == 1) == (B * P <= 32)
+        assert (cai.cai_get_stats(ctx)["kernels_per_step"] == 1) == (B * P <= 64)
         tgt = torch.arange(B * P, device="cuda") * 37 % V
         h = (W[tgt].float() * 400.0).to(torch.bfloat16).reshape(B, P, H)
         cai.cai_first_step(ctx, h)
@@ -343,14 +343,14 @@ def test_pair_partial_layouts(clusters, max_n, shape, monkeypatch):
 
 
 @pytest.mark.parametrize("shape", [
-    # (B, P, H, V, T, n_blocks), all multi-kernel.  B P = 33: one over the
-    # single-kernel limit, a 64-wide swapped tile whose odd half runs past the
-    # 48-row buffer (TMA fills zeros).  V = 130: the odd CTA's vocabulary half
+    # (B, P, H, V, T, n_blocks), all multi-kernel.  B P = 65: one over the
+    # single-kernel limit, a 96-wide swapped tile whose odd half runs past the
+    # 80-row buffer (TMA fills zeros).  V = 130: the odd CTA's vocabulary half
     # holds 2 rows; V = 128: none.  B P = 287 (buffer 288): the first step's two
     # 160-wide swapped tiles end at row 320.  B P = 400: the first steps run
     # unswapped (224-wide tiles would be needed), later ones swapped.
-    (1, 33, 64, 130, 6, 2),
-    (3, 11, 128, 128, 6, 2),
+    (1, 65, 64, 130, 6, 2),
+    (3, 22, 128, 128, 6, 2),
     (7, 41, 192, 777, 6, 1),
     (2, 200, 64, 1000, 5, 1),
 ])
@@ -842,7 +842,7 @@ def test_bench_json_line_contract():
     # steps of up to 128 rows on the rows-operand LM head (2 to 4 epilogue
     # warps with rows; rows stages of 8 and 16 KiB), ragged V (V % 8, V % 256),
     # one K block (H = 64); and the swapped-operand kernel that CAI_ROWS_HEAD=0
-    # selects, at the default limit.
+    # selects, at B P <= 32.
     ("1", "64", (2, 32, 256, 4096, 8, 2)),
     ("1", "128", (4, 32, 192, 5003, 8, 2)),
     ("1", "128", (1, 100, 64, 2085, 6, 1)),

@@ -388,6 +388,10 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
   cp.pair_swap_max_n = c->swap_max_n;
   cp.pair_min_M = c->use_pair ? c->pair_min_M : INT_MAX;
   cp.identity_rows = c->fused ? 1 : 0;
+  // The pair kernel, the last LM-head kernel of a multi-kernel step, starts
+  // its dependents only after its own wait for the gather, hence for the
+  // previous step's commit.
+  cp.prefetch_state = !c->fused && c->use_pair ? 1 : 0;
   cp.st = c->st;
   cp.list = c->list;
   cp.row_of = c->row_of;
@@ -1275,6 +1279,7 @@ int cai_shard_commit(cai_ctx* c, const void* gathered, int32_t n_shards, void* s
   cp.part = c->rowres;
   cp.n_part = 1;
   cp.pair_min_M = INT_MAX;
+  cp.prefetch_state = 0;  // the exchange before it is the caller's
   const int commit_threads = c->cfg.P < kCommitThreads / 32 ? 32 * c->cfg.P : kCommitThreads;
   if (launch_pdl(c->pdl, merge_commit_kernel, c->cfg.B, commit_threads, 0, stream, cp) !=
       cudaSuccess)

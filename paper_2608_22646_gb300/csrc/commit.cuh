@@ -68,6 +68,8 @@ struct CommitParams {
   int pair_pairs;         // pairs of the pair kernel's grid
   int pair_swap_max_n;    // the pair kernel's orientation rule (pair_swapped)
   int identity_rows;      // 1: row of (b, p) is b P + p; 0: row_of[b P + p]
+  int prefetch_state;     // merge kernel: read the sequence's state before waiting for the
+                          // LM head (the kernel before it starts only after its own wait)
   StateArrays st;
   int* list;
   int* row_of;
@@ -94,31 +96,65 @@ __device__ __forceinline__ int budget_tier(float s, int p, int half, int late) {
   return 32;
 }
 
-// One step of Algorithm 1 for sequence b, by the whole calling CTA (blockDim.x
-// a multiple of 32; every thread must call it).  The sequence's state is read
-// into shared memory in one round of loads; warps then merge the partials of
-// the still-masked positions (kPPW at a time, all loads issued before
-// any merge) and lane 0 applies the commit rule (Box 6, Eq. position_commit,
-// with the step-zero init of Boxes 2 and 5); thread 0 updates the low-yield
-// counter and the exit state (Box 7, Algorithm 1).  Global state is only
-// written, never re-read, after the first round.  Returns, in every thread,
-// the positions decoded (M_t of the sequence) and, in *left_after, the
-// positions still masked afterwards in a running sequence.
 // Per-position working set of merge_commit_sequence, in shared memory the
 // caller provides (the LM-head kernel lends its drained W ring).
 struct CommitSmem {
   int tok[kMaxP];      // token after this step (kMask while masked)
   int cand[kMaxP];     // argmax of the previous decoded step, then of this step
   float conf[kMaxP];   // confidence of this step
+  int row[kMaxP];      // partial row of the position in this step (masked positions)
   uint8_t bud[kMaxP];  // budget before this step
   uint8_t run[kMaxP];  // diagnostics: same-argmax run before this step
   int16_t stable[kMaxP];  // diagnostics: stability step before this step
+  int running;         // the sequence has not left the block
+  int ell;             // low-yield counter before this step
 };
 
+// Reads what one step of Algorithm 1 needs of sequence b's state into cs, in
+// one round of loads by the whole calling CTA (visible to it after its next
+// __syncthreads): the block's tokens and budgets, the exit state, ell, and
+// the partial row of every position.  All of it was written by the previous
+// step's commit (or by the reset) except, at a block's first step, the row
+// list, which the gather then makes the identity; so a commit that follows an
+// LM head which itself waited for the previous step may read it before
+// waiting for the partials.
+__device__ __forceinline__ void commit_load(const CommitParams& p, int b, CommitSmem& cs) {
+  const int tid = threadIdx.x;
+  const int eb = b * p.n_blocks + p.blk;
+  const size_t g0 = static_cast<size_t>(b) * p.L + p.blk * p.P;
+  if (tid == 0) {
+    cs.running = __ldcg(&p.st.exit_reason[eb]) == kRunning;
+    cs.ell = __ldcg(&p.st.ell[b]);
+  }
+  const bool diag = (p.flags & kFlagDiag) != 0;
+  const bool ident = p.identity_rows || p.t == 0;
+  for (int pp = tid; pp < p.P; pp += blockDim.x) {
+    cs.tok[pp] = __ldcg(&p.st.tok[g0 + pp]);
+    cs.bud[pp] = p.st.budget[g0 + pp];
+    cs.row[pp] = ident ? b * p.P + pp : __ldcg(&p.row_of[b * p.P + pp]);
+    if (diag) {
+      cs.cand[pp] = __ldcg(&p.st.cand[g0 + pp]);
+      cs.run[pp] = __ldcg(&p.st.run[g0 + pp]);
+      cs.stable[pp] = __ldcg(&p.st.stable[g0 + pp]);
+    }
+  }
+}
+
+// One step of Algorithm 1 for sequence b, by the whole calling CTA (blockDim.x
+// a multiple of 32; every thread must call it).  The sequence's state is in
+// cs (commit_load, by this call unless `loaded`); warps merge the partials of
+// the still-masked positions (kPPW at a time, all loads issued before any
+// merge) and lane 0 applies the commit rule (Box 6, Eq. position_commit,
+// with the step-zero init of Boxes 2 and 5); thread 0 updates the low-yield
+// counter and the exit state (Box 7, Algorithm 1).  Global state is only
+// written, never re-read.  Returns, in every thread, the positions decoded
+// (M_t of the sequence) and, in *left_after, the positions still masked
+// afterwards in a running sequence.
 template <int kPPW = kPosPerWarp>
 __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& cs,
-                                     const float4* part, int n_part, int* left_after = nullptr) {
-  __shared__ int s_eta, s_left, s_reason, s_unres, s_ell, s_running;
+                                     const float4* part, int n_part, int* left_after = nullptr,
+                                     bool loaded = false) {
+  __shared__ int s_eta, s_left, s_reason, s_unres;
   int* s_tok = cs.tok;
   int* s_cand = cs.cand;
   float* s_conf = cs.conf;
@@ -127,26 +163,16 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
   const int nwarps = blockDim.x >> 5;
   const int eb = b * p.n_blocks + p.blk;
   const size_t g0 = static_cast<size_t>(b) * p.L + p.blk * p.P;
+  if (!loaded) commit_load(p, b, cs);
   if (tid == 0) {
     s_eta = 0;
     s_left = 0;
     s_reason = kRunning;
     s_unres = 0;
-    s_running = __ldcg(&p.st.exit_reason[eb]) == kRunning;
-    s_ell = __ldcg(&p.st.ell[b]);
   }
   const bool diag = (p.flags & kFlagDiag) != 0;
-  for (int pp = tid; pp < p.P; pp += blockDim.x) {
-    s_tok[pp] = __ldcg(&p.st.tok[g0 + pp]);
-    s_bud[pp] = p.st.budget[g0 + pp];
-    if (diag) {
-      s_cand[pp] = __ldcg(&p.st.cand[g0 + pp]);
-      cs.run[pp] = __ldcg(&p.st.run[g0 + pp]);
-      cs.stable[pp] = __ldcg(&p.st.stable[g0 + pp]);
-    }
-  }
   __syncthreads();
-  const bool running = s_running != 0;
+  const bool running = cs.running != 0;
   const bool gating = (p.flags & kFlagGating) != 0;
 
   if (running) {
@@ -158,7 +184,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
         const int pp = base + j * nwarps;
         row[j] = -1;
         if (pp < p.P && s_tok[pp] == kMask) {
-          row[j] = p.identity_rows ? b * p.P + pp : p.row_of[b * p.P + pp];
+          row[j] = cs.row[pp];
           if (!CAI_IN_RANGE(row[j] < p.B * p.P, p.err)) row[j] = -2;
           if (row[j] < 0) {
             if (lane == 0) atomicOr(p.err, kErrBadRow);
@@ -239,7 +265,7 @@ __device__ int merge_commit_sequence(const CommitParams& p, int b, CommitSmem& c
                             static_cast<double>(p.eta_bar))
                          : (static_cast<float>(eta) < p.eta_bar);
     // Algorithm 1 sets ell <- 0 before the block's first step.
-    const int ell = low ? (p.t == 0 ? 0 : s_ell) + 1 : 0;
+    const int ell = low ? (p.t == 0 ? 0 : cs.ell) + 1 : 0;
     p.st.ell[b] = ell;
     int reason = kRunning;
     if (gating && ell >= p.K)

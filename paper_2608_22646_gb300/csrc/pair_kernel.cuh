@@ -221,8 +221,11 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   const int pair = blockIdx.x >> 1;
   const int n_pairs = gridDim.x >> 1;
 
-  grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();    // d_M and the gathered rows of this step
+  // Every thread (the CTA counts once all of them have), after the wait: the
+  // commit kernel, which may start from here, reads the previous step's state
+  // before waiting for this kernel.
+  grid_launch_dependents();
   const int M = *p.d_M;
   if (p.m_hist_slot && blockIdx.x == 0 && threadIdx.x == 0 && (M >= p.min_M || p.min_M <= 1))
     *p.m_hist_slot = M;

@@ -326,20 +326,29 @@ __global__ void __launch_bounds__(kCommitThreads) merge_commit_kernel(const Comm
   __shared__ int s_last;
   __shared__ CommitSmem cs;
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
-  grid_dependency_wait();    // partials of this step, state of the previous one
   // This step's M (d_M is rewritten only by the last CTA, after every CTA's
-  // merge) tells which LM-head kernel decoded it: the pair kernel's tile
-  // partials were already merged into one triple per row.
-  const int M = *p.d_M;
+  // merge; at a block's first step every row is decoded) tells which LM-head
+  // kernel decoded it: the pair kernel's tile partials were already merged
+  // into one triple per row.  With prefetch_state, the kernel before this one
+  // started only after the previous step had finished, so M and the
+  // sequence's state are read before waiting for this step's partials.
+  int M = 0;
+  if (p.prefetch_state) {
+    M = p.t == 0 ? p.B * p.P : __ldcg(p.d_M);
+    commit_load(p, blockIdx.x, cs);
+  }
+  grid_dependency_wait();    // partials of this step (and state of the previous one)
+  if (!p.prefetch_state) M = *p.d_M;
+  const bool loaded = p.prefetch_state != 0;
   if (M >= p.pair_min_M) {
     const int per_row =
         pair_partials_per_row(M, p.pair_pairs, pair_swapped(M, p.pair_swap_max_n));
     if (per_row > 0)
-      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, per_row);
+      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, per_row, nullptr, loaded);
     else
-      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.rowres, 1);
+      merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.rowres, 1, nullptr, loaded);
   } else {
-    merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, p.n_part);
+    merge_commit_sequence<kCommitPPW>(p, blockIdx.x, cs, p.part, p.n_part, nullptr, loaded);
   }
   if (gridDim.x > 1) {
     if (threadIdx.x == 0) {

@@ -123,15 +123,27 @@ class Clocks:
 
 
 def source_code_sha(path: str) -> str:
-    """sha256 prefix of a source file's code: comments and blank lines removed,
-    so that a comment edit does not count as a change of the kernel."""
+    """sha256 prefix of a kernel source's code and of the local headers it
+    includes (recursively, each once): comments and blank lines removed, so
+    that a comment edit does not count as a change of the kernel."""
     import re
-    with open(path) as f:
-        s = f.read()
-    s = re.sub(r"/\*.*?\*/", "", s, flags=re.S)
-    s = re.sub(r"//[^\n]*", "", s)
-    s = "\n".join(line.rstrip() for line in s.splitlines() if line.strip())
-    return hashlib.sha256(s.encode()).hexdigest()[:16]
+    seen, parts = set(), []
+
+    def add(fp):
+        fp = os.path.normpath(fp)
+        if fp in seen or not os.path.exists(fp):
+            return
+        seen.add(fp)
+        with open(fp) as f:
+            s = f.read()
+        for inc in re.findall(r'^\s*#\s*include\s+"([^"]+)"', s, flags=re.M):
+            add(os.path.join(os.path.dirname(fp), inc))
+        s = re.sub(r"/\*.*?\*/", "", s, flags=re.S)
+        s = re.sub(r"//[^\n]*", "", s)
+        parts.append("\n".join(line.rstrip() for line in s.splitlines() if line.strip()))
+
+    add(path)
+    return hashlib.sha256("\n".join(parts).encode()).hexdigest()[:16]
 
 
 def _traffic_record(workload: str):

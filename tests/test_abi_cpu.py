@@ -277,3 +277,18 @@ def test_theta_table_arguments():
     assert lib.cai_test_theta_table(ctypes.byref(c), 0, 0, None) == cai.CAI_ERR_ARG
     c.P = 0
     assert lib.cai_test_theta_table(ctypes.byref(c), 0, 0, ptr) == cai.CAI_ERR_SHAPE
+
+
+def test_kernel_code_sha_follows_included_headers(tmp_path):
+    # The bench reports a DRAM traffic record only while the kernel's code
+    # still has the recorded sha: a code change in a header the kernel
+    # includes (even indirectly) changes it, a comment edit does not.
+    import bench
+    (tmp_path / "a.cuh").write_text('#include "b.cuh"\nint a() { return b(); }\n')
+    (tmp_path / "b.cuh").write_text('#include "c.cuh"\nint b() { return c(); }\n')
+    (tmp_path / "c.cuh").write_text('#include "a.cuh"\nint c() { return 1; }  // one\n')
+    s0 = bench.source_code_sha(str(tmp_path / "a.cuh"))
+    (tmp_path / "c.cuh").write_text('#include "a.cuh"\n/* note */\nint c() { return 1; }  // two\n')
+    assert bench.source_code_sha(str(tmp_path / "a.cuh")) == s0
+    (tmp_path / "c.cuh").write_text('#include "a.cuh"\nint c() { return 2; }\n')
+    assert bench.source_code_sha(str(tmp_path / "a.cuh")) != s0

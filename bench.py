@@ -561,16 +561,14 @@ def e2e_run(cai, ctx, hs, wl, steps, dist, dev):
     st = cai.cai_state_download(ctx)
     n_step_calls = (cai.cai_get_stats(ctx)["steps"] - s0) / steps
     dt_ms, positions = aggregate(dt * 1e3, int(st["m_hist"].sum()) * steps, dist, dev)
-    # Single-kernel steps copy every row of each step; multi-kernel steps read
-    # only the masked rows of the page-locked host buffer in place.
-    h2d = (n_step_calls * wl.B * wl.P * wl.H * 2 if int(cai.cai_get_stats(ctx)["kernels_per_step"]) == 1
-           else int(st["m_hist"].sum()) * wl.H * 2)
+    # Every step call copies the block's rows ([B, P, H] bf16) to the device.
+    h2d = n_step_calls * wl.B * wl.P * wl.H * 2
     return {"value": round(positions / (dt_ms / 1e3), 1), "unit": UNIT,
             "h2d_bytes_per_step": int(h2d),
             "d2h_bytes_per_step": int(wl.B * wl.n_blocks * wl.P * 4 + n_step_calls * 32),
-            "timing": "host wall clock around whole generations, pinned host inputs "
-                      "(single-kernel steps: copied per step; multi-kernel steps: masked rows "
-                      "read in place by the gather)"}
+            "timing": "host wall clock around whole generations, pinned host inputs (each step "
+                      "call's rows copied on the context's side stream while the previous step "
+                      "runs)"}
 
 
 def run_reference(args, wl):

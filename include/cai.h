@@ -266,7 +266,7 @@ int cai_init_rmsnorm(const cai_config* cfg, const void* W, const void* norm_weig
  *   triple {-3e38, 0, INT32_MAX, 0} past the step's M rows.  Step zero of a
  *   block when the context's next local step is 0, else a denoising step,
  *   with the order rules of cai_first_step / cai_denoise_step; hidden as
- *   there (device, or page-locked host rows read in place).
+ *   there (device, or page-locked host rows read in place by the gather).
  *
  *   cai_shard_commit(ctx, gathered, n_shards, stream): `gathered` (device,
  *   16-byte aligned) holds every shard's triples one after the other,
@@ -293,16 +293,15 @@ int cai_shard_commit(cai_ctx* ctx, const void* gathered, int32_t n_shards, void*
  * hidden: the block's final hidden states [B, P, H] bf16, row-major; row
  * (b, p) is the one that predicts position p of the block.  Device pointer:
  * read on the stream, must stay valid until the stream passes this call.
- * Host pointer: with B P > 64 and page-locked, device-mapped memory (e.g.
- * cudaHostAlloc), the gather reads the masked rows in place over the host
- * link, on the stream (valid until the stream passes this call).  Otherwise
- * the rows are copied to the device: with B P <= 64 on a stream of the
+ * Host pointer: the rows are copied to the device on a stream of the
  * context's own into one of two alternating device buffers, which the step's
- * kernel waits for on the device (so the copy for the next step runs during
- * this one and the step's stream itself waits for nothing), with
- * B P > 64 on the step's stream; page-locked memory must stay valid until
- * the stream passes this call, pageable memory is staged by the CUDA runtime
- * before the call returns.
+ * first kernel that reads them (the single-kernel LM head, or the gather)
+ * waits for on the device, so the copy for the next step runs during this one
+ * and the step's stream itself waits for nothing (with CAI_DIAGNOSTICS, or
+ * the final norm in a single-kernel step, the step's stream waits for the
+ * copy instead).  Page-locked memory must stay valid until the stream passes
+ * this call; pageable memory is staged by the CUDA runtime before the call
+ * returns.
  * Errors: CAI_ERR_ARG, CAI_ERR_ORDER (the block already ran a step; call
  * cai_block_advance or cai_reset first).
  */

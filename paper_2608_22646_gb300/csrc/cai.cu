@@ -231,11 +231,12 @@ struct cai_ctx {
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
   const void* hid_mapped = nullptr;
-  // Single-kernel steps on host rows: the rows are copied on copy_stream into
-  // stage2[step id & 1] (hidden_stage and a second buffer), and the step's
-  // stream waits only for that copy, so the copy of step t + 1 overlaps step
-  // t and no copy sits between two step kernels in the step's stream.  A
-  // buffer is refilled after the step that read it (ev_read) has finished.
+  // Steps on host rows: the rows are copied on copy_stream into stage2[step
+  // id & 1] (hidden_stage and a second buffer), and the step's stream waits
+  // only for that copy, so the copy of step t + 1 overlaps step t and no copy
+  // sits between two step kernels in the step's stream.  A buffer is refilled
+  // after the kernel that read it (ev_read: the single-kernel step's LM head,
+  // the multi-kernel step's gather) has finished.
   void* stage2[2] = {nullptr, nullptr};
   CUtensorMap tm_stage[2]{};
   cudaStream_t copy_stream = nullptr;
@@ -243,12 +244,13 @@ struct cai_ctx {
   cudaEvent_t ev_read[2] = {nullptr, nullptr};
   bool read_pending[2] = {false, false};
   // After its copy the side stream writes the step's id + 1 into
-  // stage_seq_dev[k]; the step's kernel waits for that word before reading
-  // the rows, so the step's stream waits for nothing and consecutive steps
-  // keep their programmatic overlap.  Used when no other kernel of the step
-  // reads the rows first (no final norm, no diagnostics) and the driver
-  // provides stream memory writes; otherwise the step's stream waits for
-  // ev_copied.
+  // stage_seq_dev[k]; the step's first kernel that reads the rows (the
+  // single-kernel LM head, or the gather) waits for that word before reading
+  // them, so the step's stream waits for nothing and consecutive steps keep
+  // their programmatic overlap.  Used when no other kernel of the step reads
+  // the rows first (diagnostics; single-kernel steps: the final norm's row
+  // scales) and the driver provides stream memory writes; otherwise the
+  // step's stream waits for ev_copied.
   unsigned long long* stage_seq_dev = nullptr;
   bool stage_by_word = false;
   bool fused = false;    // single-kernel step (B P <= 64)
@@ -422,8 +424,12 @@ CommitParams commit_params(cai_ctx* c, int t, int64_t step_id) {
 
 // Multi-kernel step, kernel 1: the gather of this step's masked rows into
 // the compact operand (all rows at step zero).
-int launch_gather(cai_ctx* c, const void* hid, bool first, cudaStream_t stream) {
+int launch_gather(cai_ctx* c, const void* hid, bool first, cudaStream_t stream,
+                  const unsigned long long* stage_word = nullptr,
+                  unsigned long long stage_seq = 0) {
   GatherParams gp{};
+  gp.stage_word = stage_word;
+  gp.stage_seq = stage_seq;
   gp.hidden = static_cast<const __nv_bfloat16*>(hid);
   gp.hc = c->hc;
   gp.list = c->list;
@@ -519,17 +525,12 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   const cai_config& cfg = c->cfg;
   const void* hid = hidden;
   const int64_t step_id = c->last_step_id + 1;
-  int stage_slot = -1;  // single-kernel step on host rows: stage2 buffer used
+  int stage_slot = -1;  // step on host rows: stage2 buffer used
   if (!is_device_ptr(hidden)) {
-    // Multi-kernel step on page-locked host rows: the gather reads the masked
-    // rows in place over the host link (only they cross it).  Otherwise the
-    // rows are copied to the device first: single-kernel steps on the side
-    // stream (see stage2), multi-kernel steps in the step's stream.
-    const void* mapped = c->fused ? nullptr : host_mapped_ptr(hidden);
+    // Host rows are copied to the device on the side stream (see stage2),
+    // overlapping the previous step; the step's first reader waits for them.
     const size_t bytes = static_cast<size_t>(c->BP) * cfg.H * 2;
-    if (mapped) {
-      hid = mapped;
-    } else if (c->fused) {
+    {
       const int k = static_cast<int>(step_id & 1);
       if ((c->read_pending[k] &&
            cudaStreamWaitEvent(c->copy_stream, c->ev_read[k], 0) != cudaSuccess) ||
@@ -548,11 +549,6 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       }
       hid = c->stage2[k];
       stage_slot = k;
-    } else {
-      if (cudaMemcpyAsync(c->hidden_stage, hidden, bytes, cudaMemcpyHostToDevice, stream) !=
-          cudaSuccess)
-        return fail(c, CAI_ERR_CUDA);
-      hid = c->hidden_stage;
     }
   }
   const int t = c->t_next;
@@ -585,8 +581,17 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   }
 
   if (!c->fused) {
-    const int r = launch_gather(c, hid, first, stream);
+    const unsigned long long* word =
+        stage_slot >= 0 && c->stage_by_word ? c->stage_seq_dev + stage_slot : nullptr;
+    const int r =
+        launch_gather(c, hid, first, stream, word, static_cast<unsigned long long>(step_id + 1));
     if (r != CAI_OK) return r;
+    if (stage_slot >= 0) {
+      // stage2[stage_slot] may be refilled once the gather is done.
+      if (cudaEventRecord(c->ev_read[stage_slot], stream) != cudaSuccess)
+        return fail(c, CAI_ERR_CUDA);
+      c->read_pending[stage_slot] = true;
+    }
   } else {
     if (stage_slot < 0 && hid != c->hid_mapped) {
       // The single-kernel step reads the caller's [B P, H] rows through TMA.
@@ -969,7 +974,7 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
     CAI_ALLOC(c->rowres, float4, c->rows_cap)
   }
   CAI_ALLOC(c->hidden_stage, uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
-  if (c->fused) {
+  if (!shard) {
     c->stage2[0] = c->hidden_stage;
     CAI_ALLOC(c->stage2[1], uint8_t, static_cast<size_t>(c->BP) * cfg->H * 2)
     CAI_ALLOC(c->stage_seq_dev, unsigned long long, 2)
@@ -978,7 +983,8 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
       delete c;
       return CAI_ERR_CUDA;
     }
-    c->stage_by_word = !c->norm && !(cfg->flags & CAI_DIAGNOSTICS) && get_write_value64() != nullptr;
+    c->stage_by_word = !(c->fused && c->norm) && !(cfg->flags & CAI_DIAGNOSTICS) &&
+                       get_write_value64() != nullptr;
   }
   // The swapped-operand kernel's packed W, only where that kernel runs (every
   // single-kernel step; multi-kernel steps with CAI_PAIR_SWAP=0 or CAI_PAIR=0).
@@ -1073,9 +1079,9 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
     delete c;
     return CAI_ERR_CUDA;
   }
-  if (c->fused) {
-    bool ok = make_map(&c->tm_stage[0], c->stage2[0], c->BP, cfg->H, kBoxRowsB) &&
-              make_map(&c->tm_stage[1], c->stage2[1], c->BP, cfg->H, kBoxRowsB) &&
+  if (!shard) {
+    bool ok = (!c->fused || (make_map(&c->tm_stage[0], c->stage2[0], c->BP, cfg->H, kBoxRowsB) &&
+                             make_map(&c->tm_stage[1], c->stage2[1], c->BP, cfg->H, kBoxRowsB))) &&
               cudaStreamCreateWithFlags(&c->copy_stream, cudaStreamNonBlocking) == cudaSuccess;
     for (int k = 0; ok && k < 2; ++k)
       ok = cudaEventCreateWithFlags(&c->ev_copied[k], cudaEventDisableTiming) == cudaSuccess &&

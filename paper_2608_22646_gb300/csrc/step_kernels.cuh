@@ -37,6 +37,8 @@ struct GatherParams {
   int first;                    // step zero: every position of every sequence
   float* inv_r;                 // final norm: 1 / sqrt(mean h^2 + eps) per row, or null
   float eps;
+  const unsigned long long* stage_word;  // host rows staged by the side stream: read
+  unsigned long long stage_seq;          // once *stage_word >= stage_seq (or null)
 };
 
 // Sum of squares of eight bf16 values, in fp32.
@@ -55,6 +57,17 @@ __global__ void __launch_bounds__(kGatherThreads)
     gather_rows_kernel(const GatherParams p) {
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
   grid_dependency_wait();  // the previous step's merge wrote list, row_of and d_M
+  if (p.stage_word) {
+    // The side stream's copy of the rows: one thread waits (bounded) for its
+    // word; on giving up the error word is set and the step's results are
+    // not to be used (the host reads the error with them).
+    __shared__ volatile int s_abort;
+    if (threadIdx.x == 0) {
+      s_abort = 0;
+      wait_word_ge(p.stage_word, p.stage_seq, &s_abort, p.err, kErrWaitRows);
+    }
+    __syncthreads();
+  }
   const int M = p.first ? p.BP : *p.d_M;
   if (p.first) {
     for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < p.BP; i += gridDim.x * blockDim.x) {

@@ -440,8 +440,9 @@ def test_teacher_forced_random_states():
 @pytest.mark.parametrize("shape,host", [("toy", "pinned"), ("toy", "pageable"),
                                         ("multi", "pinned"), ("multi", "pageable")])
 def test_host_hidden_and_host_weight_match_device(shape, host):
-    # Host inputs: copied in the call (single-kernel steps, or pageable memory)
-    # or, for multi-kernel steps on page-locked memory, read in place by the gather.
+    # Host inputs: copied on the context's side stream into alternating device
+    # buffers (page-locked or pageable memory, single- or multi-kernel steps);
+    # a host W is copied once at init.
     wl = synth.WORKLOADS["toy"]
     if shape == "multi":
         wl = _wl("toy", B=5, P=64, gen_len=128)
@@ -479,15 +480,20 @@ def test_host_hidden_and_host_weight_match_device(shape, host):
         cai.cai_free(b)
 
 
-@pytest.mark.parametrize("B,host", [(1, "pinned"), (2, "pinned"), (2, "pageable"),
-                                    (5, "pinned")])
-def test_host_rows_pipelined_match_device(B, host):
+@pytest.mark.parametrize("B,host,mode", [(1, "pinned", ""), (2, "pinned", ""),
+                                         (2, "pageable", ""), (5, "pinned", ""),
+                                         (5, "pageable", ""), (5, "pinned", "norm"),
+                                         (5, "pinned", "diag"), (2, "pinned", "norm")])
+def test_host_rows_pipelined_match_device(B, host, mode):
     # Whole trajectories issued back to back with no synchronisation between
     # steps (a one-step-behind poll only), every step reading a different host
-    # buffer: single-kernel steps copy on the context's side stream into two
-    # alternating buffers while the previous step runs, multi-kernel steps
-    # (B = 5) read page-locked rows in place.  The states must equal those of
-    # the same trajectory on device inputs bit for bit.
+    # buffer: the rows are copied on the context's side stream into two
+    # alternating buffers while the previous step runs, and the step's first
+    # reader (the single-kernel LM head, B <= 2, or the gather, B = 5) waits
+    # for the copy on the device; with the final norm in single-kernel steps,
+    # or with the diagnostics' drift kernel, the step's stream waits for it
+    # instead.  The states must equal those of the same trajectory on device
+    # inputs bit for bit.
     P = 16 if B < 5 else 64
     wl = _wl("toy", B=B, P=P, gen_len=4 * P)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
@@ -496,8 +502,15 @@ def test_host_rows_pipelined_match_device(B, host):
     host_in = [[(x.cpu().pin_memory() if host == "pinned" else x.cpu().clone()) for x in row]
                for row in dev_in]
     cfg = cai.cai_config_default(0, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
-    a = cai.cai_init(cfg, W)
-    b = cai.cai_init(cfg, W)
+    if mode == "diag":
+        cfg.flags |= cai.CAI_DIAGNOSTICS
+    if mode == "norm":
+        g = synth.final_norm_weight(wl.H).cuda()
+        a = cai.cai_init_rmsnorm(cfg, W, g, 1e-5)
+        b = cai.cai_init_rmsnorm(cfg, W, g, 1e-5)
+    else:
+        a = cai.cai_init(cfg, W)
+        b = cai.cai_init(cfg, W)
     try:
         for ctx, inp in ((a, dev_in), (b, host_in)):
             for rep in range(2):
@@ -512,8 +525,11 @@ def test_host_rows_pipelined_match_device(B, host):
                         cai.cai_denoise_step(ctx, inp[blk][t])
             torch.cuda.synchronize()
         sa, sb = cai.cai_state_download(a), cai.cai_state_download(b)
-        for k in ("tok", "conf", "cand", "cstep", "exit_reason", "exit_step", "m_hist"):
-            assert np.array_equal(sa[k], sb[k]), k
+        keys = ["tok", "conf", "cand", "cstep", "exit_reason", "exit_step", "m_hist"]
+        if mode == "diag":
+            keys += ["stable", "drift"]
+        for k in keys:
+            assert np.array_equal(sa[k], sb[k], equal_nan=(k == "drift")), k
         assert int(sa["m_hist"].sum()) > 0
         assert cai.cai_test_check_guards(b) == 0
     finally:

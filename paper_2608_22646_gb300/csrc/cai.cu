@@ -620,7 +620,7 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.fused = c->fused ? 1 : 0;
   hp.M_fixed = c->BP;
   hp.max_M = c->use_pair ? c->pair_min_M - 1 : INT_MAX;
-  if (stage_slot >= 0 && c->stage_by_word) {
+  if (c->fused && stage_slot >= 0 && c->stage_by_word) {
     hp.stage_word = c->stage_seq_dev + stage_slot;
     hp.stage_seq = static_cast<unsigned long long>(step_id + 1);
   }
@@ -648,7 +648,7 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
                    hp) != cudaSuccess)
       return check_launch(c);
     c->stats.launches++;
-    if (stage_slot >= 0) {
+    if (c->fused && stage_slot >= 0) {
       // stage2[stage_slot] may be refilled once this step's kernel is done.
       if (cudaEventRecord(c->ev_read[stage_slot], stream) != cudaSuccess)
         return fail(c, CAI_ERR_CUDA);

@@ -483,8 +483,9 @@ def test_host_hidden_and_host_weight_match_device(shape, host):
 @pytest.mark.parametrize("B,host,mode", [(1, "pinned", ""), (2, "pinned", ""),
                                          (2, "pageable", ""), (5, "pinned", ""),
                                          (5, "pageable", ""), (5, "pinned", "norm"),
-                                         (5, "pinned", "diag"), (2, "pinned", "norm")])
-def test_host_rows_pipelined_match_device(B, host, mode):
+                                         (5, "pinned", "diag"), (2, "pinned", "norm"),
+                                         (5, "pinned", "swap0")])
+def test_host_rows_pipelined_match_device(B, host, mode, monkeypatch):
     # Whole trajectories issued back to back with no synchronisation between
     # steps (a one-step-behind poll only), every step reading a different host
     # buffer: the rows are copied on the context's side stream into two
@@ -492,8 +493,11 @@ def test_host_rows_pipelined_match_device(B, host, mode):
     # reader (the single-kernel LM head, B <= 2, or the gather, B = 5) waits
     # for the copy on the device; with the final norm in single-kernel steps,
     # or with the diagnostics' drift kernel, the step's stream waits for it
-    # instead.  The states must equal those of the same trajectory on device
-    # inputs bit for bit.
+    # instead.  swap0: multi-kernel steps also launch the swapped-operand LM
+    # head (CAI_PAIR_SWAP=0), which reads the gathered rows.  The states must
+    # equal those of the same trajectory on device inputs bit for bit.
+    if mode == "swap0":
+        monkeypatch.setenv("CAI_PAIR_SWAP", "0")
     P = 16 if B < 5 else 64
     wl = _wl("toy", B=B, P=P, gen_len=4 * P)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")

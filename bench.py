@@ -454,6 +454,9 @@ def main():
     ap.add_argument("--diagnostics", action="store_true",
                     help="track stability steps and hidden-state drift (CAI_DIAGNOSTICS) and "
                          "summarise them in the line")
+    ap.add_argument("--vocab-shards", type=int, default=0,
+                    help="measure the vocabulary-parallel head over this many shards instead "
+                         "(one per rank under torchrun; all on this GPU otherwise)")
     ap.add_argument("--final-norm", action="store_true",
                     help="the model's final RMSNorm inside the head (cai_init_rmsnorm): inputs "
                          "are the rows before that norm")
@@ -489,6 +492,12 @@ def main():
     cai_build.build()
     dev = torch.device("cuda", local)
     torch.cuda.set_device(dev)
+
+    if args.vocab_shards > 0:
+        run_vocab_shards(cai, args, wl, dist, dev, world, rank)
+        if dist:
+            dist.destroy_process_group()
+        return
 
     head = measure(cai, wl, args.generator, args, dist, dev, args.steps, args.warmup,
                    cpu_leg=(rank == 0 and world == 1 and not args.no_cpu_baseline))
@@ -569,6 +578,125 @@ def e2e_run(cai, ctx, hs, wl, steps, dist, dev):
             "timing": "host wall clock around whole generations, pinned host inputs (each step "
                       "call's rows copied on the context's side stream while the previous step "
                       "runs)"}
+
+
+def run_vocab_shards(cai, args, wl, dist, dev, world, rank):
+    """``--vocab-shards G``: the vocabulary-parallel head on the workload.  With
+    G ranks under torchrun each rank holds one slice of W (one shard context)
+    and a step is the shard's LM head, an NCCL all-gather of the triples and
+    the merge + commit on every rank.  On one GPU the G shard contexts run one
+    after another in one stream and the exchange is a device-side stack: the
+    line then reports each shard's own LM-head time per launch (what a rank
+    holding that shard spends) and the merge + commit time, not a multi-GPU
+    throughput.  Prints one JSON line."""
+    import torch
+    import synth
+    from paper_2608_22646_gb300.shard import exchange_triples, vocab_slices
+    G = args.vocab_shards
+    if dist and world != G:
+        raise SystemExit(f"--vocab-shards {G} under torchrun needs {G} ranks, not {world}")
+    W = synth.lm_head_weight(wl.V, wl.H, seed=wl.seed_w, device=dev)
+    hs = synth.HiddenStates(wl, W, args.generator)
+    hidden = [[hs(blk, t) for t in range(wl.T)] for blk in range(wl.n_blocks)]
+    cfg = cai.cai_config_default(cai.CAI_PRESET_LLADA, wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
+    slices = vocab_slices(wl.V, G)
+    mine = [rank] if dist else list(range(G))
+    ctxs = [cai.cai_init_vocab_shard(cfg, W[v0:v0 + n].contiguous(), v0)
+            for v0, n in (slices[k] for k in mine)]
+    del W
+    rows = cai.cai_shard_rows(ctxs[0])
+    bufs = [torch.empty((rows, 4), dtype=torch.float32, device=dev) for _ in ctxs]
+    stream = torch.cuda.current_stream(dev)
+    prof = {"head": [[] for _ in ctxs], "commit": []}
+
+    def step(h, timed):
+        evs = []
+        for k, (c, b) in enumerate(zip(ctxs, bufs)):
+            if timed:
+                e = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+                e[0].record(stream)
+            cai.cai_shard_head(c, h, b)
+            if timed:
+                e[1].record(stream)
+                evs.append(("head", k, e))
+        gathered = exchange_triples(bufs[0]) if dist else torch.stack(bufs)
+        if timed:
+            e = (torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True))
+            e[0].record(stream)
+        for c in ctxs:
+            cai.cai_shard_commit(c, gathered)
+        if timed:
+            e[1].record(stream)
+            evs.append(("commit", 0, e))
+        return evs
+
+    def generation(timed=False):
+        evs = []
+        for c in ctxs:
+            cai.cai_reset(c)
+        for blk in range(wl.n_blocks):
+            if blk:
+                for c in ctxs:
+                    cai.cai_block_advance(c)
+            evs += step(hidden[blk][0], timed)
+            for t in range(1, wl.T):
+                if t >= 2 and cai.cai_poll(ctxs[0], 1, 60000):
+                    break
+                evs += step(hidden[blk][t], timed)
+        return evs
+
+    for _ in range(args.warmup):
+        generation()
+    torch.cuda.synchronize()
+    st0 = cai.cai_state_download(ctxs[0])
+    for c in ctxs[1:]:
+        assert np.array_equal(cai.cai_state_download(c)["tok"], st0["tok"]), "shards disagree"
+    ev0, ev1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    local = dev.index or 0
+    with Clocks(local) as clk:
+        if dist:
+            dist.barrier()
+        torch.cuda.synchronize()
+        ev0.record(stream)
+        for _ in range(args.steps):
+            generation()
+        ev1.record(stream)
+        torch.cuda.synchronize()
+        if dist:
+            dist.barrier()
+    ms = ev0.elapsed_time(ev1)
+    positions = int(cai.cai_state_download(ctxs[0])["m_hist"].sum()) * args.steps
+    if dist:
+        ms, _ = aggregate(ms, 0, dist, dev)   # every rank decodes the same positions
+    evs = generation(timed=True)
+    torch.cuda.synchronize()
+    for kind, k, (a, b) in evs:
+        (prof["head"][k] if kind == "head" else prof["commit"]).append(a.elapsed_time(b))
+    n_calls = len(prof["commit"])
+    head_us = [round(1e3 * sum(x) / max(1, len(x)), 2) for x in prof["head"]]
+    line = {
+        "metric": "masked positions decoded/s, vocabulary-parallel head (fused head + commit)",
+        "value": round(positions / (ms / 1e3), 1), "unit": UNIT, "n_gpus": world,
+        "steps": args.steps, "warmup": args.warmup, "higher_is_better": True,
+        "vocab_shards": G,
+        "mode": ("one shard per GPU, NCCL all-gather of the triples" if dist else
+                 "one GPU: the shards run one after another in one stream, the exchange is a "
+                 "device-side stack (value = all shards' work on this GPU)"),
+        "ms_per_generation": round(ms / args.steps, 4),
+        "step_calls_per_generation": n_calls,
+        "shard_rows": [n for _, n in slices],
+        "per_shard_head_us": head_us if not dist else head_us[:1],
+        "merge_commit_us_per_step": round(1e3 * sum(prof["commit"]) / max(1, n_calls), 2),
+        "exchange_bytes_per_step": rows * 16 * G,
+        "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": f"{wl.name}: B={wl.B} H={wl.H} V={wl.V} gen_len={wl.gen_len} "
+                               f"block={wl.P} T={wl.T}", "hidden_generator": args.generator},
+        "clocks": clk.summary(),
+    }
+    for c in ctxs:
+        cai.cai_free(c)
+    if rank == 0:
+        print(json.dumps(line), flush=True)
 
 
 def run_reference(args, wl):

@@ -71,6 +71,7 @@ constexpr int kPairStageBytes = 2 * kPairHalfBytes;          // A half + B half
 constexpr int kPairTmemCols = 2 * kPairTileVocab;            // two accumulators
 constexpr int kSwapColStep = 32;    // swapped orientation: granularity of N
 constexpr int kSwapXchBytes = 2 * 4 * kPairTileVocab * 16;  // cross-warp exchange, two buffers
+constexpr int kPairMaxRing = 12;    // swapped stages are cut to size: up to this many
 
 // Tensor maps of the gathered rows with boxes of 16, 32, ..., 128 rows
 // (swapped orientation: a CTA's N / 2 rows of a tile, a multiple of 16, load
@@ -124,7 +125,7 @@ __host__ __device__ inline int pair_partials_per_row(int M, int n_pairs, bool sw
 
 __host__ __device__ inline size_t pair_smem_bytes(int n_stages, bool swap) {
   return 1024 + static_cast<size_t>(n_stages) * kPairStageBytes + (swap ? kSwapXchBytes : 0) +
-         static_cast<size_t>(2 * n_stages + 7) * 8 + 16;
+         static_cast<size_t>(2 * kPairMaxRing + 7) * 8 + 16;
 }
 
 // Pack W [V, H] (row-major bf16) tile-major for the pair kernel: 128-row
@@ -154,10 +155,10 @@ __global__ void pack_w_tiles_kernel(const uint4* __restrict__ W, uint4* __restri
 }
 
 struct PairSmem {
-  uint8_t* stage;      // n_stages x (A half, B half)
+  uint8_t* stage;      // n_stages x kPairStageBytes: the ring (A half, B half per stage)
   float4* xch;         // swapped orientation: 2 x [4 warps][256 columns] triples
-  uint64_t* full;      // n_stages (even CTA): both CTAs' halves of the stage landed
-  uint64_t* empty;     // n_stages: the pair's MMAs are done with the stage
+  uint64_t* full;      // kPairMaxRing (even CTA): both CTAs' halves of the stage landed
+  uint64_t* empty;     // kPairMaxRing: the pair's MMAs are done with the stage
   uint64_t* accf;      // 2: accumulator ready
   uint64_t* acce;      // 2 (even CTA): accumulator drained by both epilogues
   uint64_t* drain;     // 1 (even CTA): abort path, issued MMAs complete
@@ -175,8 +176,8 @@ __device__ __forceinline__ PairSmem pair_carve(uint8_t* raw, int n_stages, bool 
   s.xch = reinterpret_cast<float4*>(after);
   if (swap) after += kSwapXchBytes;
   s.full = reinterpret_cast<uint64_t*>(after);
-  s.empty = s.full + n_stages;
-  s.accf = s.empty + n_stages;
+  s.empty = s.full + kPairMaxRing;
+  s.accf = s.empty + kPairMaxRing;
   s.acce = s.accf + 2;
   s.drain = s.acce + 2;
   s.xchb = s.drain + 1;
@@ -239,9 +240,16 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   const int rt_rows = swap ? swap_tile_cols(M, n_rt) : kPairTileRows;
   const int n_tiles = p.n_vt * n_rt;
   const int my_tiles = pair < n_tiles ? (n_tiles - pair + n_pairs - 1) / n_pairs : 0;
+  // Swapped stages hold the W half and one box of rows_tile / 2 rows, so the
+  // ring (n_stages slots of kPairStageBytes) is re-cut to that size: more
+  // stages in flight for narrower tiles.
+  const int stage_stride =
+      swap ? kPairHalfBytes + (rt_rows / 2) * kPairBlockK * 2 : kPairStageBytes;
+  const int n_ring = swap ? min(kPairMaxRing, p.n_stages * kPairStageBytes / stage_stride)
+                          : p.n_stages;
 
   if (threadIdx.x == 0) {
-    for (int s = 0; s < p.n_stages; ++s) {
+    for (int s = 0; s < n_ring; ++s) {
       mbar_init(&sm.full[s], 1);
       mbar_init(&sm.empty[s], 1);
     }
@@ -300,7 +308,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             ok = false;
             break;
           }
-          uint8_t* dst = sm.stage + static_cast<size_t>(r.slot) * kPairStageBytes;
+          uint8_t* dst = sm.stage + static_cast<size_t>(r.slot) * stage_stride;
           const uint32_t bar = full0 + static_cast<uint32_t>(r.slot * 8);
           // The even CTA arms the stage for the bytes of both CTAs; a copy of
           // the odd CTA that completes first leaves the phase open until then.
@@ -314,13 +322,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             tma_load_2d_pair_nohint(dst + kPairHalfBytes, &tm_w, bar, 0, (w_box + kb) * kPairHalf);
           }
           ++issued;
-          r.next(p.n_stages);
+          r.next(n_ring);
         }
       }
       if (!ok && rank == 0) {
-        const long long f0 = issued > p.n_stages ? issued - p.n_stages : 0;
+        const long long f0 = issued > n_ring ? issued - n_ring : 0;
         for (long long q = f0; q < issued; ++q)
-          pair_drain(&sm.full[q % p.n_stages], static_cast<uint32_t>((q / p.n_stages) & 1), p.err);
+          pair_drain(&sm.full[q % n_ring], static_cast<uint32_t>((q / n_ring) & 1), p.err);
       }
     }
     __syncwarp();
@@ -348,14 +356,14 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
             break;
           }
           tc_fence_after();
-          const uint32_t a_addr = smem_addr(sm.stage + static_cast<size_t>(r.slot) * kPairStageBytes);
+          const uint32_t a_addr = smem_addr(sm.stage + static_cast<size_t>(r.slot) * stage_stride);
           const uint32_t b_addr = a_addr + kPairHalfBytes;
 #pragma unroll
           for (int kk = 0; kk < kPairBlockK / 16; ++kk)
             mma_bf16_pair(d_tmem, sdesc_k_sw128(a_addr + kk * 32), sdesc_k_sw128(b_addr + kk * 32),
                           idesc, (kb | kk) != 0 ? 1u : 0u);
           mma_commit_pair(&sm.empty[r.slot], 0x3);
-          r.next(p.n_stages);
+          r.next(n_ring);
         }
         if (!ok) break;
         mma_commit_pair(&sm.accf[acc], 0x3);

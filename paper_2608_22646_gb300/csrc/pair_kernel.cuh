@@ -242,11 +242,13 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
   const int my_tiles = pair < n_tiles ? (n_tiles - pair + n_pairs - 1) / n_pairs : 0;
   // Swapped stages hold the W half and one box of rows_tile / 2 rows, so the
   // ring (n_stages slots of kPairStageBytes) is re-cut to that size: more
-  // stages in flight for narrower tiles.
+  // stages in flight for narrower tiles.  Unswapped steps do not use the
+  // swapped epilogue's exchange buffer, which follows the ring: one more stage.
   const int stage_stride =
       swap ? kPairHalfBytes + (rt_rows / 2) * kPairBlockK * 2 : kPairStageBytes;
-  const int n_ring = swap ? min(kPairMaxRing, p.n_stages * kPairStageBytes / stage_stride)
-                          : p.n_stages;
+  const int ring_bytes =
+      p.n_stages * kPairStageBytes + (!swap && p.swap_max_n > 0 ? kSwapXchBytes : 0);
+  const int n_ring = min(kPairMaxRing, ring_bytes / stage_stride);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < n_ring; ++s) {

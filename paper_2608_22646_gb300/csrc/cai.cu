@@ -227,6 +227,11 @@ struct cai_ctx {
   void (*head_kernel)(CUtensorMap, HeadParams) = nullptr;
   void (*pair_kernel)(CUtensorMap, CUtensorMap, PairRowMaps, PairParams) = nullptr;
   int pair_min_M = 0, pair_grid = 0, pair_stages = 0, n_vt = 0, reduce_grid = 0;
+  // Most pair stages in flight: swapped stages cut to size would give up to
+  // 10 for narrow tiles, but beyond 8 the narrowest steps slow down again
+  // (measured at fixed M, long-Dream shape: M = 30 160.8 us at 8, 165 at 10).
+  // CAI_PAIR_RING_MAX overrides (2..12; tuning knob).
+  int pair_ring_max = 8;
   size_t pair_smem = 0;
   CUtensorMap tm_h{};    // compact gathered rows (multi-kernel step)
   CUtensorMap tm_hid{};  // the caller's rows (single-kernel step), for hid_mapped
@@ -466,6 +471,7 @@ int launch_pair_head(cai_ctx* c, int t, cudaStream_t stream) {
   pp.swap_max_n = c->swap_max_n;
   pp.n_stages = c->pair_stages;
   pp.inv_r = c->inv_r;
+  pp.ring_max = c->pair_ring_max;
   if (launch_pdl(c->pdl, c->pair_kernel, c->pair_grid, kPairThreads, c->pair_smem, stream,
                  c->tm_a, c->tm_w, c->tm_rows, pp) != cudaSuccess)
     return check_launch(c);
@@ -895,6 +901,8 @@ int init_impl(const cai_config* cfg_in, const void* W, const void* g, double eps
     while (ps > 2 && pair_smem_bytes(ps, c->swap_max_n > 0) > plimit) --ps;
     c->pair_stages = ps;
     c->pair_smem = pair_smem_bytes(ps, c->swap_max_n > 0);
+    const int rmax = env_int("CAI_PAIR_RING_MAX");
+    if (rmax >= 2 && rmax <= kPairMaxRing) c->pair_ring_max = rmax;
     int clusters = 0;
     if (cudaFuncSetAttribute(c->pair_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize,
                              static_cast<int>(c->pair_smem)) != cudaSuccess) {

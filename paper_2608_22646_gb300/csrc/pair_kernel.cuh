@@ -93,6 +93,7 @@ struct PairParams {
   int swap_max_n;      // steps whose swapped tile width is at most this run swapped
   int n_stages;
   const float* inv_r;  // final-norm row scales [rows] (kNorm only)
+  int ring_max;        // most stages in flight (<= kPairMaxRing)
 };
 
 // Row tiles of a pair step with M rows (both orientations).
@@ -248,7 +249,7 @@ __global__ void __cluster_dims__(2, 1, 1) __launch_bounds__(kPairThreads, 1)
       swap ? kPairHalfBytes + (rt_rows / 2) * kPairBlockK * 2 : kPairStageBytes;
   const int ring_bytes =
       p.n_stages * kPairStageBytes + (!swap && p.swap_max_n > 0 ? kSwapXchBytes : 0);
-  const int n_ring = min(kPairMaxRing, ring_bytes / stage_stride);
+  const int n_ring = min(p.ring_max, ring_bytes / stage_stride);
 
   if (threadIdx.x == 0) {
     for (int s = 0; s < n_ring; ++s) {

@@ -367,6 +367,24 @@ def test_multi_kernel_edge_shapes(shape):
         cai.cai_free(ctx)
 
 
+@pytest.mark.parametrize("ring_max", ["2", "12"])
+def test_pair_ring_depths(ring_max, monkeypatch):
+    # The pair kernel's ring at its smallest (two stages, every copy waits
+    # for the previous stage's MMAs) and largest depth (swapped stages cut to
+    # size: up to 10 in flight), over steps of both orientations and of one
+    # and two row tiles (B P = 320).
+    monkeypatch.setenv("CAI_PAIR_RING_MAX", ring_max)
+    B, P, H, V, T, nb = 5, 64, 256, 4096, 8, 2
+    wl = synth.Workload("ring", B=B, H=H, V=V, gen_len=P * nb, P=P, T=T, a0="u04")
+    ctx, W = _ctx(B, P, H, V, T, nb, flags=cai.CAI_GATING | cai.CAI_POS_FACTOR)
+    hs = synth.HiddenStates(wl, W, "calibrated", seed=53)
+    try:
+        rep, final = parity.run_checked_trajectory(ctx, W, hs)
+        assert rep.rows >= B * P and int(final["m_hist"].max()) > 256
+    finally:
+        cai.cai_free(ctx)
+
+
 def _random_shapes(n, seed=2608):
     rng = np.random.default_rng(seed)
     out = []

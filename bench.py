@@ -165,15 +165,23 @@ def _traffic_record(workload: str):
 
 
 def run_trajectory(cai, ctx, hidden, wl, lag_poll=True, stream=None):
-    """All blocks of one generation.  ``hidden[blk][t]`` is the step's input."""
-    for blk in range(wl.n_blocks):
-        if blk:
-            cai.cai_block_advance(ctx, stream)
-        cai.cai_first_step(ctx, hidden[blk][0], stream)
-        for t in range(1, wl.T):
-            if lag_poll and t >= 2 and cai.cai_poll(ctx, 1, 60000):
-                break
-            cai.cai_denoise_step(ctx, hidden[blk][t], stream)
+    """All blocks of one generation.  ``hidden[blk][t]`` is the step's input.
+    A kernel's failed bounded wait raises with the device error bits named."""
+    try:
+        for blk in range(wl.n_blocks):
+            if blk:
+                cai.cai_block_advance(ctx, stream)
+            cai.cai_first_step(ctx, hidden[blk][0], stream)
+            for t in range(1, wl.T):
+                if lag_poll and t >= 2 and cai.cai_poll(ctx, 1, 60000):
+                    break
+                cai.cai_denoise_step(ctx, hidden[blk][t], stream)
+    except cai.CaiError as e:
+        if e.status == cai.CAI_ERR_DEVICE:
+            bits = cai.cai_device_error_bits(ctx)
+            names = [n for k, n in enumerate(cai.DEVERR_NAMES) if bits >> k & 1]
+            e.args = (f"{e.args[0]} [device error bits {bits:#x}: {', '.join(names)}]",)
+        raise
 
 
 def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0, norm=None):

@@ -51,7 +51,7 @@
  * Status.  Every int-returning call returns CAI_OK (0) or a negative CAI_ERR_*
  * code; no C++ exception crosses the ABI.  After CAI_ERR_CUDA or
  * CAI_ERR_DEVICE the context is poisoned ("sticky"): every later call except
- * cai_free and cai_strerror returns the same code.
+ * cai_free, cai_strerror and cai_device_error_bits returns the same code.
  */
 #ifndef CAI_H
 #define CAI_H
@@ -356,6 +356,21 @@ int cai_read_tokens(cai_ctx* ctx, int32_t* host_tokens, void* stream);
  * cai_get_stats synchronises the events and reports the sums. */
 int cai_profile(cai_ctx* ctx, int32_t enable);
 int cai_get_stats(cai_ctx* ctx, cai_stats* out);
+
+/* The context's device error word, which kernels set when a bounded wait
+ * gives up (the reason behind CAI_ERR_DEVICE): one bit per kind of wait,
+ * 0 while none has.  A synchronous copy (after the device's work so far);
+ * also answers on a sticky context.  Errors: CAI_ERR_ARG, CAI_ERR_CUDA. */
+#define CAI_DEVERR_WAIT_EMPTY     (1u << 0) /* producer waiting for a free stage          */
+#define CAI_DEVERR_WAIT_FULL      (1u << 1) /* MMA issuer waiting for a loaded stage      */
+#define CAI_DEVERR_WAIT_ACC_FULL  (1u << 2) /* epilogue waiting for an accumulator        */
+#define CAI_DEVERR_WAIT_ACC_EMPTY (1u << 3) /* MMA issuer waiting for a drained accum.    */
+#define CAI_DEVERR_DRAIN          (1u << 4) /* abort path draining copies in flight       */
+#define CAI_DEVERR_BAD_ROW        (1u << 5) /* a masked token had no row in the list      */
+#define CAI_DEVERR_WAIT_EPI       (1u << 6) /* epilogue warps waiting for each other      */
+#define CAI_DEVERR_BOUNDS         (1u << 7) /* debug builds: index or offset out of range */
+#define CAI_DEVERR_WAIT_ROWS      (1u << 8) /* staged host rows did not arrive            */
+int cai_device_error_bits(cai_ctx* ctx, uint32_t* bits);
 
 /* Release everything the context owns.  Synchronises the device first.
  * NULL is a no-op. */

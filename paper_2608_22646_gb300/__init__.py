@@ -55,7 +55,8 @@ EXPORTS = ("cai_config_default", "cai_init", "cai_init_rmsnorm", "cai_first_step
            "cai_test_pair_plan", "cai_test_theta_table", "cai_test_wait_timeout",
            "cai_test_check_guards",
            "cai_head_rows_static", "cai_test_static_wait_timeout",
-           "cai_init_vocab_shard", "cai_shard_rows", "cai_shard_head", "cai_shard_commit")
+           "cai_init_vocab_shard", "cai_shard_rows", "cai_shard_head", "cai_shard_commit",
+           "cai_device_error_bits")
 
 
 class CaiError(RuntimeError):
@@ -120,6 +121,7 @@ def _load():
         "cai_read_tokens": (ctypes.c_int, [vp, vp, vp]),
         "cai_profile": (ctypes.c_int, [vp, i32]),
         "cai_get_stats": (ctypes.c_int, [vp, ctypes.POINTER(cai_stats)]),
+        "cai_device_error_bits": (ctypes.c_int, [vp, ctypes.POINTER(ctypes.c_uint32)]),
         "cai_free": (None, [vp]),
         "cai_strerror": (ctypes.c_char_p, [ctypes.c_int]),
         "cai_test_fail_alloc_after": (ctypes.c_int, [i32]),
@@ -367,6 +369,18 @@ def cai_get_stats(ctx: Ctx) -> dict:
     s = cai_stats()
     _check(lib().cai_get_stats(ctx.handle, ctypes.byref(s)), "cai_get_stats")
     return {n: getattr(s, n) for n, _ in cai_stats._fields_}
+
+
+DEVERR_NAMES = ("wait_empty", "wait_full", "wait_acc_full", "wait_acc_empty", "drain", "bad_row",
+                "wait_epi", "bounds", "wait_rows")
+
+
+def cai_device_error_bits(ctx: Ctx) -> int:
+    """The context's device error word (bit k: DEVERR_NAMES[k]); works on a
+    context that returned CAI_ERR_DEVICE."""
+    v = ctypes.c_uint32(0)
+    _check(lib().cai_device_error_bits(ctx.handle, ctypes.byref(v)), "cai_device_error_bits")
+    return int(v.value)
 
 
 def cai_free(ctx: Ctx) -> None:

@@ -252,10 +252,11 @@ struct cai_ctx {
   // stage_seq_dev[k]; the step's first kernel that reads the rows (the
   // single-kernel LM head, or the gather) waits for that word before reading
   // them, so the step's stream waits for nothing and consecutive steps keep
-  // their programmatic overlap.  Used when no other kernel of the step reads
-  // the rows first (diagnostics; single-kernel steps: the final norm's row
-  // scales) and the driver provides stream memory writes; otherwise the
-  // step's stream waits for ev_copied.
+  // their programmatic overlap.  Used when nothing else of the step reads the
+  // rows (not with the diagnostics' drift kernel, nor with the final norm in
+  // single-kernel steps, whose row scales are computed from the rows outside
+  // the TMA pipeline) and the driver provides stream memory writes;
+  // otherwise the step's stream waits for ev_copied.
   unsigned long long* stage_seq_dev = nullptr;
   bool stage_by_word = false;
   bool fused = false;    // single-kernel step (B P <= 64)
@@ -604,19 +605,8 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
       if (!make_map(&c->tm_hid, hid, c->BP, cfg.H, kBoxRowsB)) return CAI_ERR_ARG;
       c->hid_mapped = hid;
     }
-    if (c->norm) {
-      RmsParams rp{};
-      rp.hidden = static_cast<const __nv_bfloat16*>(hid);
-      rp.inv_r = c->inv_r;
-      rp.rows = c->BP;
-      rp.H = cfg.H;
-      rp.eps = c->norm_eps;
-      const int warps = kGatherThreads / 32;
-      if (launch_pdl(c->pdl, row_rms_kernel, (c->BP + warps - 1) / warps, kGatherThreads, 0,
-                     stream, rp) != cudaSuccess)
-        return check_launch(c);
-      c->stats.launches++;
-    }
+    // With the final norm the LM-head kernel computes the row scales from
+    // the rows itself.
   }
 
   HeadParams hp{};
@@ -644,6 +634,8 @@ int step_impl(cai_ctx* c, const void* hidden, void* stream_v, bool first) {
   hp.gmax = c->gmax;
   hp.tmem_cols = c->tmem_cols;
   hp.inv_r = c->inv_r;
+  hp.hid = static_cast<const __nv_bfloat16*>(hid);
+  hp.norm_eps = c->norm_eps;
   const CommitParams cp = commit_params(c, t, step_id);
   if (c->fused) hp.cp = cp;
   if (c->profiling) cudaEventRecord(ev[1], stream);
@@ -1444,6 +1436,21 @@ int cai_read_tokens(cai_ctx* c, int32_t* host_tokens, void* stream) {
 int cai_profile(cai_ctx* c, int32_t enable) {
   if (!c) return CAI_ERR_ARG;
   c->profiling = enable != 0;
+  return CAI_OK;
+}
+
+int cai_device_error_bits(cai_ctx* c, uint32_t* bits) {
+  if (!c || !bits) return CAI_ERR_ARG;
+  static_assert(CAI_DEVERR_WAIT_EMPTY == kErrWaitEmpty && CAI_DEVERR_WAIT_FULL == kErrWaitFull &&
+                    CAI_DEVERR_WAIT_ACC_FULL == kErrWaitAccFull &&
+                    CAI_DEVERR_WAIT_ACC_EMPTY == kErrWaitAccEmpty && CAI_DEVERR_DRAIN == kErrDrain &&
+                    CAI_DEVERR_BAD_ROW == kErrBadRow && CAI_DEVERR_WAIT_EPI == kErrWaitEpi &&
+                    CAI_DEVERR_BOUNDS == kErrBounds && CAI_DEVERR_WAIT_ROWS == kErrWaitRows,
+                "error bits of the header and the kernels");
+  if (cudaMemcpy(bits, c->err, sizeof(uint32_t), cudaMemcpyDeviceToHost) != cudaSuccess) {
+    cudaGetLastError();
+    return CAI_ERR_CUDA;
+  }
   return CAI_OK;
 }
 

@@ -93,6 +93,8 @@ struct HeadParams {
   int gmax;            // largest tile group
   int tmem_cols;       // allocated tensor-memory columns (>= 2 gmax slot_cols)
   const float* inv_r;  // final-norm row scales 1 / sqrt(mean h^2 + eps) [rows] (kNorm only)
+  const __nv_bfloat16* hid;  // single-kernel step, kNorm: the step's rows [M_fixed, H], from
+  float norm_eps;            // which the kernel computes the row scales itself (and epsilon)
   CommitParams cp;     // commit rule, run by the last CTA of a single-kernel step
 };
 
@@ -315,8 +317,9 @@ __device__ __forceinline__ void fused_step_commit(const CommitParams& cp, uint8_
 // ---------------------------------------------------------------- kernel --
 
 // kNorm: the model's final RMSNorm is part of the head.  Its weight is
-// already folded into W; row n's logits are scaled by inv_r[n] (written by
-// the previous kernel in the stream: row_rms_kernel or the gather).
+// already folded into W; row n's logits are scaled by 1 / sqrt(mean h^2 +
+// eps) of the row: computed by the epilogue warps from the caller's rows in a
+// single-kernel step, inv_r[n] (written by the gather) in a multi-kernel one.
 template <bool kNorm>
 __global__ void __launch_bounds__(kHeadThreads, 1)
     lm_head_softmax_kernel(const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
@@ -553,6 +556,17 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     const int ew = warp - 2;       // 0..3: slot in the cross-warp merge
     const int quarter = warp & 3;  // tensor-memory lanes this warp may read
     const uint32_t lane_base = static_cast<uint32_t>(quarter * 32) << 16;
+    // Final-norm row scales: a single-kernel step computes them from the
+    // caller's rows (nothing then waits on an earlier kernel); a multi-kernel
+    // step reads the gather's.
+    const float* scale = p.inv_r;
+    if constexpr (kNorm) {
+      __shared__ float s_scale[kChunkN];
+      if (p.fused) {
+        epilogue_row_scales(p.hid, M, p.H, p.norm_eps, s_scale, ew, lane);
+        scale = s_scale;
+      }
+    }
     Ring racc;
     bool ok = true;
     for (int q = 0; q < n_chunks && ok; ++q) {
@@ -593,11 +607,9 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
 #pragma unroll
           for (int c = 0; c < 32; ++c) sc[c] = kLog2e;
           if constexpr (kNorm) {
-            // The row scales come from the previous kernel in the stream.
-            if (p.fused) grid_dependency_wait();
 #pragma unroll
             for (int c = 0; c < 32; ++c)
-              if (n0 + c < M) sc[c] = kLog2e * __ldg(p.inv_r + n0 + c);
+              if (n0 + c < M) sc[c] = kLog2e * scale[n0 + c];
           }
           const uint32_t tgroup =
               tmem_base + lane_base + static_cast<uint32_t>(racc.slot * group_cols);
@@ -653,9 +665,7 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
                 float m, s;
                 int i;
                 if constexpr (kNorm) {
-                  if (p.fused && g == 0 && t == pl.group_first(g) && c == 0)
-                    grid_dependency_wait();  // row scales from the previous kernel
-                  transpose_reduce32(v, valid, vrow, lane, m, s, i, p.inv_r + n0 + 32 * c);
+                  transpose_reduce32(v, valid, vrow, lane, m, s, i, scale + n0 + 32 * c);
                 } else {
                   transpose_reduce32(v, valid, vrow, lane, m, s, i);
                 }

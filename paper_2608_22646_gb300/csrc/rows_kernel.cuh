@@ -177,9 +177,9 @@ __global__ void pack_weight_rows_kernel(const uint4* __restrict__ W, uint4* __re
 
 // Single-kernel step only (p.fused = 1, p.M_fixed <= 128), W packed by
 // pack_weight_rows_kernel.  p.n_stages is the W ring depth (32 KiB stages),
-// p.n_bslots the rows ring depth (stages rows_h_stride(M) apart).  kNorm: row r's logits are
-// scaled by inv_r[r] (written by row_rms_kernel, the previous kernel in the
-// stream).
+// p.n_bslots the rows ring depth (stages rows_h_stride(M) apart).  kNorm: row
+// r's logits are scaled by 1 / sqrt(mean h^2 + eps) of the row, which the
+// epilogue warps compute from the step's rows (p.hid).
 template <bool kNorm>
 __global__ void __launch_bounds__(kHeadThreads, 1)
     lm_head_rows_kernel(const __grid_constant__ CUtensorMap tm_h, const HeadParams p) {
@@ -371,8 +371,12 @@ __global__ void __launch_bounds__(kHeadThreads, 1)
     int ix = INT_MAX;
     float rs = kLog2e;
     if constexpr (kNorm) {
-      grid_dependency_wait();  // the row scales come from the previous kernel
-      if (row < M) rs = kLog2e * __ldg(p.inv_r + row);
+      // The final RMSNorm's row scales, from the step's rows while the first
+      // group accumulates.  Nothing here depends on an earlier kernel, so the
+      // accumulators are drained as in a step without the norm.
+      __shared__ float s_scale[kRowsM];
+      epilogue_row_scales(p.hid, M, p.H, p.norm_eps, s_scale, warp - 2, lane);
+      if (row < M) rs = kLog2e * s_scale[row];
     }
     Ring racc;
     bool ok = true;

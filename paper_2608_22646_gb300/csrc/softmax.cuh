@@ -7,11 +7,54 @@
 
 #include <climits>
 #include <cstdint>
+#include <cuda_bf16.h>
 
 namespace cai {
 
 constexpr float kLog2e = 1.4426950408889634f;
 constexpr float kNegBig = -3.0e38f;  // "no logit yet": exp2(x - m) underflows to 0
+
+// Sum of squares of eight bf16 values, in fp32 (the final RMSNorm's row
+// statistic).
+__device__ __forceinline__ float sumsq8(uint4 x) {
+  const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&x);
+  float s = 0.0f;
+#pragma unroll
+  for (int i = 0; i < 8; ++i) {
+    const float f = __bfloat162float(e[i]);
+    s = fmaf(f, f, s);
+  }
+  return s;
+}
+
+// Final RMSNorm row scales 1 / sqrt(mean h^2 + eps) of rows [0, M) of the
+// [M, H] bf16 rows `hid` into s_scale (shared memory), by the four epilogue
+// warps of an LM-head kernel (ew = 0..3, each a whole warp; every one must
+// call it), which then meet at named barrier 1: a row at a time per warp, 32
+// lanes with eight 16-byte loads each in flight.
+__device__ __forceinline__ void epilogue_row_scales(const __nv_bfloat16* hid, int M, int H,
+                                                    float eps, float* s_scale, int ew,
+                                                    int lane) {
+  const int nvec = H / 8;
+  for (int r = ew; r < M; r += 4) {
+    const uint4* src = reinterpret_cast<const uint4*>(hid + static_cast<size_t>(r) * H);
+    float ss = 0.0f;
+    for (int v0 = lane; v0 < nvec; v0 += 32 * 8) {
+      uint4 x[8];
+#pragma unroll
+      for (int j = 0; j < 8; ++j) {
+        const int v = v0 + 32 * j;
+        x[j] = v < nvec ? __ldg(src + v) : make_uint4(0u, 0u, 0u, 0u);
+      }
+#pragma unroll
+      for (int j = 0; j < 8; ++j) ss += sumsq8(x[j]);
+    }
+#pragma unroll
+    for (int off = 16; off >= 1; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
+    if (lane == 0) s_scale[r] = rsqrtf(ss / static_cast<float>(H) + eps);
+  }
+  asm volatile("bar.sync 1, 128;" ::: "memory");  // the four epilogue warps
+}
 
 __device__ __forceinline__ float fast_exp2(float x) {
   float y;
@@ -116,7 +159,8 @@ __device__ __forceinline__ void transpose_logits32(float (&z)[32], bool valid, b
 // 32 rows (one per lane) x 32 columns of logits -> lane l holds the
 // (max, sum, argmax) of column l over the 32 rows.  Column c's logits are
 // scaled by log2 e, times col_scale[c] when given (a per-row normalisation
-// of the decoded hidden states, see lm_head_softmax_kernel).
+// of the decoded hidden states, see lm_head_softmax_kernel; global or shared
+// memory).
 __device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool valid, int vrow,
                                                    int lane, float& om, float& os, int& oi,
                                                    const float* col_scale = nullptr) {
@@ -124,7 +168,7 @@ __device__ __forceinline__ void transpose_reduce32(const uint32_t (&v)[32], bool
   int ix[32];
 #pragma unroll
   for (int c = 0; c < 32; ++c) {
-    const float sc = col_scale ? kLog2e * __ldg(col_scale + c) : kLog2e;
+    const float sc = col_scale ? kLog2e * col_scale[c] : kLog2e;
     m[c] = valid ? __uint_as_float(v[c]) * sc : kNegBig;
     s[c] = valid ? 1.0f : 0.0f;
     ix[c] = valid ? vrow : INT_MAX;

@@ -41,18 +41,6 @@ struct GatherParams {
   unsigned long long stage_seq;          // once *stage_word >= stage_seq (or null)
 };
 
-// Sum of squares of eight bf16 values, in fp32.
-__device__ __forceinline__ float sumsq8(uint4 x) {
-  const __nv_bfloat16* e = reinterpret_cast<const __nv_bfloat16*>(&x);
-  float s = 0.0f;
-#pragma unroll
-  for (int i = 0; i < 8; ++i) {
-    const float f = __bfloat162float(e[i]);
-    s = fmaf(f, f, s);
-  }
-  return s;
-}
-
 __global__ void __launch_bounds__(kGatherThreads)
     gather_rows_kernel(const GatherParams p) {
   grid_launch_dependents();  // every thread: the CTA counts once all of them have
@@ -179,32 +167,6 @@ __global__ void __launch_bounds__(kGatherThreads) drift_kernel(const DriftParams
     for (int w = 0; w < nw; ++w) tot += s_sum[w];
     p.drift[(static_cast<size_t>(b) * p.n_blocks + p.blk) * p.T + p.t] = tot / static_cast<float>(p.P);
   }
-}
-
-// ------------------------------------------------ final-norm row scales --
-
-struct RmsParams {
-  const __nv_bfloat16* hidden;  // [rows, H] the caller's rows (single-kernel step)
-  float* inv_r;                 // [rows] 1 / sqrt(mean h^2 + eps)
-  int rows, H;
-  float eps;
-};
-
-// One warp per row.  Reads only the caller's rows; writes inv_r, which the
-// previous LM-head launch may still read, so it waits for that kernel first.
-__global__ void __launch_bounds__(kGatherThreads) row_rms_kernel(const RmsParams p) {
-  grid_launch_dependents();  // every thread: the CTA counts once all of them have
-  const int row = (blockIdx.x * blockDim.x + threadIdx.x) >> 5;
-  const int lane = threadIdx.x & 31;
-  float ss = 0.0f;
-  if (row < p.rows) {
-    const uint4* src = reinterpret_cast<const uint4*>(p.hidden + static_cast<size_t>(row) * p.H);
-    for (int v = lane; v < p.H / 8; v += 32) ss += sumsq8(__ldg(src + v));
-  }
-#pragma unroll
-  for (int off = 16; off >= 1; off >>= 1) ss += __shfl_xor_sync(0xffffffffu, ss, off);
-  grid_dependency_wait();
-  if (row < p.rows && lane == 0) p.inv_r[row] = rsqrtf(ss / static_cast<float>(p.H) + p.eps);
 }
 
 // ------------------------------------------------- bounded-wait test hook --

@@ -127,10 +127,17 @@ def test_fixed_threshold_rule(theta):
             cai.cai_free(ctx)
 
 
-@pytest.mark.parametrize("B,P,gen", [(2, 16, 64), (5, 64, 128)])
-def test_rmsnorm_in_head(B, P, gen):
-    # Final RMSNorm folded into the head, on a single-kernel context (B P = 32)
-    # and a multi-kernel one (B P = 320: gather scales, pair and swapped kernels).
+@pytest.mark.parametrize("B,P,gen,env", [
+    (2, 16, 64, {}), (5, 64, 128, {}), (2, 16, 64, {"CAI_ROWS_HEAD": "0"}),
+    (4, 64, 128, {"CAI_FUSED_MAX_BP": "256"}), (5, 64, 128, {"CAI_PAIR_SWAP": "0"})])
+def test_rmsnorm_in_head(B, P, gen, env, monkeypatch):
+    # Final RMSNorm folded into the head: single-kernel contexts (B P = 32 on
+    # the rows-operand kernel, and on the swapped-operand one; B P = 256 on the
+    # swapped-operand one), whose LM head computes the row scales itself, and
+    # multi-kernel ones (B P = 320: the gather's scales, pair kernel; with
+    # CAI_PAIR_SWAP=0 the swapped-operand kernel takes the narrow steps).
+    for k, v in env.items():
+        monkeypatch.setenv(k, v)
     wl = _wl("toy", B=B, P=P, a0="bimodal", gen_len=gen)
     W = synth.lm_head_weight(wl.V, wl.H, device="cuda")
     g = synth.final_norm_weight(wl.H, seed=9, device="cuda")
@@ -563,8 +570,9 @@ def test_device_wait_timeout_reports_and_device_stays_usable():
     # A kernel waits, through the step kernels' bounded barrier wait, on a
     # barrier nothing arrives at: after the limit it records the failure in
     # the context's error word and returns.  The host then reads
-    # CAI_ERR_DEVICE, the context stays sticky, and a new context on the same
-    # GPU runs a checked trajectory.
+    # CAI_ERR_DEVICE, the context stays sticky (its device error word names
+    # the wait that gave up), and a new context on the same GPU runs a checked
+    # trajectory.
     import time
     wl = synth.WORKLOADS["toy"]
     ctx, W = _ctx(wl.B, wl.P, wl.H, wl.V, wl.T, wl.n_blocks)
@@ -577,9 +585,11 @@ def test_device_wait_timeout_reports_and_device_stays_usable():
         cai.cai_test_wait_timeout(ctx)
         torch.cuda.synchronize()
         assert 1.5 < time.perf_counter() - t0 < 30.0     # the wait ran to its limit
+        assert cai.cai_device_error_bits(ctx) == (1 << cai.DEVERR_NAMES.index("wait_full"))
         with pytest.raises(cai.CaiError) as e:
             cai.cai_state_download(ctx)
         assert e.value.status == cai.CAI_ERR_DEVICE
+        assert cai.cai_device_error_bits(ctx) == (1 << cai.DEVERR_NAMES.index("wait_full"))
         with pytest.raises(cai.CaiError) as e:
             cai.cai_denoise_step(ctx, hs(0, 1))
         assert e.value.status == cai.CAI_ERR_DEVICE

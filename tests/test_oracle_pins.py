@@ -31,7 +31,6 @@ import os
 import mpmath
 import numpy as np
 import pytest
-import torch
 
 import oracle
 import synth

@@ -214,11 +214,14 @@ def cpu_baseline(wl, W, hs_fn, budget_s: float = 12.0, norm=None):
 
 def _trajectory_summary(st: dict) -> dict:
     """One generation of the workload: steps per block (max over the batch),
-    exits by reason, tokens left unresolved, and the step-zero budgets."""
+    the masked rows M_t decoded at each step of each block, exits by reason,
+    tokens left unresolved, and the step-zero budgets."""
     ex = st["exit_reason"]
     reasons = {"done": 1, "grinding": 2, "t_exhausted": 3}
     bud = st["budget"].reshape(-1)
-    return {"steps_per_block": [int(x) for x in (st["exit_step"].max(axis=0) + 1)],
+    steps = st["exit_step"].max(axis=0) + 1
+    return {"steps_per_block": [int(x) for x in steps],
+            "m_t": [[int(m) for m in st["m_hist"][b, :int(steps[b])]] for b in range(len(steps))],
             "exits": {k: int((ex == v).sum()) for k, v in reasons.items()},
             "unresolved_tokens": int(st["unresolved"].sum()),
             "budgets": {str(b): int((bud == b).sum()) for b in (8, 32, 64)}}
@@ -519,7 +522,6 @@ def main():
     for name in extra:
         wname, gen = EXTRA_WORKLOADS[name]
         r = measure(cai, synth.WORKLOADS[wname], gen, args, dist, dev, args.steps, args.warmup)
-        r.pop("trajectory", None)
         workloads[name] = r
 
     cfg = head["config"]

@@ -52,6 +52,16 @@
 // the even CTA's barrier (cta_group::2 loads), which the even CTA's producer
 // arms with the bytes of both.  Two accumulator buffers let the epilogue of
 // one tile overlap the next tile's MMAs.
+//
+// What bounds a step: reading W from HBM with one row tile; with two or more,
+// the MMAs.  The tensor core runs the MMAs of the one issuing thread one after
+// another, about 63 + 0.085 N ns each (M = 256, K = 16, measured on GB300),
+// so a 160-column tile costs nearly as much per K block as a 256-column one
+// and two row tiles take twice one; each orientation issues the fewest MMAs
+// its M allows (ceil(M / 256) per vocabulary tile and K slice).  A second
+// issuing thread would run MMAs side by side, but two threads accumulating
+// into one accumulator do so in no fixed order, and the fp32 logits (and the
+// commit decisions at a threshold) would then change from run to run.
 #pragma once
 
 #include <climits>
